@@ -1,0 +1,258 @@
+"""Float64 CPU oracle of the SPADE verify step.
+
+TEST INFRASTRUCTURE ONLY.  Nothing on the product path imports this module:
+only the tests, the smoke check and the CPU-baseline leg of the benchmark do.
+It shares no code with the CUDA library and is deliberately plain and slow.
+
+What it computes (the verifier side of one speculative-decoding iteration):
+
+* ``verify_attention`` -- causal attention of the k+1 verify positions of each
+  sequence against its KV cache (the verifier's single forward pass over the
+  draft block, Sec. III-B "Verification Stage" and Algorithm 1, "Cloud: in
+  parallel ... in a single forward pass"; the residual block x_{l+1} = x_l +
+  f_l(x_l) of Sec. III-A contains this attention).
+* ``lm_logits`` -- the LM head o = g(x_L) (Sec. III-A).
+* ``verify_accept`` -- softmax of the logits (Sec. III-A), the acceptance
+  probability alpha(x) = min(1, p(x)/q(x)) and the residual distribution
+  p'(x) = norm(max(0, p(x) - q(x))) (Sec. III-C "Verification Criterion"),
+  the longest accepted prefix and the correction token (Algorithm 1).
+* ``kv_commit`` -- the context update m <- m + k + 1 of Algorithm 1 applied to
+  a KV cache: accepted slots stay, rejected slots are cleared.
+
+Readings taken where the paper is silent (each also listed in the design
+notes): greedy verification accepts a draft iff it equals the verifier's
+argmax (lowest index on ties); the uniform u of position i decides acceptance
+iff u < p/q (q(d) = 0 accepts iff p(d) > 0); when every draft is accepted a
+bonus token is drawn from p of the last row; sampling is the inverse CDF in
+ascending vocabulary order, the first x whose cumulative mass exceeds u*Z; a
+residual with no positive finite mass falls back to p.
+
+Inputs are numpy arrays.  Floating inputs are the exact values of the bf16 /
+fp32 tensors handed to the GPU, converted to float64 before any arithmetic.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+GREEDY = 0
+STOCHASTIC = 1
+
+
+def _f64(x):
+    return np.asarray(x, dtype=np.float64)
+
+
+# ----------------------------------------------------------------------------
+# Attention (Sec. III-B verification stage; Algorithm 1 cloud step)
+# ----------------------------------------------------------------------------
+def attention_row(qv, K, V):
+    """softmax(q K^T / sqrt(D)) V for one query vector over the keys given.
+
+    Returns (o, lse) with lse the natural-log log-sum-exp of the scaled scores.
+    """
+    qv = _f64(qv)
+    K = _f64(K)
+    V = _f64(V)
+    s = K @ qv / math.sqrt(qv.shape[-1])
+    m = s.max()
+    w = np.exp(s - m)
+    den = w.sum()
+    return (w @ V) / den, m + math.log(den)
+
+
+def verify_attention(q, k_cache, v_cache, ctx_lens, n_draft, cu_q, rows=None):
+    """Verify attention of every (row, head), or of the (row, head) pairs in ``rows``.
+
+    q [R, Hq, D]; k_cache, v_cache [B, Hkv, cap, D]; ctx_lens, n_draft [B];
+    cu_q [B+1] with row cu_q[b]+i holding position i (0 <= i <= k_b) of
+    sequence b.  Position i sees keys 0 .. ctx_b + i (the committed context plus
+    the draft block up to itself); query head h reads KV head h // (Hq/Hkv).
+    Returns (out [R, Hq, D], lse [R, Hq]) in float64; with ``rows`` given only
+    those entries are filled (the rest stay NaN).
+    """
+    q = np.asarray(q)
+    R, Hq, D = q.shape
+    B, Hkv = k_cache.shape[0], k_cache.shape[1]
+    G = Hq // Hkv
+    out = np.full((R, Hq, D), np.nan)
+    lse = np.full((R, Hq), np.nan)
+    row_seq = np.empty(R, dtype=np.int64)
+    row_pos = np.empty(R, dtype=np.int64)
+    for b in range(B):
+        for i in range(int(n_draft[b]) + 1):
+            row_seq[cu_q[b] + i] = b
+            row_pos[cu_q[b] + i] = i
+    pairs = rows if rows is not None else [(r, h) for r in range(R) for h in range(Hq)]
+    for r, h in pairs:
+        b = row_seq[r]
+        last = int(ctx_lens[b]) + int(row_pos[r])
+        kvh = h // G
+        o, l = attention_row(q[r, h], k_cache[b, kvh, :last + 1], v_cache[b, kvh, :last + 1])
+        out[r, h] = o
+        lse[r, h] = l
+    return out, lse
+
+
+# ----------------------------------------------------------------------------
+# LM head and softmax (Sec. III-A)
+# ----------------------------------------------------------------------------
+def lm_logits(hidden, w_lm, chunk=8192):
+    """o = g(x_L): logits[r, x] = sum_j hidden[r, j] * W[x, j], float64."""
+    h = _f64(hidden)
+    V = w_lm.shape[0]
+    out = np.empty((h.shape[0], V))
+    for v0 in range(0, V, chunk):
+        out[:, v0:v0 + chunk] = h @ _f64(w_lm[v0:v0 + chunk]).T
+    return out
+
+
+def softmax(logits):
+    """P(y | prefix) = softmax(o) (Sec. III-A), temperature 1."""
+    l = _f64(logits)
+    e = np.exp(l - l.max(axis=-1, keepdims=True))
+    return e / e.sum(axis=-1, keepdims=True)
+
+
+def acceptance_probability(p_x, q_x):
+    """alpha(x) = min(1, p(x)/q(x)) (Sec. III-C)."""
+    if q_x <= 0.0:
+        return 1.0 if p_x > 0.0 else 0.0
+    return min(1.0, p_x / q_x)
+
+
+def residual_distribution(p, q):
+    """p'(x) = norm(max(0, p(x) - q(x))) (Sec. III-C), unnormalised mass and Z.
+
+    Returns (r, Z, fell_back).  If the residual has no positive finite mass,
+    it is replaced by p (reading for float or malformed q).
+    """
+    r = np.maximum(0.0, _f64(p) - _f64(q))
+    Z = r.sum()
+    if not (Z > 0.0 and np.isfinite(Z)):
+        r = _f64(p).copy()
+        return r, r.sum(), True
+    return r, Z, False
+
+
+def inverse_cdf(r, Z, u):
+    """Smallest x with sum_{y<=x} r(y) > u*Z (ascending vocabulary order).
+
+    Returns (x, margin) where margin is the distance of u*Z to the nearer edge
+    of x's CDF interval divided by r(x) (0.5 = dead centre, 0 = on an edge).
+    If rounding leaves u*Z beyond the total, the last x with r > 0 is taken.
+    """
+    c = np.cumsum(r)
+    T = u * Z
+    hit = np.nonzero(c > T)[0]
+    pos = np.nonzero(r > 0)[0]
+    x = int(hit[0]) if hit.size else int(pos[-1])
+    lo = c[x] - r[x]
+    margin = min(T - lo, c[x] - T) / r[x] if r[x] > 0 else 0.0
+    return x, margin
+
+
+def _top2_margin(l):
+    top = np.partition(l, -2)[-2:] if l.shape[0] > 1 else np.array([-np.inf, l[0]])
+    return float(top[1] - top[0])
+
+
+def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
+                  margin=1e-3):
+    """Accept/reject of every sequence, given its verifier logits.
+
+    logits [R, V] (rows as in ``verify_attention``); draft_tokens [R-B] with
+    draft i of sequence b at index cu_q[b] - b + i; draft_probs [R-B, V] (q of
+    the draft model at the same positions, may be None if no sequence is
+    stochastic); uniforms [R]: u[cu_q[b]+i] is the accept test of draft i,
+    u[cu_q[b]+k_b] the sampling uniform; mode [B] 0 greedy / 1 stochastic.
+
+    Returns dict with accepted_len [B], next_token [B] and diagnostics:
+      flag_decision [B]  some decided position has top-2 logit margin (greedy)
+                         or |u - p/q| (stochastic) below ``margin``;
+      flag_sample [B]    the sampled token's u*Z lies within margin*r(x) of an
+                         edge of its CDF interval (stochastic only);
+      fallback [B]       residual had no mass, p used instead.
+    """
+    B = len(n_draft)
+    acc = np.zeros(B, dtype=np.int64)
+    tok = np.zeros(B, dtype=np.int64)
+    flag_dec = np.zeros(B, dtype=bool)
+    flag_smp = np.zeros(B, dtype=bool)
+    fallback = np.zeros(B, dtype=bool)
+    for b in range(B):
+        k = int(n_draft[b])
+        r0 = int(cu_q[b])
+        d0 = r0 - b
+        stochastic = int(mode[b]) == STOCHASTIC
+        a = 0
+        for i in range(k):
+            l = _f64(logits[r0 + i])
+            d = int(draft_tokens[d0 + i])
+            if not stochastic:
+                ok = d == int(np.argmax(l))
+                if _top2_margin(l) < margin:
+                    flag_dec[b] = True
+            else:
+                p = softmax(l)
+                qd = float(draft_probs[d0 + i][d])
+                u = float(uniforms[r0 + i])
+                if qd > 0.0:
+                    ratio = p[d] / qd
+                    ok = u < ratio
+                    if abs(u - ratio) < margin:
+                        flag_dec[b] = True
+                else:
+                    ok = p[d] > 0.0
+            if not ok:
+                break
+            a += 1
+        acc[b] = a
+        lr = _f64(logits[r0 + a])
+        if not stochastic:
+            tok[b] = int(np.argmax(lr))
+            if _top2_margin(lr) < margin:
+                flag_dec[b] = True
+        else:
+            p = softmax(lr)
+            if a < k:
+                r, Z, fb = residual_distribution(p, draft_probs[d0 + a])
+            else:
+                r, Z, fb = p, p.sum(), False
+            fallback[b] = fb
+            x, m = inverse_cdf(r, Z, float(uniforms[r0 + k]))
+            tok[b] = x
+            if m < margin:
+                flag_smp[b] = True
+    return dict(accepted_len=acc, next_token=tok, flag_decision=flag_dec,
+                flag_sample=flag_smp, fallback=fallback)
+
+
+def verify_accept_from_hidden(hidden, w_lm, *args, **kw):
+    """``verify_accept`` on logits computed by ``lm_logits`` (the full step)."""
+    return verify_accept(lm_logits(hidden, w_lm), *args, **kw)
+
+
+# ----------------------------------------------------------------------------
+# KV commit (Algorithm 1 context update)
+# ----------------------------------------------------------------------------
+def kv_commit(k_cache, v_cache, ctx_lens, accepted_len, n_draft):
+    """Append the accepted positions and roll back the rejected ones.
+
+    The verify block of sequence b occupies cache slots ctx_b .. ctx_b + k_b.
+    After acceptance of a_b drafts the committed context is ctx_b + a_b + 1
+    (last accepted token + a_b drafts); slots ctx_b + a_b + 1 .. ctx_b + k_b
+    are cleared to zero.  Returns new (k_cache, v_cache, ctx_lens) copies.
+    """
+    k = np.array(k_cache, copy=True)
+    v = np.array(v_cache, copy=True)
+    ctx = np.array(ctx_lens, dtype=np.int64, copy=True)
+    for b in range(len(ctx)):
+        a = int(accepted_len[b])
+        lo = int(ctx[b]) + a + 1
+        hi = int(ctx[b]) + int(n_draft[b]) + 1
+        k[b, :, lo:hi] = 0
+        v[b, :, lo:hi] = 0
+        ctx[b] = lo
+    return k, v, ctx

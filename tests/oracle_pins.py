@@ -1,0 +1,352 @@
+"""Pins of the float64 oracle against facts fixed by the paper and by mathematics.
+
+Each ``check_*`` takes an oracle module and raises AssertionError when the
+module disagrees with a fact that does not come from the oracle itself:
+hand-derived worked examples, closed forms, a textbook library routine
+(torch's scaled_dot_product_attention in float64), the output-equivalence
+theorem of speculative decoding (Sec. III-B/III-C: greedy SD reproduces plain
+argmax decoding token for token, rejection sampling reproduces p), and the
+invariants of Algorithm 1.  ``test_oracle_pins.py`` runs them on the oracle;
+``test_oracle_mutants.py`` runs them on copies of the oracle with planted
+mistakes and requires that each mistake is caught.
+"""
+from __future__ import annotations
+
+import json
+import math
+import os
+
+import numpy as np
+import torch
+from scipy import stats
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "worked_examples.json")
+
+
+def _golden():
+    with open(GOLDEN) as f:
+        return json.load(f)
+
+
+def _ln(s):
+    return math.log(float(s.split()[1]))
+
+
+# ----------------------------------------------------------------------------
+# Attention
+# ----------------------------------------------------------------------------
+def _single_seq_cache(K, V):
+    K = np.asarray(K, dtype=np.float64)[None, None]
+    V = np.asarray(V, dtype=np.float64)[None, None]
+    return K, V
+
+
+def check_attention_worked_examples(o):
+    for ex in _golden()["attention"]:
+        K, V = _single_seq_cache(ex["K"], ex["V"])
+        q = np.asarray(ex["q"], dtype=np.float64)[:, None, :]
+        out, lse = o.verify_attention(q, K, V, [ex["ctx"]], [ex["k"]], [0, ex["k"] + 1])
+        np.testing.assert_allclose(out[:, 0], np.asarray(ex["out"]), rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lse[:, 0], [_ln(s) for s in ex["lse"]], rtol=0, atol=1e-12)
+
+
+def _random_attention_case(rng, B, Hq, Hkv, D, ctx, kd, extra=3):
+    cap = max(c + k + 1 for c, k in zip(ctx, kd)) + extra
+    cu = np.concatenate([[0], np.cumsum(np.asarray(kd) + 1)])
+    R = int(cu[-1])
+    q = rng.standard_normal((R, Hq, D))
+    kc = rng.standard_normal((B, Hkv, cap, D))
+    vc = rng.standard_normal((B, Hkv, cap, D))
+    return q, kc, vc, cu
+
+
+def _sdpa_reference(q, kc, vc, ctx, kd, cu):
+    """torch SDPA in float64 with an explicit boolean mask and GQA by repeat."""
+    R, Hq, D = q.shape
+    B, Hkv, cap, _ = kc.shape
+    G = Hq // Hkv
+    out = np.zeros((R, Hq, D))
+    for b in range(B):
+        rows = slice(int(cu[b]), int(cu[b + 1]))
+        nq = int(kd[b]) + 1
+        qb = torch.from_numpy(q[rows]).permute(1, 0, 2)              # [Hq, nq, D]
+        kb = torch.from_numpy(kc[b]).repeat_interleave(G, dim=0)     # [Hq, cap, D]
+        vb = torch.from_numpy(vc[b]).repeat_interleave(G, dim=0)
+        mask = torch.zeros((nq, cap), dtype=torch.bool)
+        for i in range(nq):
+            mask[i, : int(ctx[b]) + i + 1] = True
+        ob = torch.nn.functional.scaled_dot_product_attention(qb, kb, vb, attn_mask=mask)
+        out[rows] = ob.permute(1, 0, 2).numpy()
+    return out
+
+
+def check_attention_vs_sdpa(o, seed=0):
+    rng = np.random.default_rng(seed)
+    for (B, Hq, Hkv, D, ctx, kd) in [(2, 4, 2, 8, [5, 3], [2, 3]),
+                                    (3, 6, 3, 16, [0, 7, 1], [4, 0, 1]),
+                                    (1, 2, 1, 4, [9], [5])]:
+        q, kc, vc, cu = _random_attention_case(rng, B, Hq, Hkv, D, ctx, kd)
+        got, _ = o.verify_attention(q, kc, vc, ctx, kd, cu)
+        ref = _sdpa_reference(q, kc, vc, ctx, kd, cu)
+        np.testing.assert_allclose(got, ref, rtol=1e-10, atol=1e-12)
+
+
+def check_attention_special_cases(o, seed=1):
+    rng = np.random.default_rng(seed)
+    D = 8
+    # k = 0: plain decode attention, the single query sees all ctx+1 keys.
+    q, kc, vc, cu = _random_attention_case(rng, 1, 2, 2, D, [6], [0])
+    got, _ = o.verify_attention(q, kc, vc, [6], [0], cu)
+    for h in range(2):
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            torch.from_numpy(q[:, h][None]), torch.from_numpy(kc[0, h, :7][None]),
+            torch.from_numpy(vc[0, h, :7][None]))
+        np.testing.assert_allclose(got[:, h], ref[0].numpy(), rtol=1e-10, atol=1e-12)
+    # ctx = 0: causal self-attention over the verify block alone.
+    q, kc, vc, cu = _random_attention_case(rng, 1, 2, 2, D, [0], [4])
+    got, _ = o.verify_attention(q, kc, vc, [0], [4], cu)
+    for h in range(2):
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            torch.from_numpy(q[:, h][None]), torch.from_numpy(kc[0, h, :5][None]),
+            torch.from_numpy(vc[0, h, :5][None]), is_causal=True)
+        np.testing.assert_allclose(got[:, h], ref[0].numpy(), rtol=1e-10, atol=1e-12)
+    # q = 0: the output is the mean of the visible values (mask width ctx+i+1).
+    ctx, kd = [5], [3]
+    q, kc, vc, cu = _random_attention_case(rng, 1, 2, 1, D, ctx, kd)
+    q[:] = 0.0
+    got, lse = o.verify_attention(q, kc, vc, ctx, kd, cu)
+    for i in range(4):
+        np.testing.assert_allclose(got[i, 0], vc[0, 0, : ctx[0] + i + 1].mean(0), rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lse[i, 1], math.log(ctx[0] + i + 1), rtol=0, atol=1e-12)
+
+
+def check_attention_gqa_mapping(o):
+    # Values constant per KV head: query head h must read KV head h // G.
+    B, Hq, Hkv, D, ctx, kd = 1, 6, 3, 4, [3], [2]
+    rng = np.random.default_rng(2)
+    q, kc, vc, cu = _random_attention_case(rng, B, Hq, Hkv, D, ctx, kd)
+    for j in range(Hkv):
+        vc[0, j] = float(j + 1)
+    got, _ = o.verify_attention(q, kc, vc, ctx, kd, cu)
+    for h in range(Hq):
+        np.testing.assert_allclose(got[:, h], float(h // (Hq // Hkv) + 1), rtol=0, atol=1e-12)
+
+
+# ----------------------------------------------------------------------------
+# LM head
+# ----------------------------------------------------------------------------
+def check_logits_one_hot(o):
+    rng = np.random.default_rng(3)
+    V, H = 11, 5
+    W = rng.standard_normal((V, H))
+    hidden = np.eye(H)
+    got = o.lm_logits(hidden, W, chunk=4)
+    np.testing.assert_array_equal(got, W.T)
+    got2 = o.lm_logits(2.0 * hidden[[1, 3]], W, chunk=3)
+    np.testing.assert_array_equal(got2, 2.0 * W.T[[1, 3]])
+
+
+# ----------------------------------------------------------------------------
+# Acceptance / residual (Sec. III-C)
+# ----------------------------------------------------------------------------
+def check_acceptance_worked_examples(o):
+    g = _golden()
+    for ex in g["acceptance_residual"]:
+        p, q = np.asarray(ex["p"]), np.asarray(ex["q"])
+        for x in range(len(p)):
+            assert abs(o.acceptance_probability(p[x], q[x]) - ex["alpha"][x]) < 1e-15
+        r, Z, fb = o.residual_distribution(p, q)
+        assert not fb
+        np.testing.assert_allclose(r, ex["residual_unnormalised"], rtol=0, atol=1e-15)
+        np.testing.assert_allclose(r / Z, ex["residual"], rtol=0, atol=1e-15)
+    ic = g["inverse_cdf"]
+    r = np.asarray(ic["r"])
+    for u, x in ic["cases"]:
+        assert o.inverse_cdf(r, r.sum(), u)[0] == x, (u, x)
+    ga = g["greedy_argmax"]
+    lg = np.asarray(ga["logits"])[None]
+    res = o.verify_accept(np.repeat(lg, 2, 0), [ga["argmax"]], None, [0.5, 0.5], [0], [0, 2], [1])
+    assert res["accepted_len"][0] == 1 and res["next_token"][0] == ga["argmax"]
+    res = o.verify_accept(np.repeat(lg, 2, 0), [2], None, [0.5, 0.5], [0], [0, 2], [1])
+    assert res["accepted_len"][0] == 0 and res["next_token"][0] == ga["argmax"]
+
+
+def check_residual_properties(o, seed=4):
+    rng = np.random.default_rng(seed)
+    for _ in range(50):
+        V = int(rng.integers(2, 40))
+        p = rng.dirichlet(np.ones(V) * 0.5)
+        q = rng.dirichlet(np.ones(V) * 0.5)
+        r, Z, fb = o.residual_distribution(p, q)
+        assert not fb
+        assert (r >= 0).all()
+        assert abs((r / Z).sum() - 1.0) < 1e-12
+        assert (r[q >= p] == 0).all()
+        # Z equals the total variation distance = 1 - sum(min(p, q)).
+        assert abs(Z - (1.0 - np.minimum(p, q).sum())) < 1e-12
+    # q == p: no residual mass, p is used.
+    p = rng.dirichlet(np.ones(7))
+    r, Z, fb = o.residual_distribution(p, p)
+    assert fb and np.allclose(r, p)
+
+
+def _uniform_logits_rows(p_rows, scale=1.0):
+    return np.log(np.asarray(p_rows)) * scale
+
+
+def check_q_equals_p_accepts_all(o, seed=5):
+    rng = np.random.default_rng(seed)
+    V, k, B = 9, 4, 200
+    P = rng.dirichlet(np.ones(V), size=k + 1)
+    logits = np.tile(np.log(P), (B, 1))
+    q = np.tile(P[:k], (B, 1))
+    drafts = np.concatenate([[rng.choice(V, p=P[i]) for i in range(k)] for _ in range(B)])
+    u = rng.random(B * (k + 1)) * 0.999999
+    cu = np.arange(B + 1) * (k + 1)
+    res = o.verify_accept(logits, drafts, q, u, np.ones(B, int), cu, np.full(B, k))
+    assert (res["accepted_len"] == k).all()
+
+
+def check_strict_comparison(o):
+    # u exactly equal to p/q must reject (accept iff u < p/q).
+    p = np.array([0.5, 0.25, 0.25])
+    q = np.array([0.5, 0.5, 0.0])
+    logits = np.log(np.stack([p, p]))
+    res = o.verify_accept(logits, [1], q[None], [0.5, 0.3], [1], [0, 2], [1])
+    assert res["accepted_len"][0] == 0
+    res = o.verify_accept(logits, [1], q[None], [0.4999999, 0.3], [1], [0, 2], [1])
+    assert res["accepted_len"][0] == 1
+    # q(d) = 0 with p(d) > 0 accepts whatever u is.
+    q2 = np.array([[0.5, 0.5, 0.0]])
+    res = o.verify_accept(logits, [2], q2, [0.99, 0.3], [1], [0, 2], [1])
+    assert res["accepted_len"][0] == 1
+
+
+def _stochastic_trials(o, P, Q, n, seed):
+    """n independent verify steps of one sequence with fixed p rows P[0..k], q rows Q[0..k-1]."""
+    rng = np.random.default_rng(seed)
+    k, V = Q.shape
+    drafts = np.stack([rng.choice(V, size=n, p=Q[i]) for i in range(k)], axis=1).reshape(-1)
+    u = rng.random(n * (k + 1))
+    logits = np.tile(np.log(P), (n, 1))
+    q = np.tile(Q, (n, 1))
+    cu = np.arange(n + 1) * (k + 1)
+    res = o.verify_accept(logits, drafts, q, u, np.ones(n, int), cu, np.full(n, k))
+    return drafts.reshape(n, k), res
+
+
+def check_stochastic_output_law(o, n=60000, seed=6):
+    """Rejection sampling reproduces the verifier's distribution (Sec. III-B/III-C).
+
+    The first emitted token must follow p_0; the token emitted at position 1
+    (given at least one acceptance) p_1; the bonus token (all k accepted) p_k.
+    """
+    rng = np.random.default_rng(seed)
+    V, k = 8, 2
+    P = rng.dirichlet(np.ones(V) * 0.7, size=k + 1)
+    Q = rng.dirichlet(np.ones(V) * 0.7, size=k)
+    drafts, res = _stochastic_trials(o, P, Q, n, seed + 100)
+    a, t = res["accepted_len"], res["next_token"]
+    first = np.where(a >= 1, drafts[:, 0], t)
+    _, pv = stats.chisquare(np.bincount(first, minlength=V), P[0] * n)
+    assert pv > 1e-3, ("first token law", pv)
+    sel = a >= 1
+    second = np.where(a[sel] >= 2, drafts[sel, 1], t[sel])
+    _, pv = stats.chisquare(np.bincount(second, minlength=V), P[1] * sel.sum())
+    assert pv > 1e-3, ("second token law", pv)
+    sel = a == k
+    _, pv = stats.chisquare(np.bincount(t[sel], minlength=V), P[k] * sel.sum())
+    assert pv > 1e-3, ("bonus token law", pv)
+    # Acceptance of draft 0 has probability sum_x min(p_0(x), q_0(x)).
+    pacc = np.minimum(P[0], Q[0]).sum()
+    n_acc = int((a >= 1).sum())
+    assert stats.binomtest(n_acc, n, pacc).pvalue > 1e-3, (n_acc / n, pacc)
+
+
+def check_progress_and_bounds(o, seed=7):
+    rng = np.random.default_rng(seed)
+    V, k = 6, 3
+    P = rng.dirichlet(np.ones(V), size=k + 1)
+    Q = rng.dirichlet(np.ones(V), size=k)
+    _, res = _stochastic_trials(o, P, Q, 3000, seed)
+    a = res["accepted_len"]
+    assert ((a >= 0) & (a <= k)).all()
+    assert ((res["next_token"] >= 0) & (res["next_token"] < V)).all()
+
+
+# ----------------------------------------------------------------------------
+# Greedy speculative decoding == plain argmax decoding (Sec. III-B)
+# ----------------------------------------------------------------------------
+class _ToyLM:
+    """A deterministic toy language model: hidden state of a prefix -> logits."""
+
+    def __init__(self, V, H, seed):
+        rng = np.random.default_rng(seed)
+        self.E1 = rng.standard_normal((V, H))
+        self.E2 = rng.standard_normal((V, H)) * 0.5
+        self.P = rng.standard_normal((7, H)) * 0.3
+        self.W = rng.standard_normal((V, H))
+
+    def hidden(self, prefix):
+        prev = prefix[-2] if len(prefix) > 1 else 0
+        return self.E1[prefix[-1]] + self.E2[prev] + self.P[len(prefix) % 7]
+
+
+def check_greedy_identity(o, seed=8):
+    V, H = 16, 8
+    verifier = _ToyLM(V, H, seed)
+    drafter = _ToyLM(V, H, seed + 1)
+    drafter.W = verifier.W + 0.8 * np.random.default_rng(seed + 2).standard_normal((V, H))
+    prompt = [3, 1, 4]
+    n_new = 60
+    # Plain greedy decoding with the verifier alone.
+    ref = list(prompt)
+    while len(ref) < len(prompt) + n_new:
+        ref.append(int(np.argmax(verifier.W @ verifier.hidden(ref))))
+    for d in (1, 3, 5):
+        y = list(prompt)
+        calls = 0
+        while len(y) < len(prompt) + n_new:
+            drafts = []
+            for _ in range(d):
+                drafts.append(int(np.argmax(drafter.W @ drafter.hidden(y + drafts))))
+            hid = np.stack([verifier.hidden(y + drafts[:i]) for i in range(d + 1)])
+            res = o.verify_accept(o.lm_logits(hid, verifier.W), drafts, None,
+                                  np.full(d + 1, 0.5), [0], [0, d + 1], [d])
+            a = int(res["accepted_len"][0])
+            y += drafts[:a] + [int(res["next_token"][0])]
+            calls += 1
+        assert y[: len(ref)] == ref, (d, y[:len(ref)], ref)
+        assert calls <= n_new
+
+
+# ----------------------------------------------------------------------------
+# KV commit (Algorithm 1 context update)
+# ----------------------------------------------------------------------------
+def check_kv_commit(o, seed=9):
+    rng = np.random.default_rng(seed)
+    B, Hkv, D = 4, 2, 3
+    ctx = np.array([5, 0, 3, 7])
+    kd = np.array([3, 2, 0, 4])
+    acc = np.array([1, 2, 0, 0])
+    cap = 14
+    kc = rng.standard_normal((B, Hkv, cap, D)) + 5.0
+    vc = rng.standard_normal((B, Hkv, cap, D)) + 5.0
+    k2, v2, c2 = o.kv_commit(kc, vc, ctx, acc, kd)
+    np.testing.assert_array_equal(c2, ctx + acc + 1)
+    for b in range(B):
+        for s in range(cap):
+            cleared = ctx[b] + acc[b] + 1 <= s <= ctx[b] + kd[b]
+            if cleared:
+                assert (k2[b, :, s] == 0).all() and (v2[b, :, s] == 0).all()
+            else:
+                assert (k2[b, :, s] == kc[b, :, s]).all() and (v2[b, :, s] == vc[b, :, s]).all()
+
+
+ALL_CHECKS = [
+    check_attention_worked_examples, check_attention_vs_sdpa, check_attention_special_cases,
+    check_attention_gqa_mapping, check_logits_one_hot, check_acceptance_worked_examples,
+    check_residual_properties, check_q_equals_p_accepts_all, check_strict_comparison,
+    check_stochastic_output_law, check_progress_and_bounds, check_greedy_identity,
+    check_kv_commit,
+]

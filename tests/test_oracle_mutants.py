@@ -1,0 +1,55 @@
+"""The oracle's pins must catch plausible mistakes (planted in a copy, on the CPU).
+
+Each case applies one source edit to a private copy of the oracle -- a dropped
+term, a wrong sign or index, an inverted ratio -- and requires that at least one
+pin of ``oracle_pins`` fails on the mutant.  The real oracle is untouched.
+"""
+import inspect
+import types
+
+import pytest
+
+import oracle.spade_oracle as O
+from tests import oracle_pins as pins
+
+MUTANTS = {
+    "dropped_score_scale": ("s = K @ qv / math.sqrt(qv.shape[-1])", "s = K @ qv"),
+    "mask_off_by_one": ("last = int(ctx_lens[b]) + int(row_pos[r])",
+                        "last = int(ctx_lens[b]) + int(row_pos[r]) - 1"),
+    "gqa_modulo": ("kvh = h // G", "kvh = h % Hkv"),
+    "inverted_ratio": ("ratio = p[d] / qd", "ratio = qd / p[d]"),
+    "non_strict_accept": ("ok = u < ratio", "ok = u <= ratio"),
+    "residual_sign": ("r = np.maximum(0.0, _f64(p) - _f64(q))",
+                      "r = np.maximum(0.0, _f64(q) - _f64(p))"),
+    "sample_wrong_row": ("lr = _f64(logits[r0 + a])", "lr = _f64(logits[r0 + k])"),
+    "bonus_from_residual": ("r, Z, fb = p, p.sum(), False",
+                            "r, Z, fb = residual_distribution(p, draft_probs[d0 + a - 1])"),
+    "cdf_non_strict": ("hit = np.nonzero(c > T)[0]", "hit = np.nonzero(c >= T)[0]"),
+    "cdf_descending": ("c = np.cumsum(r)", "c = np.cumsum(r[::-1])[::-1]"),
+    "commit_keeps_correction_slot": ("lo = int(ctx[b]) + a + 1", "lo = int(ctx[b]) + a + 2"),
+    "temperature_2": ("e = np.exp(l - l.max(axis=-1, keepdims=True))",
+                      "e = np.exp(2.0 * (l - l.max(axis=-1, keepdims=True)))"),
+    "greedy_uses_draft_row_shift": ("l = _f64(logits[r0 + i])", "l = _f64(logits[r0 + i + 1])"),
+    "uniform_of_wrong_row": ("u = float(uniforms[r0 + i])", "u = float(uniforms[r0 + k])"),
+}
+
+
+def _mutant(old, new):
+    src = inspect.getsource(O)
+    assert src.count(old) == 1, old
+    mod = types.ModuleType("spade_oracle_mutant")
+    exec(compile(src.replace(old, new), "<mutant>", "exec"), mod.__dict__)
+    return mod
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_pins_catch_mutant(name):
+    mod = _mutant(*MUTANTS[name])
+    caught = []
+    for check in pins.ALL_CHECKS:
+        try:
+            check(mod)
+        except Exception as e:  # AssertionError or a crash both count as caught
+            caught.append((check.__name__, type(e).__name__))
+            break
+    assert caught, f"no pin catches mutant {name}"
