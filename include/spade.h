@@ -1,0 +1,192 @@
+/*
+ * spade.h -- C ABI of the SPADE verify step on GB300 (sm_103a).
+ *
+ * SPADE (edge-cloud speculative decoding) sends a block of k draft tokens from
+ * an edge draft model to a cloud verifier, which scores all k+1 positions in a
+ * single forward pass and keeps the longest accepted prefix plus one corrected
+ * (or bonus) token (Sec. III-B, Sec. III-C, Algorithm 1).  This library holds
+ * the verifier's hot path of that step:
+ *
+ *   spade_verify_attention  attention of the k+1 verify positions against the
+ *                           KV cache (the verifier's forward pass, Algorithm 1
+ *                           "Cloud: in parallel ... in a single forward pass")
+ *   spade_verify_accept     LM head o = g(x_L), softmax (Sec. III-A) fused with
+ *                           the accept test alpha = min(1, p/q) and the residual
+ *                           sampling from norm(max(0, p - q)) (Sec. III-C)
+ *   spade_kv_commit         context update m <- m + a + 1 (Algorithm 1) on the
+ *                           KV cache: keep accepted slots, clear rejected ones
+ *
+ * Conventions shared by every call
+ *  - Every pointer argument is a DEVICE pointer owned by the caller; the
+ *    library keeps no reference after the call returns.
+ *  - Calls are asynchronous on `stream` and never synchronise the host.
+ *  - The return value reports host-side validation and launch errors.  Errors
+ *    found on the device (bad indices, capacity overflow, an expired bounded
+ *    wait) are OR-ed into the caller's device int32 `status` word (the
+ *    SPADE_DEV_* bits); the caller zeroes it and reads it back when it chooses.
+ *  - Every kernel targets sm_103a only; other devices get
+ *    SPADE_ERR_UNSUPPORTED_DEVICE.  There is no fallback path.
+ *  - spade_last_error() returns a thread-local message for the last non-OK
+ *    status returned on the calling thread.
+ *
+ * Row layout of a verify step with B sequences: sequence b has n_draft[b] = k_b
+ * drafts and k_b + 1 verify positions; position i (0 <= i <= k_b) of sequence b
+ * is row cu_q[b] + i, with cu_q[0] = 0 and cu_q[b+1] = cu_q[b] + k_b + 1, so
+ * R = cu_q[B] rows in total.  Position 0 is the last accepted token; position
+ * i >= 1 is draft i-1.
+ */
+#ifndef SPADE_H_
+#define SPADE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same object as cudaStream_t; 0 is the legacy default stream. */
+typedef struct CUstream_st *spade_stream_t;
+
+typedef enum {
+  SPADE_OK = 0,
+  SPADE_ERR_INVALID_ARG = 1,       /* null pointer, negative size, bad mode   */
+  SPADE_ERR_SHAPE = 2,             /* unsupported shape (e.g. D not 64/128)   */
+  SPADE_ERR_CAPACITY = 3,          /* host-visible capacity bound exceeded    */
+  SPADE_ERR_UNSUPPORTED_DEVICE = 4,/* current device is not sm_103            */
+  SPADE_ERR_CUDA = 5,              /* a CUDA runtime / driver call failed     */
+  SPADE_ERR_WORKSPACE = 6,         /* workspace missing, too small, misaligned*/
+} spade_status;
+
+/* Device status word bits (OR-ed by kernels into the caller's int32). */
+#define SPADE_DEV_BAD_INDEX 0x1  /* cu_q inconsistent, n_draft > max_k, token id out of range */
+#define SPADE_DEV_CAPACITY  0x2  /* ctx_lens[b] + n_draft[b] + 1 > cap                       */
+#define SPADE_DEV_TIMEOUT   0x4  /* a bounded device-side wait expired; outputs are invalid  */
+#define SPADE_DEV_FALLBACK  0x8  /* a residual had no positive mass; p was sampled instead   */
+
+/* ------------------------------------------------------------------------ */
+/* Verify attention (Sec. III-B verification stage; Algorithm 1 cloud step)  */
+/* ------------------------------------------------------------------------ */
+/*
+ * For every sequence b, position i in [0, k_b] and query head h:
+ *   out[cu_q[b]+i, h, :] = softmax(q . K^T / sqrt(D)) V
+ * over the keys in slots [0, ctx_lens[b] + i] of KV head h / (Hq / Hkv).  Slots
+ * [0, ctx_b) hold the committed context and slots [ctx_b, ctx_b + k_b] the
+ * verify block itself (written by the caller before this call), so the mask is
+ * causal inside the draft block only.  Scores are scaled by 1/sqrt(D); inputs
+ * are post-RoPE; no softcap, window or ALiBi.
+ *
+ *   q          bf16 [R, Hq, D] row-major (row = cu_q[b] + i)
+ *   k_cache    bf16 [B, Hkv, cap, D] row-major; 16-byte aligned
+ *   v_cache    bf16 [B, Hkv, cap, D] row-major; 16-byte aligned
+ *   ctx_lens   int32 [B] committed context length per sequence
+ *   n_draft    int32 [B] draft count k_b, 0 <= k_b <= max_k
+ *   cu_q       int32 [B+1] row offsets (see above)
+ *   out        bf16 [R, Hq, D] written
+ *   lse        float32 [R, Hq] natural-log sum-exp of the scaled scores, or NULL
+ *   B, Hq, Hkv, D, cap, max_k, R   sizes; Hq % Hkv == 0; D in {64, 128};
+ *              Hq / Hkv * (max_k + 1) query rows share each KV head
+ *   workspace  device scratch of at least spade_attn_workspace_size(...) bytes,
+ *              256-byte aligned, ZEROED ONCE by the caller after allocation;
+ *              every call that completes leaves it zeroed again.  Calls that
+ *              share a workspace must be ordered (same stream or events).
+ *   status     device int32, SPADE_DEV_* bits OR-ed in
+ * Slots beyond ctx_b + k_b are never read into the result, whatever they hold.
+ */
+spade_status spade_verify_attention(const void *q, const void *k_cache, const void *v_cache,
+                                    const int32_t *ctx_lens, const int32_t *n_draft,
+                                    const int32_t *cu_q, void *out, float *lse, int32_t B,
+                                    int32_t Hq, int32_t Hkv, int32_t D, int32_t cap,
+                                    int32_t max_k, int32_t R, void *workspace,
+                                    size_t workspace_bytes, int32_t *status,
+                                    spade_stream_t stream);
+
+/* Bytes of workspace spade_verify_attention needs for these sizes on the
+ * current device (0 on invalid sizes). */
+size_t spade_attn_workspace_size(int32_t B, int32_t Hq, int32_t Hkv, int32_t D, int32_t cap,
+                                 int32_t max_k);
+
+/* ------------------------------------------------------------------------ */
+/* LM head + softmax + accept/reject + residual sampling (Sec. III-A/III-C)  */
+/* ------------------------------------------------------------------------ */
+/*
+ * logits[r, x] = sum_j hidden[r, j] * w_lm[x, j] (fp32 accumulation on the
+ * tensor cores; the logits never leave the chip) and p_r = softmax(logits[r]).
+ * For every sequence b (rows r_i = cu_q[b] + i, draft d_i = draft_tokens[cu_q[b]
+ * - b + i] for i < k_b):
+ *   greedy (mode 0):     draft i is accepted iff d_i == argmax_x logits[r_i, x]
+ *                        (lowest index on ties);
+ *   stochastic (mode 1): draft i is accepted iff u[r_i] < p_{r_i}(d_i) / q_i(d_i)
+ *                        with q_i = draft_probs[cu_q[b] - b + i, :] (q_i(d_i) = 0
+ *                        accepts iff p(d_i) > 0);
+ * acceptance stops at the first rejection; a_b = number of accepted drafts is
+ * written to accepted_len[b].  next_token[b] is, with r* = cu_q[b] + a_b:
+ *   greedy:      argmax_x logits[r*, x];
+ *   stochastic:  if a_b < k_b a draw from norm(max(0, p_{r*} - q_{a_b})), else
+ *                (bonus) a draw from p_{r*}; the draw is the smallest x whose
+ *                cumulative mass (ascending x, fp64) exceeds u[cu_q[b] + k_b] * Z.
+ *
+ *   hidden        bf16 [R, H] row-major, 16-byte aligned, H % 8 == 0
+ *   w_lm          bf16 [V, H] row-major (nn.Linear layout), 16-byte aligned
+ *   draft_tokens  int32 [R - B]
+ *   draft_probs   float32 [R - B, V] row-major, or NULL when no sequence is
+ *                 stochastic
+ *   uniforms      float32 [R] in [0, 1)
+ *   mode          int32 [B], 0 greedy / 1 stochastic
+ *   cu_q, n_draft int32 [B+1], [B]
+ *   accepted_len  int32 [B] written;  next_token int32 [B] written
+ *   workspace     scratch of spade_accept_workspace_size(...) bytes, 256-byte
+ *                 aligned, ZEROED ONCE by the caller; completed calls leave the
+ *                 parts that must start at zero zeroed again.
+ *   status        device int32, SPADE_DEV_* bits OR-ed in
+ * The kernel keeps every block of the grid resident at once (cooperative
+ * launch) and meets at bounded device-wide barriers; if a barrier expires the
+ * outputs are invalid and SPADE_DEV_TIMEOUT is set; zero the workspace again
+ * before the next call.
+ */
+spade_status spade_verify_accept(const void *hidden, const void *w_lm,
+                                 const int32_t *draft_tokens, const float *draft_probs,
+                                 const float *uniforms, const int32_t *mode,
+                                 const int32_t *cu_q, const int32_t *n_draft,
+                                 int32_t *accepted_len, int32_t *next_token, int32_t B,
+                                 int32_t R, int32_t H, int32_t V, void *workspace,
+                                 size_t workspace_bytes, int32_t *status,
+                                 spade_stream_t stream);
+
+/* Bytes of workspace spade_verify_accept needs (0 on invalid sizes). */
+size_t spade_accept_workspace_size(int32_t B, int32_t R, int32_t H, int32_t V);
+
+/* ------------------------------------------------------------------------ */
+/* KV commit (Algorithm 1 context update)                                    */
+/* ------------------------------------------------------------------------ */
+/*
+ * For every sequence b with a_b = accepted_len[b] (0 <= a_b <= n_draft[b]):
+ * slots [ctx_b + a_b + 1, ctx_b + n_draft[b]] of k_cache and v_cache (every KV
+ * head) are cleared to zero and ctx_lens[b] += a_b + 1 (the last accepted
+ * token plus a_b drafts are now committed; the corrected / bonus token is
+ * position 0 of the next verify block).
+ *   k_cache, v_cache bf16 [B, Hkv, cap, D] updated in place
+ *   ctx_lens         int32 [B] updated in place
+ *   accepted_len     int32 [B];  n_draft int32 [B]
+ *   status           device int32 (SPADE_DEV_BAD_INDEX if a_b is out of range,
+ *                    SPADE_DEV_CAPACITY if the block exceeds cap; such a
+ *                    sequence is left untouched)
+ */
+spade_status spade_kv_commit(void *k_cache, void *v_cache, int32_t *ctx_lens,
+                             const int32_t *accepted_len, const int32_t *n_draft, int32_t B,
+                             int32_t Hkv, int32_t D, int32_t cap, int32_t *status,
+                             spade_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* Diagnostics                                                               */
+/* ------------------------------------------------------------------------ */
+const char *spade_status_string(spade_status s);
+const char *spade_last_error(void);
+/* Library version, e.g. "spade-gb300 0.1 sm_103a". */
+const char *spade_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPADE_H_ */

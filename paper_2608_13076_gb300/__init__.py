@@ -1,0 +1,223 @@
+"""SPADE verify step on GB300: Python binding of the C-ABI library libspade.so.
+
+This module only marshals arguments: it checks dtypes and layouts of torch
+tensors and passes raw device pointers, sizes and the current CUDA stream to
+the library's entry points.  Every step of the verify path runs in the
+library's CUDA kernels; there is no Python or CPU fallback, and a call fails
+loudly if the library is missing.
+
+Entry points (same names as the C ABI in include/spade.h):
+    spade_verify_attention  verify-position attention against the KV cache
+    spade_verify_accept     LM head + softmax + accept/reject + residual sampling
+    spade_kv_commit         append accepted positions, roll back rejected ones
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import _build
+
+__all__ = [
+    "SpadeError", "load", "build", "library_path",
+    "spade_verify_attention", "spade_verify_accept", "spade_kv_commit",
+    "spade_attn_workspace_size", "spade_accept_workspace_size",
+    "attn_workspace", "accept_workspace", "status_tensor", "check_status",
+    "DEV_BAD_INDEX", "DEV_CAPACITY", "DEV_TIMEOUT", "DEV_FALLBACK",
+]
+
+DEV_BAD_INDEX = 0x1
+DEV_CAPACITY = 0x2
+DEV_TIMEOUT = 0x4
+DEV_FALLBACK = 0x8
+
+_lib = None
+
+
+class SpadeError(RuntimeError):
+    """A non-OK status returned by the library (message from spade_last_error)."""
+
+    def __init__(self, status, message):
+        super().__init__(f"{message} [status {status}]")
+        self.status = status
+
+
+def library_path() -> str:
+    return _build.LIB_PATH
+
+
+def build(force: bool = False) -> str:
+    return _build.build(force=force)
+
+
+_i32 = ctypes.c_int32
+_vp = ctypes.c_void_p
+_sz = ctypes.c_size_t
+
+
+def load():
+    """Load libspade.so (built in-tree); raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = library_path()
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build the CUDA library first "
+                           "(python -c 'import __graft_entry__ as g; g.build()')")
+    lib = ctypes.CDLL(path)
+    lib.spade_verify_attention.restype = _i32
+    lib.spade_verify_attention.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                           _i32, _i32, _i32, _i32, _i32, _i32, _i32,
+                                           _vp, _sz, _vp, _vp]
+    lib.spade_attn_workspace_size.restype = _sz
+    lib.spade_attn_workspace_size.argtypes = [_i32] * 6
+    lib.spade_verify_accept.restype = _i32
+    lib.spade_verify_accept.argtypes = [_vp] * 10 + [_i32] * 4 + [_vp, _sz, _vp, _vp]
+    lib.spade_accept_workspace_size.restype = _sz
+    lib.spade_accept_workspace_size.argtypes = [_i32] * 4
+    lib.spade_kv_commit.restype = _i32
+    lib.spade_kv_commit.argtypes = [_vp] * 5 + [_i32] * 4 + [_vp, _vp]
+    lib.spade_status_string.restype = ctypes.c_char_p
+    lib.spade_status_string.argtypes = [_i32]
+    lib.spade_last_error.restype = ctypes.c_char_p
+    lib.spade_last_error.argtypes = []
+    lib.spade_version.restype = ctypes.c_char_p
+    lib.spade_version.argtypes = []
+    _lib = lib
+    return lib
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check_rc(rc):
+    if rc != 0:
+        lib = load()
+        raise SpadeError(rc, f"{lib.spade_status_string(rc).decode()}: {lib.spade_last_error().decode()}")
+
+
+def _need(t, name, dtype, ndim=None):
+    if t is None:
+        raise ValueError(f"{name} is required")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if ndim is not None and t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims, got {t.dim()}")
+
+
+def status_tensor(device="cuda"):
+    """A zeroed device int32 status word."""
+    return torch.zeros(1, dtype=torch.int32, device=device)
+
+
+def check_status(status):
+    """Reads the device status word (synchronises) and returns its SPADE_DEV_* bits."""
+    return int(status.item())
+
+
+# ---------------------------------------------------------------------------
+def spade_attn_workspace_size(B, Hq, Hkv, D, cap, max_k):
+    return int(load().spade_attn_workspace_size(B, Hq, Hkv, D, cap, max_k))
+
+
+def attn_workspace(B, Hq, Hkv, D, cap, max_k, device="cuda"):
+    """A zeroed workspace for spade_verify_attention (zeroed once; calls keep it zeroed)."""
+    n = spade_attn_workspace_size(B, Hq, Hkv, D, cap, max_k)
+    if n == 0:
+        raise SpadeError(-1, "spade_attn_workspace_size returned 0: " + load().spade_last_error().decode())
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def spade_verify_attention(q, k_cache, v_cache, ctx_lens, n_draft, cu_q, out, lse=None, *,
+                           max_k, workspace, status, stream=None):
+    """out[cu_q[b]+i, h] = softmax(q K^T / sqrt(D)) V over keys [0, ctx_b + i] (KV head h // G)."""
+    _need(q, "q", torch.bfloat16, 3)
+    _need(k_cache, "k_cache", torch.bfloat16, 4)
+    _need(v_cache, "v_cache", torch.bfloat16, 4)
+    for t, n in ((ctx_lens, "ctx_lens"), (n_draft, "n_draft"), (cu_q, "cu_q"), (status, "status")):
+        _need(t, n, torch.int32, 1)
+    _need(out, "out", torch.bfloat16, 3)
+    if lse is not None:
+        _need(lse, "lse", torch.float32, 2)
+    _need(workspace, "workspace", torch.uint8, 1)
+    if v_cache.shape != k_cache.shape:
+        raise ValueError("k_cache and v_cache shapes differ")
+    R, Hq, D = q.shape
+    B, Hkv, cap, Dk = k_cache.shape
+    if Dk != D or tuple(out.shape) != (R, Hq, D) or ctx_lens.numel() != B or n_draft.numel() != B \
+            or cu_q.numel() != B + 1:
+        raise ValueError("inconsistent attention shapes")
+    rc = load().spade_verify_attention(
+        _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(ctx_lens), _ptr(n_draft), _ptr(cu_q), _ptr(out),
+        _ptr(lse), B, Hq, Hkv, D, cap, int(max_k), R, _ptr(workspace), workspace.numel(),
+        _ptr(status), _stream(stream))
+    _check_rc(rc)
+    return out
+
+
+# ---------------------------------------------------------------------------
+def spade_accept_workspace_size(B, R, H, V):
+    return int(load().spade_accept_workspace_size(B, R, H, V))
+
+
+def accept_workspace(B, R, H, V, device="cuda"):
+    """A zeroed workspace for spade_verify_accept (zeroed once; calls keep it usable)."""
+    n = spade_accept_workspace_size(B, R, H, V)
+    if n == 0:
+        raise SpadeError(-1, "spade_accept_workspace_size returned 0: " + load().spade_last_error().decode())
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def spade_verify_accept(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
+                        accepted_len, next_token, *, workspace, status, stream=None):
+    """Greedy / rejection-sampling verification of every sequence (see include/spade.h)."""
+    _need(hidden, "hidden", torch.bfloat16, 2)
+    _need(w_lm, "w_lm", torch.bfloat16, 2)
+    _need(uniforms, "uniforms", torch.float32, 1)
+    for t, n in ((draft_tokens, "draft_tokens"), (mode, "mode"), (cu_q, "cu_q"), (n_draft, "n_draft"),
+                 (accepted_len, "accepted_len"), (next_token, "next_token"), (status, "status")):
+        _need(t, n, torch.int32, 1)
+    if draft_probs is not None:
+        _need(draft_probs, "draft_probs", torch.float32, 2)
+    _need(workspace, "workspace", torch.uint8, 1)
+    R, H = hidden.shape
+    V, H2 = w_lm.shape
+    B = n_draft.numel()
+    if H2 != H or uniforms.numel() != R or draft_tokens.numel() != R - B or cu_q.numel() != B + 1 \
+            or mode.numel() != B or accepted_len.numel() != B or next_token.numel() != B:
+        raise ValueError("inconsistent accept shapes")
+    if draft_probs is not None and tuple(draft_probs.shape) != (R - B, V):
+        raise ValueError("draft_probs must be [R - B, V]")
+    rc = load().spade_verify_accept(
+        _ptr(hidden), _ptr(w_lm), _ptr(draft_tokens), _ptr(draft_probs), _ptr(uniforms), _ptr(mode),
+        _ptr(cu_q), _ptr(n_draft), _ptr(accepted_len), _ptr(next_token), B, R, H, V,
+        _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream))
+    _check_rc(rc)
+    return accepted_len, next_token
+
+
+# ---------------------------------------------------------------------------
+def spade_kv_commit(k_cache, v_cache, ctx_lens, accepted_len, n_draft, *, status, stream=None):
+    """ctx_lens += accepted_len + 1; rejected draft slots of the caches are cleared."""
+    _need(k_cache, "k_cache", torch.bfloat16, 4)
+    _need(v_cache, "v_cache", torch.bfloat16, 4)
+    for t, n in ((ctx_lens, "ctx_lens"), (accepted_len, "accepted_len"), (n_draft, "n_draft"),
+                 (status, "status")):
+        _need(t, n, torch.int32, 1)
+    B, Hkv, cap, D = k_cache.shape
+    rc = load().spade_kv_commit(_ptr(k_cache), _ptr(v_cache), _ptr(ctx_lens), _ptr(accepted_len),
+                                _ptr(n_draft), B, Hkv, D, cap, _ptr(status), _stream(stream))
+    _check_rc(rc)

@@ -1,0 +1,71 @@
+// kv_commit.cu -- the context update of Algorithm 1 (m <- m + a + 1) applied to
+// the KV cache: the accepted prefix of the verify block stays, the rejected
+// draft slots are cleared, ctx_lens advances by a + 1.
+#include <cuda_bf16.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace spade {
+namespace commit {
+
+// One CTA per sequence: every thread reads ctx_lens[b] before any thread
+// writes it, so the in-place update cannot race.
+__global__ void __launch_bounds__(256) kv_commit_kernel(uint4 *k_cache, uint4 *v_cache,
+                                                       int32_t *ctx_lens, const int32_t *accepted,
+                                                       const int32_t *n_draft, int Hkv, int D,
+                                                       int cap, int32_t *status) {
+  const int b = blockIdx.x;
+  const int ctx = ctx_lens[b];
+  const int a = accepted[b];
+  const int k = n_draft[b];
+  int bad = 0;
+  if (ctx < 0 || k < 0 || a < 0 || a > k) bad = SPADE_DEV_BAD_INDEX;
+  else if (static_cast<int64_t>(ctx) + k + 1 > cap) bad = SPADE_DEV_CAPACITY;
+  __syncthreads();
+  if (bad) {
+    if (threadIdx.x == 0) atomicOr(status, bad);
+    return;
+  }
+  const int lo = ctx + a + 1;        // first rejected slot
+  const int n_slots = k - a;         // slots lo .. ctx + k
+  const int vec = D / 8;             // 16-byte vectors per slot
+  const int per_head = n_slots * vec;
+  const int total = Hkv * per_head;
+  const uint4 z = make_uint4(0, 0, 0, 0);
+  for (int e = threadIdx.x; e < total; e += blockDim.x) {
+    const int h = e / per_head;
+    const int r = e - h * per_head;
+    const size_t off = ((static_cast<size_t>(b) * Hkv + h) * cap + lo) * vec + r;
+    k_cache[off] = z;
+    v_cache[off] = z;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) ctx_lens[b] = lo;
+}
+
+}  // namespace commit
+}  // namespace spade
+
+using namespace spade;
+
+extern "C" spade_status spade_kv_commit(void *k_cache, void *v_cache, int32_t *ctx_lens,
+                                        const int32_t *accepted_len, const int32_t *n_draft,
+                                        int32_t B, int32_t Hkv, int32_t D, int32_t cap,
+                                        int32_t *status, spade_stream_t stream) {
+  if (!k_cache || !v_cache || !ctx_lens || !accepted_len || !n_draft || !status)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_kv_commit: null pointer argument");
+  if (B <= 0 || Hkv <= 0 || cap <= 0 || D <= 0)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_kv_commit: non-positive size");
+  if (D % 8) return fail(SPADE_ERR_SHAPE, "spade_kv_commit: D = %d must be a multiple of 8", D);
+  if (!aligned(k_cache, 16) || !aligned(v_cache, 16))
+    return fail(SPADE_ERR_INVALID_ARG, "spade_kv_commit: caches must be 16-byte aligned");
+  spade_status st = device_info(nullptr, nullptr);
+  if (st != SPADE_OK) return st;
+  commit::kv_commit_kernel<<<B, 256, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      static_cast<uint4 *>(k_cache), static_cast<uint4 *>(v_cache), ctx_lens, accepted_len,
+      n_draft, Hkv, D, cap, status);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "kv_commit launch");
+  return SPADE_OK;
+}

@@ -1,0 +1,82 @@
+"""The C-ABI library builds for sm_103a, loads, and exports what include/spade.h declares.
+
+CPU only: no call here launches a kernel.  Host-side validation runs before
+any device query, so argument errors are checked without a GPU.
+"""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+import paper_2608_13076_gb300 as spade
+from paper_2608_13076_gb300 import _build
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "spade.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(spade_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    _build.build()
+    return spade.load()
+
+
+def test_header_declares_the_entry_points():
+    names = declared_functions()
+    for n in ("spade_verify_attention", "spade_verify_accept", "spade_kv_commit",
+              "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_last_error",
+              "spade_status_string"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    out = subprocess.run(["nm", "-D", "--defined-only", _build.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r" T (\w+)$", out, flags=re.M))
+    missing = [n for n in declared_functions() if n not in exported]
+    assert not missing, missing
+    for n in declared_functions():
+        assert hasattr(lib, n)
+
+
+def test_library_is_built_for_sm103a(lib):
+    # The fatbinary holds sm_103a code only (names from cuobjdump's listing, not its contents).
+    r = subprocess.run(["cuobjdump", "--list-elf", _build.LIB_PATH], capture_output=True, text=True)
+    assert r.returncode == 0
+    assert "sm_103a" in r.stdout
+    assert all("sm_103" in line for line in r.stdout.splitlines() if line.strip())
+
+
+def test_status_strings(lib):
+    assert lib.spade_status_string(0) == b"SPADE_OK"
+    assert lib.spade_status_string(4) == b"SPADE_ERR_UNSUPPORTED_DEVICE"
+    assert b"sm_103a" in lib.spade_version()
+
+
+def test_null_arguments_rejected_before_any_device_work(lib):
+    rc = lib.spade_verify_attention(*([None] * 8), 1, 8, 8, 128, 300, 4, 5, None, 0, None, None)
+    assert rc == 1 and b"null" in lib.spade_last_error()
+    rc = lib.spade_verify_accept(*([None] * 10), 1, 5, 512, 1024, None, 0, None, None)
+    assert rc == 1
+    rc = lib.spade_kv_commit(*([None] * 5), 1, 8, 128, 300, None, None)
+    assert rc == 1
+
+
+def test_bad_shapes_rejected(lib):
+    p = ctypes.c_void_p(16)
+    args = [p] * 7 + [None]
+    # Hq not a multiple of Hkv
+    assert lib.spade_verify_attention(*args, 1, 6, 4, 128, 300, 4, 5, p, 1 << 20, p, None) == 2
+    # head dim 96 unsupported
+    assert lib.spade_verify_attention(*args, 1, 8, 8, 96, 300, 4, 5, p, 1 << 20, p, None) == 2
+    # hidden size not a multiple of 8
+    assert lib.spade_verify_accept(*([p] * 10), 1, 5, 500, 1024, p, 1 << 20, p, None) == 2
+    # head dim not a multiple of 8 for commit
+    assert lib.spade_kv_commit(*([p] * 5), 1, 8, 12, 300, p, None) == 2

@@ -1,0 +1,141 @@
+"""GPU parity: the CUDA verify step (through the C ABI) against the float64 oracle.
+
+Small cases span several key chunks, vocabulary tiles and ragged tails and are
+checked element by element; the benchmark workloads are checked at full size
+(attention on sampled (row, head) pairs, accept decisions on every sequence).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle.spade_oracle as O
+import paper_2608_13076_gb300 as spade
+from paper_2608_13076_gb300 import workloads as W
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+SMALL = {
+    "gqa_mixed": W.WorkloadSpec("gqa_mixed", B=3, Hq=8, Hkv=2, D=128, H=520, V=1000, ctx=(50, 700),
+                                k=(0, 7), mode="mixed", seed=11),
+    "d64_stochastic": W.WorkloadSpec("d64_stochastic", B=2, Hq=4, Hkv=4, D=64, H=256, V=3000,
+                                     ctx=(1, 200), k=(1, 3), mode="stochastic", seed=12),
+    "plain_decode_k0": W.WorkloadSpec("plain_decode_k0", B=4, Hq=8, Hkv=8, D=128, H=512, V=700,
+                                      ctx=(10, 500), k=(0, 0), mode="greedy", seed=13),
+    "empty_context": W.WorkloadSpec("empty_context", B=2, Hq=4, Hkv=1, D=128, H=128, V=513,
+                                    ctx=(0, 0), k=(3, 3), mode="stochastic", seed=14),
+    "long_split": W.WorkloadSpec("long_split", B=1, Hq=8, Hkv=1, D=128, H=1024, V=20000,
+                                 ctx=(20000, 20000), k=(6, 6), mode="greedy", match_prob=0.9, seed=15),
+    "many_rows": W.WorkloadSpec("many_rows", B=16, Hq=16, Hkv=2, D=128, H=384, V=5000, ctx=(30, 900),
+                                k=(1, 8), mode="mixed", seed=16),
+}
+
+
+@pytest.fixture(scope="module")
+def dev(gpu_lib):
+    return torch.device("cuda:0")
+
+
+def _poison_unused_slots(wl):
+    """Fill cache slots beyond ctx+k with NaN: they must never reach the result."""
+    for b in range(wl["B"]):
+        L = int(wl["ctx_lens"][b] + wl["n_draft"][b] + 1)
+        wl["k_cache"][b, :, L:] = float("nan")
+        wl["v_cache"][b, :, L:] = float("nan")
+
+
+@pytest.mark.parametrize("name", sorted(SMALL))
+def test_attention_small(dev, name):
+    wl = W.make_workload(SMALL[name], device=dev, cache_pad=70)
+    _poison_unused_slots(wl)
+    out, lse, st = parity.gpu_attention(wl)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    ref, ref_lse = parity.oracle_attention(wl)
+    n, bad, worst = parity.compare_attention(out, ref)
+    assert bad == 0, f"{bad} elements out of tolerance, worst {worst:.3g}"
+    np.testing.assert_allclose(parity.to_np(lse), ref_lse, rtol=0, atol=2e-3)
+
+
+@pytest.mark.parametrize("name", sorted(SMALL))
+def test_accept_small(dev, name):
+    wl = W.make_workload(SMALL[name], device=dev)
+    acc, tok, st = parity.gpu_accept(wl)
+    torch.cuda.synchronize()
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0
+    ref = parity.oracle_accept(wl)
+    cmp = parity.compare_accept(acc, tok, ref)
+    assert cmp["mismatch_unflagged"] == 0, cmp
+
+
+@pytest.mark.parametrize("name", sorted(SMALL))
+def test_kv_commit_small(dev, name):
+    wl = W.make_workload(SMALL[name], device=dev, cache_pad=5)
+    acc, _, st = parity.gpu_accept(wl)
+    kc, vc, ctx = wl["k_cache"].clone(), wl["v_cache"].clone(), wl["ctx_lens"].clone()
+    spade.spade_kv_commit(kc, vc, ctx, acc, wl["n_draft"], status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0
+    rk, rv, rctx = O.kv_commit(parity.to_np(wl["k_cache"]), parity.to_np(wl["v_cache"]),
+                               parity.to_np(wl["ctx_lens"]), parity.to_np(acc), parity.to_np(wl["n_draft"]))
+    assert np.array_equal(parity.to_np(ctx), rctx)
+    assert np.array_equal(parity.to_np(kc), rk)
+    assert np.array_equal(parity.to_np(vc), rv)
+
+
+def test_repeat_calls_reuse_workspace(dev):
+    """Workspaces stay valid across calls (self-resetting counters / barriers)."""
+    spec = SMALL["many_rows"]
+    wl = W.make_workload(spec, device=dev)
+    max_k = int(wl["n_draft"].max())
+    ws_a = spade.attn_workspace(wl["B"], wl["Hq"], wl["Hkv"], wl["D"], wl["cap"], max_k, device=dev)
+    ws_b = spade.accept_workspace(wl["B"], wl["R"], wl["H"], wl["V"], device=dev)
+    outs, toks = [], []
+    for _ in range(3):
+        out, _, st = parity.gpu_attention(wl, workspace=ws_a)
+        acc, tok, st2 = parity.gpu_accept(wl, workspace=ws_b)
+        outs.append(out.clone())
+        toks.append((acc.clone(), tok.clone()))
+    torch.cuda.synchronize()
+    for o in outs[1:]:
+        assert torch.equal(o, outs[0])
+    for a, t in toks[1:]:
+        assert torch.equal(a, toks[0][0]) and torch.equal(t, toks[0][1])
+    assert int(ws_a[:1024].sum()) == 0  # counters back at zero
+
+
+# ---------------------------------------------------------------------------
+# Benchmark workloads at full size (the launch configuration bench.py times).
+FULL = ["tiny", "llama2_7b_greedy", "llama2_7b_stochastic", "llama3_8b", "long_70b"]
+
+
+def _sample_pairs(wl, n, seed):
+    rng = np.random.default_rng(seed)
+    R, Hq = wl["R"], wl["Hq"]
+    if R * Hq <= n:
+        return [(r, h) for r in range(R) for h in range(Hq)]
+    cu = parity.to_np(wl["cu_q"])
+    pairs = {(int(cu[b]), 0) for b in range(wl["B"])}            # position 0 of each sequence
+    pairs |= {(int(cu[b + 1]) - 1, Hq - 1) for b in range(wl["B"])}  # last position
+    while len(pairs) < n:
+        pairs.add((int(rng.integers(R)), int(rng.integers(Hq))))
+    return sorted(pairs)
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_full_workload(dev, name):
+    wl = W.make_workload(W.SPECS[name], device=dev)
+    out, lse, st = parity.gpu_attention(wl)
+    acc, tok, st2 = parity.gpu_accept(wl)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert int(st2.item()) & ~spade.DEV_FALLBACK == 0
+    pairs = _sample_pairs(wl, 256, 7)
+    ref, _ = parity.oracle_attention(wl, rows=pairs)
+    n, bad, worst = parity.compare_attention(out, ref, rows=pairs)
+    assert bad == 0, f"attention: {bad} bad elements over {n} pairs, worst {worst:.3g}"
+    ref_acc = parity.oracle_accept(wl)
+    cmp = parity.compare_accept(acc, tok, ref_acc)
+    print(f"{name}: accepted {parity.to_np(acc).tolist()} flagged {cmp['flagged']} "
+          f"flagged-mismatch {cmp['mismatch_flagged']}")
+    assert cmp["mismatch_unflagged"] == 0, cmp
