@@ -1,0 +1,379 @@
+#!/usr/bin/env python
+"""Benchmark of the SPADE verify step on GB300.
+
+One step = one pass of the whole hot path over one batch of synthetic input:
+verify attention (one layer) -> LM head + accept/reject + residual sampling ->
+KV commit, all on one stream through the C-ABI library.  The metric is the
+number of committed tokens (sum over sequences of accepted drafts + 1) per
+second of device time, with inputs resident in HBM.  `e2e` repeats it through
+the same public calls with the per-step inputs in pinned host memory, copied
+in and the step's result read back inside the timed region.
+
+Default workload: the Llama-3-8B-shaped verifier step (batch 8, GQA 32/8,
+head_dim 128, hidden 4096, vocab 128256, ctx 4096, k = 8, stochastic), the
+paper's own verifier shape.  `--impl reference` times the float64 CPU oracle
+on the same workload instead (bounded samples: one sequence per step).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import signal
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+from paper_2608_13076_gb300 import workloads as W  # noqa: E402
+
+L2_BYTES = 129 * 1024 * 1024
+METRIC = "verified tokens/s per verify step (1 GB300); verify-attn HBM GB/s vs peak"
+UNIT = "tokens/s"
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _work_bytes(wl):
+    """Algorithmic bytes of the two dominant kernels for one step."""
+    ctx = wl["ctx_lens"].long().cpu()
+    kd = wl["n_draft"].long().cpu()
+    keys = int((ctx + kd + 1).sum())
+    attn = keys * wl["Hkv"] * wl["D"] * 2 * 2 + 2 * wl["R"] * wl["Hq"] * wl["D"] * 2
+    n_stoch = int((wl["mode"].cpu() == W.STOCHASTIC).sum()) if wl["draft_probs"] is not None else 0
+    lm = wl["V"] * wl["H"] * 2 + wl["R"] * wl["H"] * 2 + n_stoch * wl["V"] * 4
+    lm_flop = 2.0 * wl["R"] * wl["V"] * wl["H"]
+    attn_flop = 0.0
+    G = wl["Hq"] // wl["Hkv"]
+    for b in range(wl["B"]):
+        for i in range(int(kd[b]) + 1):
+            attn_flop += 4.0 * wl["D"] * (int(ctx[b]) + i + 1) * wl["Hkv"] * G
+    return attn, lm, lm_flop, attn_flop, keys
+
+
+class Clocks:
+    """Samples nvidia-smi clocks and throttle reasons while running."""
+
+    def __init__(self, index):
+        self.proc = None
+        self.path = None
+        self.index = index
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index),
+                 "--query-gpu=clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.send_signal(signal.SIGTERM)
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path:
+            return None
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 8:
+                    continue
+                try:
+                    sm.append(float(parts[0]))
+                    mx.append(float(parts[1]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[4:8]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------
+def run_spade(args, ws, rank, local):
+    import paper_2608_13076_gb300 as spade
+    from paper_2608_13076_gb300 import _build
+
+    if rank == 0 or not _build.up_to_date():
+        _build.build()
+    if ws > 1:
+        torch.distributed.barrier()
+    spade.load()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    spec = W.SPECS[args.workload]
+    wl = W.make_workload(spec, device=dev)
+    B, R = wl["B"], wl["R"]
+    max_k = int(wl["n_draft"].max())
+    out = torch.empty_like(wl["q"])
+    acc = torch.zeros(B, dtype=torch.int32, device=dev)
+    tok = torch.zeros(B, dtype=torch.int32, device=dev)
+    status = spade.status_tensor(dev)
+    ws_attn = spade.attn_workspace(B, wl["Hq"], wl["Hkv"], wl["D"], wl["cap"], max_k, device=dev)
+    ws_acc = spade.accept_workspace(B, R, wl["H"], wl["V"], device=dev)
+    ctx0 = wl["ctx_lens"].clone()
+    stream = torch.cuda.current_stream()
+
+    def step(inputs, evs=None):
+        if evs:
+            evs[0].record(stream)
+        spade.spade_verify_attention(inputs["q"], wl["k_cache"], wl["v_cache"], inputs["ctx_lens"],
+                                     inputs["n_draft"], inputs["cu_q"], out, None, max_k=max_k,
+                                     workspace=ws_attn, status=status)
+        if evs:
+            evs[1].record(stream)
+        spade.spade_verify_accept(inputs["hidden"], wl["w_lm"], inputs["draft_tokens"], inputs["draft_probs"],
+                                  inputs["uniforms"], inputs["mode"], inputs["cu_q"], inputs["n_draft"], acc,
+                                  tok, workspace=ws_acc, status=status)
+        if evs:
+            evs[2].record(stream)
+        spade.spade_kv_commit(wl["k_cache"], wl["v_cache"], inputs["ctx_lens"], acc, inputs["n_draft"],
+                              status=status)
+        if evs:
+            evs[3].record(stream)
+
+    attn_bytes, lm_bytes, lm_flop, attn_flop, keys = _work_bytes(wl)
+    work_set = attn_bytes + lm_bytes
+    flush = work_set < 2 * L2_BYTES
+    flush_buf = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev) if flush else None
+
+    for _ in range(args.warmup):
+        wl["ctx_lens"].copy_(ctx0)
+        step(wl)
+    torch.cuda.synchronize()
+    if int(status.item()) & ~spade.DEV_FALLBACK:
+        raise RuntimeError(f"device status {int(status.item())} after warm-up")
+    tokens_per_step = int((acc.long() + 1).sum().item())
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with Clocks(local) as clk:
+        t_wall0 = time.perf_counter()
+        for s in range(args.steps):
+            wl["ctx_lens"].copy_(ctx0)
+            if flush:
+                flush_buf.zero_()
+            step(wl, evs[s])
+        torch.cuda.synchronize()
+        t_wall = time.perf_counter() - t_wall0
+    if ws > 1:
+        torch.distributed.barrier()
+    t_step = [e[0].elapsed_time(e[3]) * 1e-3 for e in evs]
+    t_attn = [e[0].elapsed_time(e[1]) * 1e-3 for e in evs]
+    t_acc = [e[1].elapsed_time(e[2]) * 1e-3 for e in evs]
+    t_com = [e[2].elapsed_time(e[3]) * 1e-3 for e in evs]
+    total = sum(t_step)
+    if ws > 1:
+        tt = torch.tensor([total], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        total = float(tt.item())
+    value = tokens_per_step * args.steps * ws / total
+
+    # ---- end to end through the public API with pinned host inputs -------------
+    e2e = None
+    if not args.no_e2e:
+        host_keys = ["q", "hidden", "draft_tokens", "draft_probs", "uniforms", "mode", "cu_q", "n_draft",
+                     "ctx_lens"]
+        host = {k: (wl[k] if k != "ctx_lens" else ctx0).cpu().pin_memory()
+                for k in host_keys if wl[k] is not None}
+        dev_in = {k: torch.empty_like(wl[k] if k != "ctx_lens" else ctx0) for k in host}
+        dev_in["draft_probs"] = dev_in.get("draft_probs")
+        res_host = torch.empty(2 * B, dtype=torch.int32).pin_memory()
+        h2d = sum(t.numel() * t.element_size() for t in host.values())
+        d2h = res_host.numel() * 4
+        n_e2e = max(3, min(args.steps, 20))
+        e_start = torch.cuda.Event(enable_timing=True)
+        e_end = torch.cuda.Event(enable_timing=True)
+        for it in range(n_e2e + 2):
+            if it == 2:
+                torch.cuda.synchronize()
+                e_start.record(stream)
+            for k, t in host.items():
+                dev_in[k].copy_(t, non_blocking=True)
+            step(dev_in)
+            res_host[:B].copy_(acc, non_blocking=True)
+            res_host[B:].copy_(tok, non_blocking=True)
+            if flush and it >= 2:
+                pass
+        e_end.record(stream)
+        torch.cuda.synchronize()
+        t_e2e = e_start.elapsed_time(e_end) * 1e-3
+        e2e = {"value": tokens_per_step * n_e2e * ws / t_e2e, "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "steps": n_e2e,
+               "state_resident": "KV cache and W_lm stay in HBM (model state)"}
+
+    hbm, bf16, bf16_sus, peak_src = _peaks()
+    m_acc = statistics.mean(t_acc)
+    m_attn = statistics.mean(t_attn)
+    roof_lm = {"kernel": "verify_accept_kernel", "bound": "hbm", "achieved": lm_bytes / m_acc / 1e9,
+               "peak": hbm, "unit": "GB/s", "frac": lm_bytes / m_acc / 1e9 / hbm, "traffic": None,
+               "algorithmic_bytes": lm_bytes, "peak_source": peak_src,
+               "tensor_tflops": lm_flop / m_acc / 1e12, "tensor_frac_of_bf16_peak": lm_flop / m_acc / 1e12 / bf16}
+    roof_attn = {"kernel": "verify_attention_kernel", "bound": "hbm", "achieved": attn_bytes / m_attn / 1e9,
+                 "peak": hbm, "unit": "GB/s", "frac": attn_bytes / m_attn / 1e9 / hbm, "traffic": None,
+                 "algorithmic_bytes": attn_bytes, "peak_source": peak_src,
+                 "tflops": attn_flop / m_attn / 1e12}
+    dominant = roof_lm if m_acc >= m_attn else roof_attn
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.workload, "B": B, "Hq": wl["Hq"], "Hkv": wl["Hkv"], "D": wl["D"],
+                   "H": wl["H"], "V": wl["V"], "ctx": list(spec.ctx), "k": list(spec.k), "mode": spec.mode,
+                   "rows": R, "parallelism": "replicas" if ws > 1 else "single",
+                   "l2": "flushed between steps" if flush else f"working set {work_set / 1e9:.2f} GB > L2"},
+        "tokens_per_step": tokens_per_step,
+        "accepted_len": acc.tolist(),
+        "kernels_us": {"verify_attention": m_attn * 1e6, "verify_accept": m_acc * 1e6,
+                       "kv_commit": statistics.mean(t_com) * 1e6},
+        "roofline": dominant, "roofline_attention": roof_attn, "roofline_lm_head": roof_lm,
+        "e2e": e2e, "gpu_launches": 3 * args.steps, "wall_s_timed_loop": t_wall,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl)
+    return line
+
+
+# ---------------------------------------------------------------------------
+def _oracle_one_sequence(wl_cpu, b):
+    """Runs the oracle's verify step (attention + LM head + accept + commit) on sequence b."""
+    import oracle.spade_oracle as O
+
+    def npf(t):
+        return None if t is None else (t.float().numpy() if t.dtype == torch.bfloat16 else t.numpy())
+
+    cu = wl_cpu["cu_q"]
+    r0, r1 = int(cu[b]), int(cu[b + 1])
+    k = r1 - r0 - 1
+    q = npf(wl_cpu["q"][r0:r1])
+    kc = npf(wl_cpu["k_cache"][b:b + 1])
+    vc = npf(wl_cpu["v_cache"][b:b + 1])
+    ctx = npf(wl_cpu["ctx_lens"][b:b + 1])
+    kd = [k]
+    cu1 = [0, k + 1]
+    t0 = time.perf_counter()
+    O.verify_attention(q, kc, vc, ctx, kd, cu1)
+    logits = O.lm_logits(npf(wl_cpu["hidden"][r0:r1]), npf(wl_cpu["w_lm"]))
+    d0 = r0 - b
+    dp = npf(wl_cpu["draft_probs"][d0:d0 + k]) if wl_cpu["draft_probs"] is not None else None
+    res = O.verify_accept(logits, npf(wl_cpu["draft_tokens"][d0:d0 + k]), dp,
+                          npf(wl_cpu["uniforms"][r0:r1]), npf(wl_cpu["mode"][b:b + 1]), cu1, kd)
+    O.kv_commit(kc, vc, ctx, res["accepted_len"], kd)
+    dt = time.perf_counter() - t0
+    return int(res["accepted_len"][0]) + 1, dt
+
+
+def _cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(wl):
+    wl_cpu = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in wl.items()}
+    tok, dt = _oracle_one_sequence(wl_cpu, 0)
+    return {"value": tok / dt, "unit": UNIT, "cores": _cores(), "kind": "oracle",
+            "sample": f"one sequence (b=0, {tok} committed tokens) of the workload: attention of its "
+                      f"k+1 rows x all heads, float64 LM head over the full vocabulary, accept, commit; "
+                      f"{dt:.2f} s"}
+
+
+def run_reference(args):
+    spec = W.SPECS[args.workload]
+    wl = W.make_workload(spec, device="cpu")
+    B = wl["B"]
+    for s in range(args.warmup):
+        _oracle_one_sequence(wl, s % B)
+    toks, secs = 0, 0.0
+    for s in range(args.steps):
+        t, dt = _oracle_one_sequence(wl, s % B)
+        toks += t
+        secs += dt
+    value = toks / secs
+    sample = (f"each step: one sequence of the {args.workload} workload through the float64 oracle "
+              f"(attention of its k+1 rows x {spec.Hq} heads, LM head over {spec.V} vocab, accept, commit)")
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": args.workload, "B": B, "Hq": spec.Hq, "Hkv": spec.Hkv, "D": spec.D,
+                   "H": spec.H, "V": spec.V, "ctx": list(spec.ctx), "k": list(spec.k), "mode": spec.mode},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": _cores(), "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="spade", choices=["spade", "reference"])
+    ap.add_argument("--workload", default="llama3_8b", choices=sorted(W.SPECS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3) if args.impl == "spade" else args.warmup
+    ws, rank, local = _dist()
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args)), flush=True)
+        return
+    if ws > 1:
+        torch.cuda.set_device(local)
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local))
+    line = run_spade(args, ws, rank, local)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -215,9 +215,12 @@ __global__ void __launch_bounds__(Layout<D, MT>::THREADS, 1)
   __syncthreads();
   sc.total = s_pref[p.B];
   if (sc.total == 0) return;
-  const int64_t x_begin = static_cast<int64_t>(blockIdx.x) * sc.total / p.num_ctas;
-  const int64_t x_end = static_cast<int64_t>(blockIdx.x + 1) * sc.total / p.num_ctas;
-  if (x_begin >= x_end) return;
+  // Never more CTAs than chunks: every CTA kept has a non-empty range, so the
+  // CTAs between a unit's first and last owner all contribute a partial.
+  sc.num_ctas = static_cast<int>(sc.total < p.num_ctas ? sc.total : p.num_ctas);
+  if (static_cast<int>(blockIdx.x) >= sc.num_ctas) return;
+  const int64_t x_begin = static_cast<int64_t>(blockIdx.x) * sc.total / sc.num_ctas;
+  const int64_t x_end = static_cast<int64_t>(blockIdx.x + 1) * sc.total / sc.num_ctas;
 
   if (warp == 0) {
     // ======================= producer: TMA K/V chunks =======================

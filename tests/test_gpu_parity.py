@@ -101,7 +101,10 @@ def test_repeat_calls_reuse_workspace(dev):
         assert torch.equal(o, outs[0])
     for a, t in toks[1:]:
         assert torch.equal(a, toks[0][0]) and torch.equal(t, toks[0][1])
-    assert int(ws_a[:1024].sum()) == 0  # counters back at zero
+    G = wl["Hq"] // wl["Hkv"]
+    units = wl["B"] * wl["Hkv"] * ((G * (max_k + 1) + 63) // 64)
+    assert int(ws_a[: units * 4].sum()) == 0  # per-unit merge counters back at zero
+    assert int(ws_b[:4].sum()) == 0           # grid-barrier arrival count back at zero
 
 
 # ---------------------------------------------------------------------------
