@@ -106,6 +106,30 @@ spade_status spade_verify_attention(const void *q, const void *k_cache, const vo
 size_t spade_attn_workspace_size(int32_t B, int32_t Hq, int32_t Hkv, int32_t D, int32_t cap,
                                  int32_t max_k);
 
+/*
+ * spade_verify_attention_noalloc -- the same attention for callers that cannot
+ * allocate device memory (for example plugin hosts that pass a kernel only its
+ * inputs and outputs, or serving loops whose memory pool is frozen after
+ * start-up).  The paper has no counterpart: this is a deployment variant.
+ *
+ * Arguments are those of spade_verify_attention without the workspace.  The
+ * scratch is a 32 MiB file-scope device array that every GPU loading this
+ * library holds until the process exits; the call allocates nothing.
+ *  - Sizes whose workspace (spade_attn_workspace_size) exceeds 32 MiB are
+ *    rejected with SPADE_ERR_CAPACITY and a message giving both sizes.
+ *  - The first call on each device resolves the array's device address
+ *    (cudaGetSymbolAddress); make that first call before any stream capture.
+ *  - Every call shares the one array and clears its merge counters first
+ *    (cudaMemsetAsync on `stream`): calls that overlap on the GPU, on any
+ *    streams, race and corrupt each other's results.  Order them.
+ */
+spade_status spade_verify_attention_noalloc(const void *q, const void *k_cache,
+                                            const void *v_cache, const int32_t *ctx_lens,
+                                            const int32_t *n_draft, const int32_t *cu_q, void *out,
+                                            float *lse, int32_t B, int32_t Hq, int32_t Hkv,
+                                            int32_t D, int32_t cap, int32_t max_k, int32_t R,
+                                            int32_t *status, spade_stream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* LM head + softmax + accept/reject + residual sampling (Sec. III-A/III-C)  */
 /* ------------------------------------------------------------------------ */

@@ -22,7 +22,7 @@ from . import _build
 
 __all__ = [
     "SpadeError", "load", "build", "library_path",
-    "spade_verify_attention", "spade_verify_accept", "spade_kv_commit",
+    "spade_verify_attention", "spade_verify_accept", "spade_kv_commit", "spade_verify_attention_noalloc",
     "spade_attn_workspace_size", "spade_accept_workspace_size",
     "attn_workspace", "accept_workspace", "status_tensor", "check_status",
     "DEV_BAD_INDEX", "DEV_CAPACITY", "DEV_TIMEOUT", "DEV_FALLBACK",
@@ -71,6 +71,8 @@ def load():
     lib.spade_verify_attention.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                            _i32, _i32, _i32, _i32, _i32, _i32, _i32,
                                            _vp, _sz, _vp, _vp]
+    lib.spade_verify_attention_noalloc.restype = _i32
+    lib.spade_verify_attention_noalloc.argtypes = [_vp] * 8 + [_i32] * 7 + [_vp, _vp]
     lib.spade_attn_workspace_size.restype = _sz
     lib.spade_attn_workspace_size.argtypes = [_i32] * 6
     lib.spade_verify_accept.restype = _i32
@@ -164,6 +166,26 @@ def spade_verify_attention(q, k_cache, v_cache, ctx_lens, n_draft, cu_q, out, ls
         _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(ctx_lens), _ptr(n_draft), _ptr(cu_q), _ptr(out),
         _ptr(lse), B, Hq, Hkv, D, cap, int(max_k), R, _ptr(workspace), workspace.numel(),
         _ptr(status), _stream(stream))
+    _check_rc(rc)
+    return out
+
+
+def spade_verify_attention_noalloc(q, k_cache, v_cache, ctx_lens, n_draft, cu_q, out, lse=None, *,
+                                   max_k, status, stream=None):
+    """spade_verify_attention for callers that cannot allocate: scratch in a static device array.
+
+    Calls that overlap on the GPU share that array and race; the first call on
+    a device resolves the array's address and should precede any stream capture.
+    """
+    R, Hq, D = q.shape
+    B, Hkv, cap, _ = k_cache.shape
+    for t, n in ((q, "q"), (k_cache, "k_cache"), (v_cache, "v_cache"), (out, "out")):
+        _need(t, n, torch.bfloat16)
+    for t, n in ((ctx_lens, "ctx_lens"), (n_draft, "n_draft"), (cu_q, "cu_q"), (status, "status")):
+        _need(t, n, torch.int32, 1)
+    rc = load().spade_verify_attention_noalloc(
+        _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(ctx_lens), _ptr(n_draft), _ptr(cu_q), _ptr(out),
+        _ptr(lse), B, Hq, Hkv, D, cap, int(max_k), R, _ptr(status), _stream(stream))
     _check_rc(rc)
     return out
 

@@ -21,6 +21,7 @@
 #include <cuda_bf16.h>
 
 #include <cfloat>
+#include <mutex>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -694,4 +695,72 @@ extern "C" spade_status spade_verify_attention(
   }
   if (e != cudaSuccess) return cuda_fail(e, "verify_attention launch");
   return SPADE_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant.  Some callers cannot allocate device memory at all:
+// plugin hosts that hand a kernel only its input and output buffers, or
+// serving loops that freeze their memory pool after start-up.  For them the
+// attention's scratch (merge counters and split partials) lives in a
+// file-scope device array instead of a caller-provided workspace.  The array
+// is reserved on every GPU that loads this library, until the process exits.
+namespace spade {
+namespace attn_noalloc {
+
+constexpr size_t kScratchBytes = size_t(32) << 20;  // 32 MiB
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) uint8_t g_scratch[kScratchBytes];
+
+static std::mutex g_mu;
+static void *g_ptr[kMaxDevices];  // device address of g_scratch, per device
+
+// Host code must not pass `g_scratch` itself to a kernel: on the host that
+// name is a stand-in, not a device address.  Resolve it once per device.
+static spade_status scratch_address(int dev, void **out) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_ptr[dev]) {
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(attention scratch)");
+    g_ptr[dev] = p;
+  }
+  *out = g_ptr[dev];
+  return SPADE_OK;
+}
+
+}  // namespace attn_noalloc
+}  // namespace spade
+
+extern "C" spade_status spade_verify_attention_noalloc(
+    const void *q, const void *k_cache, const void *v_cache, const int32_t *ctx_lens,
+    const int32_t *n_draft, const int32_t *cu_q, void *out, float *lse, int32_t B, int32_t Hq,
+    int32_t Hkv, int32_t D, int32_t cap, int32_t max_k, int32_t R, int32_t *status,
+    spade_stream_t stream) {
+  using namespace attn_noalloc;
+  if (B <= 0 || Hq <= 0 || Hkv <= 0 || cap <= 0 || max_k < 0 || R <= 0 || Hq % Hkv ||
+      (D != 64 && D != 128))
+    return fail(SPADE_ERR_INVALID_ARG, "spade_verify_attention_noalloc: bad sizes");
+  int dev = 0;
+  spade_status st = device_info(nullptr, &dev);
+  if (st != SPADE_OK) return st;
+  if (dev >= kMaxDevices) return fail(SPADE_ERR_UNSUPPORTED_DEVICE, "device %d", dev);
+  const size_t need = spade_attn_workspace_size(B, Hq, Hkv, D, cap, max_k);
+  if (need == 0) return fail(SPADE_ERR_INVALID_ARG, "spade_verify_attention_noalloc: bad sizes");
+  if (need > kScratchBytes)
+    return fail(SPADE_ERR_CAPACITY,
+                "spade_verify_attention_noalloc: these sizes need %zu bytes of scratch; the static "
+                "scratch holds %zu bytes (use spade_verify_attention with a workspace)",
+                need, kScratchBytes);
+  void *scratch = nullptr;
+  st = scratch_address(dev, &scratch);
+  if (st != SPADE_OK) return st;
+  // The merge counters must start at zero; the array keeps whatever the last
+  // call (possibly an interrupted one) left there.
+  const size_t units = static_cast<size_t>(B) * Hkv * attn::row_blocks(Hq / Hkv, max_k);
+  const cudaError_t e = cudaMemsetAsync(scratch, 0, round_up(units * 4, 256),
+                                        reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync(attention scratch counters)");
+  return spade_verify_attention(q, k_cache, v_cache, ctx_lens, n_draft, cu_q, out, lse, B, Hq, Hkv,
+                                D, cap, max_k, R, scratch, kScratchBytes, status, stream);
 }
