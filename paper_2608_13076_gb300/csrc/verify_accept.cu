@@ -9,21 +9,23 @@
 //    The vocabulary is the M side of the MMA (128 vocab rows per tile) and the
 //    R verify rows are the N side, so W -- the only large operand -- streams
 //    from HBM exactly once while the few hidden rows are re-read from L2.
+//  * W and hidden arrive by TMA in 32 KB boxes: a 3-D view of the row-major
+//    matrix fetches 128 rows x 2 k-chunks at once and lands them as two
+//    canonical 128B-swizzled K-major tiles (a 2-D view covers a ragged tail).
 //  * One CTA per SM (cooperative launch) owns a contiguous vocabulary slice.
 //    All its tiles' logits stay resident in TMEM (512 columns x 128 lanes);
-//    when the padded MMA width does not leave room for every tile, finished
-//    tiles are compacted to the exact row count and the next round of tiles
-//    accumulates in the freed columns.  Logits never reach HBM.
-//  * Warp roles: warp 0 issues TMA loads of W and hidden chunks (128-byte
-//    swizzle) into mbarrier rings, warp 1 owns TMEM and issues the MMAs from a
-//    single thread, warps 2-5 read accumulators back (tcgen05.ld) and reduce
-//    per-row max / sum-exp / argmax across the vocabulary with warp shuffles.
+//    finished tiles are compacted from the padded MMA width to the row count,
+//    which frees columns for the next round of tiles.  Logits never reach HBM.
+//  * Warp roles: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
+//    MMAs from a single thread, warps 2-5 read accumulators back (tcgen05.ld)
+//    and reduce per-row max / sum-exp / argmax across the vocabulary (an
+//    8-row shared-memory transpose, then a 4-lane shuffle merge).
 //  * Two bounded device-wide barriers: after the first every CTA merges the
 //    per-slice statistics into p(d) and argmax for every row and takes the
 //    accept decisions; after the second the slice masses of the distribution
 //    to sample (residual or p, fp64) are known, and the CTA whose slice holds
-//    the point u*Z scans its resident logits in vocabulary order to pick the
-//    token.
+//    the point u*Z locates its 32-entry segment and scans it in vocabulary
+//    order to pick the token.
 #include <cuda_bf16.h>
 
 #include <cfloat>
@@ -35,14 +37,17 @@ namespace spade {
 namespace accept {
 
 constexpr int kTileV = 128;    // vocab rows per tile (MMA M)
-constexpr int kKChunk = 64;    // K elements per TMA box row (128 bytes)
+constexpr int kKChunk = 64;    // K elements per 128-byte swizzle row
 constexpr int kEpiWarps = 4;
 constexpr int kThreads = 32 * (2 + kEpiWarps);
 constexpr int kMaxR = 256;     // verify rows per call on the resident path (MMA N <= 256)
+constexpr int kMaxB = 256;
 constexpr int kMaxRounds = 8;
+constexpr int kMaxTilesPerCta = 32;
 constexpr int kTmemCols = 512;
 constexpr int kSmemBudget = 216 * 1024;
-constexpr int kWSlotBytes = kTileV * kKChunk * 2;  // 16 KB
+constexpr int kWChunkBytes = kTileV * kKChunk * 2;  // 16 KB: one tile x one k-chunk
+constexpr float kLog2e = 1.4426950408889634f;
 
 struct Params {
   const int32_t *draft_tokens;
@@ -58,7 +63,12 @@ struct Params {
   float4 *pstat;     // [NC][R]: slice max, slice sum-exp, slice argmax (bits), -
   float *ldraft;     // [R]: logit of the row's draft token
   double2 *zpart;    // [NC][B]: slice mass of the distribution to sample, of p
-  int B, R, H, V, T, NC, Ncols, Rs, KC, nrounds;
+  int B, R, H, V, T, NC, Ncols, Rs;
+  int KC;            // k-chunks of 64 (the last may be partial)
+  int KCF;           // full k-chunks (H / 64)
+  int KG;            // k-chunks per pipeline stage
+  int NS;            // pipeline stages per tile pass = ceil(KC / KG)
+  int nrounds;
   int round_tiles[kMaxRounds];
   int HS, WS;        // hidden / W ring slots
   uint32_t idesc;
@@ -66,17 +76,21 @@ struct Params {
 };
 
 struct Smem {
-  int off_h, off_bar, off_misc, off_draft, off_wst, total;
+  int w_slot, h_slot;
+  int off_h, off_bar, off_misc, off_rows, off_wst, off_tbuf, total;
 };
 
 __host__ __device__ inline Smem smem_layout(const Params &p) {
   Smem s;
-  s.off_h = p.WS * kWSlotBytes;
-  s.off_bar = s.off_h + p.HS * p.Ncols * 128;
+  s.w_slot = p.KG * kWChunkBytes;
+  s.h_slot = p.KG * p.Ncols * 128;
+  s.off_h = p.WS * s.w_slot;
+  s.off_bar = s.off_h + p.HS * s.h_slot;
   s.off_misc = s.off_bar + (2 * p.WS + 2 * p.HS + 2) * 8;
-  s.off_draft = s.off_misc + 64;
-  s.off_wst = s.off_draft + kMaxR * 4;
-  s.total = s.off_wst + kEpiWarps * kMaxR * 16 + 1024;
+  s.off_rows = s.off_misc + 64;                     // int [3][kMaxR]: draft, seq, pos
+  s.off_wst = s.off_rows + 3 * kMaxR * 4;           // float4 [kEpiWarps][kMaxR]
+  s.off_tbuf = s.off_wst + kEpiWarps * kMaxR * 16;  // float [kEpiWarps][16][32]
+  s.total = s.off_tbuf + kEpiWarps * 16 * 32 * 4 + 1024;
   return s;
 }
 
@@ -88,6 +102,15 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned *p) {
   unsigned v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
+}
+
+__device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, int32_t x,
+                                            int32_t y, int32_t z, uint64_t *bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "l"(pol)
+      : "memory");
 }
 
 // Device-wide barrier among the NC co-resident CTAs (cooperative launch).  The
@@ -117,9 +140,16 @@ __device__ bool grid_barrier(unsigned *bar, int nctas) {
   return s_ok != 0;
 }
 
-// (max, argmax) merge with the lowest index winning ties.
-__device__ __forceinline__ void argmax_merge(float &m, int &i, float om, int oi) {
-  if (om > m || (om == m && oi < i)) { m = om; i = oi; }
+// Merge of (max, sum of exp(x - max), argmax) summaries; lowest index wins ties.
+__device__ __forceinline__ void stat_merge(float &m, float &s, int &i, float om, float os, int oi) {
+  const float M = fmaxf(m, om);
+  if (M == -INFINITY) {
+    s = 0.f;
+  } else {
+    s = s * ex2((m - M) * kLog2e) + os * ex2((om - M) * kLog2e);
+  }
+  if (om > m || (om == m && oi < i)) i = oi;
+  m = M;
 }
 
 __device__ __forceinline__ double warp_sum_d(double v) {
@@ -128,9 +158,55 @@ __device__ __forceinline__ double warp_sum_d(double v) {
   return v;
 }
 
+// Per-row running statistics of one epilogue warp: the 8 rows c8*8..c8*8+7 of
+// the 32 vocab entries held in registers by the warp's lanes.
+__device__ __forceinline__ void reduce_rows8(const uint32_t *raw, int c8, int vlane0, int lane,
+                                             const Params &p, const int32_t *s_draft,
+                                             float *tbuf, float4 *wst) {
+#pragma unroll
+  for (int e = 0; e < 8; ++e) tbuf[e * 32 + lane] = __uint_as_float(raw[e]);
+  __syncwarp();
+  const int r = lane >> 2, part = lane & 3;
+  const int n = c8 * 8 + r;
+  const float4 lo = *reinterpret_cast<const float4 *>(tbuf + r * 32 + part * 8);
+  const float4 hi = *reinterpret_cast<const float4 *>(tbuf + r * 32 + part * 8 + 4);
+  float x[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+  const int v0 = vlane0 + part * 8;  // vocab id of x[0]
+  const int d = (n < p.R) ? s_draft[n] : -1;
+  float m = -INFINITY;
+  int mi = INT_MAX;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    if (v0 + i >= p.V) x[i] = -INFINITY;
+    if (v0 + i == d) p.ldraft[n] = x[i];
+    if (x[i] > m) { m = x[i]; mi = v0 + i; }
+  }
+  float s = 0.f;
+  if (m != -INFINITY) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s += ex2((x[i] - m) * kLog2e);
+  }
+#pragma unroll
+  for (int o = 1; o <= 2; o <<= 1) {
+    const float om = __shfl_xor_sync(0xffffffffu, m, o);
+    const float os = __shfl_xor_sync(0xffffffffu, s, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, mi, o);
+    stat_merge(m, s, mi, om, os, oi);
+  }
+  __syncwarp();
+  if (part == 0 && n < p.R) {
+    float4 st = wst[n];
+    int si = __float_as_int(st.z);
+    stat_merge(st.x, st.y, si, m, s, mi);
+    st.z = __int_as_float(si);
+    wst[n] = st;
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
-    const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tm_w,
-    const __grid_constant__ CUtensorMap tm_h) {
+    const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tm_w3,
+    const __grid_constant__ CUtensorMap tm_w2, const __grid_constant__ CUtensorMap tm_h3,
+    const __grid_constant__ CUtensorMap tm_h2) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -146,8 +222,11 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L.off_misc);
   uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + L.off_misc + 8);
   int *s_any_stoch = reinterpret_cast<int *>(smem + L.off_misc + 16);
-  int32_t *s_draft = reinterpret_cast<int32_t *>(smem + L.off_draft);
+  int32_t *s_draft = reinterpret_cast<int32_t *>(smem + L.off_rows);
+  int32_t *s_seq = s_draft + kMaxR;
+  int32_t *s_pos = s_seq + kMaxR;
   float4 *s_wst = reinterpret_cast<float4 *>(smem + L.off_wst);
+  float *s_tbuf = reinterpret_cast<float *>(smem + L.off_tbuf);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c = blockIdx.x;
@@ -155,7 +234,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   const int t_hi = static_cast<int>(static_cast<int64_t>(c + 1) * p.T / p.NC);
   const int ntiles = t_hi - t_lo;
 
-  // ---- set-up: barriers, TMEM, per-row draft tokens ------------------------
+  // ---- set-up: barriers, TMEM, per-row bookkeeping -------------------------
   if (tid == 0) {
     *s_abort = 0;
     *s_any_stoch = 0;
@@ -169,16 +248,20 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     tmem_alloc(s_tmem, p.tmem_cols);
     tmem_relinquish();
   }
-  for (int n = tid; n < kMaxR; n += kThreads) s_draft[n] = -1;
+  for (int n = tid; n < kMaxR; n += kThreads) { s_draft[n] = -1; s_seq[n] = -1; s_pos[n] = 0; }
   __syncthreads();
-  // Row n = cu_q[b] + i holds draft i of sequence b for i < k_b.
+  // Row n = cu_q[b] + i is position i of sequence b; it holds draft i for i < k_b.
   for (int b = tid; b < p.B; b += kThreads) {
     const int r0 = p.cu_q[b], k = p.n_draft[b], r1 = p.cu_q[b + 1];
     if (r0 < 0 || k < 0 || r1 - r0 != k + 1 || r1 > p.R) {
       atomicOr(p.status, SPADE_DEV_BAD_INDEX);
       continue;
     }
-    for (int i = 0; i < k; ++i) s_draft[r0 + i] = p.draft_tokens[r0 - b + i];
+    for (int i = 0; i <= k; ++i) {
+      s_seq[r0 + i] = b;
+      s_pos[r0 + i] = i;
+      if (i < k) s_draft[r0 + i] = p.draft_tokens[r0 - b + i];
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -189,21 +272,30 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   // ======================= phase A: logits + slice statistics =============
   if (warp == 0) {
     if (lane == 0 && ntiles > 0) {
-      tma_prefetch_desc(&tm_w);
-      tma_prefetch_desc(&tm_h);
+      tma_prefetch_desc(&tm_w3);
+      tma_prefetch_desc(&tm_h3);
       const uint64_t pol_w = l2_policy_evict_first();
       const uint64_t pol_h = l2_policy_evict_last();
       uint32_t wi = 0, hi = 0, w_issued = 0, h_issued = 0;
       int tdone = 0;
       for (int r = 0; r < p.nrounds && tdone < ntiles; ++r) {
         const int nt = min(p.round_tiles[r], ntiles - tdone);
-        for (int kc = 0; kc < p.KC; ++kc) {
+        for (int ks = 0; ks < p.NS; ++ks) {
+          const int c0 = ks * p.KG;
+          const int nch = min(p.KG, p.KC - c0);
+          const bool box3 = (nch == p.KG) && (c0 + p.KG <= p.KCF);
           {
             const int s = hi % p.HS;
             mbar_wait(&h_empty[s], ((hi / p.HS) & 1) ^ 1, s_abort);
             if (!*s_abort) {
-              mbar_arrive_expect_tx(&h_full[s], p.Ncols * 128);
-              tma_load_2d(h_ring + s * p.Ncols * 128, &tm_h, kc * kKChunk, 0, &h_full[s], pol_h);
+              uint8_t *dst = h_ring + s * L.h_slot;
+              mbar_arrive_expect_tx(&h_full[s], nch * p.Ncols * 128);
+              if (box3) {
+                tma_load_3d(dst, &tm_h3, 0, 0, c0, &h_full[s], pol_h);
+              } else {
+                for (int j = 0; j < nch; ++j)
+                  tma_load_2d(dst + j * p.Ncols * 128, &tm_h2, (c0 + j) * kKChunk, 0, &h_full[s], pol_h);
+              }
               h_issued = hi + 1;
             }
             ++hi;
@@ -212,9 +304,15 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             const int s = wi % p.WS;
             mbar_wait(&w_empty[s], ((wi / p.WS) & 1) ^ 1, s_abort);
             if (!*s_abort) {
-              mbar_arrive_expect_tx(&w_full[s], kWSlotBytes);
-              tma_load_2d(w_ring + s * kWSlotBytes, &tm_w, kc * kKChunk,
-                          (t_lo + tdone + j) * kTileV, &w_full[s], pol_w);
+              uint8_t *dst = w_ring + s * L.w_slot;
+              const int row0 = (t_lo + tdone + j) * kTileV;
+              mbar_arrive_expect_tx(&w_full[s], nch * kWChunkBytes);
+              if (box3) {
+                tma_load_3d(dst, &tm_w3, 0, row0, c0, &w_full[s], pol_w);
+              } else {
+                for (int jj = 0; jj < nch; ++jj)
+                  tma_load_2d(dst + jj * kWChunkBytes, &tm_w2, (c0 + jj) * kKChunk, row0, &w_full[s], pol_w);
+              }
               w_issued = wi + 1;
             }
             ++wi;
@@ -234,26 +332,29 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     if (lane == 0 && ntiles > 0) {
       uint32_t wi = 0, hi = 0;
       int tdone = 0, used = 0;
-      rounds_issued = 0;
       for (int r = 0; r < p.nrounds && tdone < ntiles; ++r) {
         const int nt = min(p.round_tiles[r], ntiles - tdone);
         if (r > 0) mbar_wait(acc_empty, (r - 1) & 1, s_abort);
         tc_fence_after();
-        for (int kc = 0; kc < p.KC; ++kc) {
+        for (int ks = 0; ks < p.NS; ++ks) {
+          const int nch = min(p.KG, p.KC - ks * p.KG);
           const int hs = hi % p.HS;
           mbar_wait(&h_full[hs], (hi / p.HS) & 1, s_abort);
           tc_fence_after();
-          const uint32_t h_addr = smem_u32(h_ring + hs * p.Ncols * 128);
+          const uint32_t h_addr = smem_u32(h_ring + hs * L.h_slot);
           for (int j = 0; j < nt; ++j) {
             const int ws = wi % p.WS;
             mbar_wait(&w_full[ws], (wi / p.WS) & 1, s_abort);
             tc_fence_after();
-            const uint32_t w_addr = smem_u32(w_ring + ws * kWSlotBytes);
+            const uint32_t w_addr = smem_u32(w_ring + ws * L.w_slot);
             const uint32_t d_tmem = tmem + static_cast<uint32_t>(used + j * p.Ncols);
+            for (int jj = 0; jj < nch; ++jj) {
 #pragma unroll
-            for (int k16 = 0; k16 < kKChunk / 16; ++k16) {
-              tc_mma_f16(d_tmem, smem_desc_sw128(w_addr + 32 * k16),
-                         smem_desc_sw128(h_addr + 32 * k16), p.idesc, (kc | k16) != 0);
+              for (int k16 = 0; k16 < kKChunk / 16; ++k16) {
+                tc_mma_f16(d_tmem, smem_desc_sw128(w_addr + jj * kWChunkBytes + 32 * k16),
+                           smem_desc_sw128(h_addr + jj * p.Ncols * 128 + 32 * k16), p.idesc,
+                           (ks | jj | k16) != 0);
+              }
             }
             tc_commit(&w_empty[ws]);
             ++wi;
@@ -268,11 +369,12 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       }
     }
   } else {
-    // ---- epilogue warps: slice statistics per row, compaction -----------
+    // ---- epilogue warps: compaction, then slice statistics per row -------
     const int ew = warp - 2;             // 0..3
     const int q4 = warp & 3;             // TMEM lane quarter this warp may access
     const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
     float4 *wst = s_wst + ew * kMaxR;    // this warp's running stats per row
+    float *tbuf = s_tbuf + ew * 16 * 32;
     for (int n = lane; n < p.R; n += 32) wst[n] = make_float4(-INFINITY, 0.f, __int_as_float(INT_MAX), 0.f);
     __syncwarp();
     int tdone = 0, used = 0;
@@ -280,47 +382,9 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       const int nt = min(p.round_tiles[r], ntiles - tdone);
       if (!mbar_wait(acc_full, r & 1, s_abort)) atomicOr(p.status, SPADE_DEV_TIMEOUT);
       tc_fence_after();
-      for (int j = 0; j < nt; ++j) {
-        const int v = (t_lo + tdone + j) * kTileV + q4 * 32 + lane;
-        const bool valid = v < p.V;
-        const uint32_t col0 = tmem + lane_base + static_cast<uint32_t>(used + j * p.Ncols);
-        for (int c8 = 0; c8 * 8 < p.R; ++c8) {
-          uint32_t raw[8];
-          tmem_ld8(col0 + c8 * 8, raw);
-          tmem_wait_ld();
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const int n = c8 * 8 + e;
-            if (n < p.R) {
-              const float x = valid ? __uint_as_float(raw[e]) : -INFINITY;
-              if (valid && s_draft[n] == v) p.ldraft[n] = x;
-              float mv = x;
-              int mi = v;
-#pragma unroll
-              for (int o = 16; o > 0; o >>= 1)
-                argmax_merge(mv, mi, __shfl_xor_sync(0xffffffffu, mv, o),
-                             __shfl_xor_sync(0xffffffffu, mi, o));
-              float ev = (x == -INFINITY) ? 0.f : ex2((x - mv) * 1.4426950408889634f);
-#pragma unroll
-              for (int o = 16; o > 0; o >>= 1) ev += __shfl_xor_sync(0xffffffffu, ev, o);
-              if (lane == (n & 31)) {
-                float4 st = wst[n];
-                const float M = fmaxf(st.x, mv);
-                if (M != -INFINITY) {
-                  st.y = st.y * ex2((st.x - M) * 1.4426950408889634f) +
-                         ev * ex2((mv - M) * 1.4426950408889634f);
-                }
-                int si = __float_as_int(st.z);
-                argmax_merge(st.x, si, mv, mi);
-                st.x = M;
-                st.z = __int_as_float(si);
-                wst[n] = st;
-              }
-            }
-          }
-        }
-      }
-      // Compaction: move this round's tiles from stride Ncols to stride Rs.
+      // Compaction: this round's tiles move from stride Ncols to stride Rs, so
+      // tile t of the slice ends at column t * Rs and the next round's MMAs
+      // may start at once in the columns after it.
       if (p.Ncols != p.Rs) {
         for (int j = 0; j < nt; ++j) {
           const uint32_t src = tmem + lane_base + static_cast<uint32_t>(used + j * p.Ncols);
@@ -338,6 +402,26 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(acc_empty);
+      for (int j = 0; j < nt; ++j) {
+        const int t = tdone + j;
+        const int vlane0 = (t_lo + t) * kTileV + q4 * 32;  // vocab id of lane 0's row
+        const uint32_t col = tmem + lane_base + static_cast<uint32_t>(t * p.Rs);
+        int c8 = 0;
+        for (; (c8 + 1) * 8 < p.R; c8 += 2) {
+          uint32_t raw[16];
+          tmem_ld8(col + c8 * 8, raw);
+          tmem_ld8(col + c8 * 8 + 8, raw + 8);
+          tmem_wait_ld();
+          reduce_rows8(raw, c8, vlane0, lane, p, s_draft, tbuf, wst);
+          reduce_rows8(raw + 8, c8 + 1, vlane0, lane, p, s_draft, tbuf + 256, wst);
+        }
+        if (c8 * 8 < p.R) {
+          uint32_t raw[8];
+          tmem_ld8(col + c8 * 8, raw);
+          tmem_wait_ld();
+          reduce_rows8(raw, c8, vlane0, lane, p, s_draft, tbuf, wst);
+        }
+      }
       used += nt * p.Rs;
       tdone += nt;
     }
@@ -348,13 +432,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       int idx = INT_MAX;
       for (int w = 0; w < kEpiWarps; ++w) {
         const float4 st = s_wst[w * kMaxR + n];
-        const float M = fmaxf(m, st.x);
-        if (M != -INFINITY)
-          s = s * ex2((m - M) * 1.4426950408889634f) + st.y * ex2((st.x - M) * 1.4426950408889634f);
-        int i2 = idx;
-        argmax_merge(m, i2, st.x, __float_as_int(st.z));
-        m = M;
-        idx = i2;
+        stat_merge(m, s, idx, st.x, st.y, __float_as_int(st.z));
       }
       __stcg(&p.pstat[static_cast<size_t>(c) * p.R + n], make_float4(m, s, __int_as_float(idx), 0.f));
     }
@@ -370,111 +448,126 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   float *g_m = reinterpret_cast<float *>(w_ring);           // [R]
   float *g_s = g_m + kMaxR;                                 // [R]
   int *g_arg = reinterpret_cast<int *>(g_s + kMaxR);        // [R]
-  int *s_acc = g_arg + kMaxR;                               // [B]
-  int *s_rstar = s_acc + kMaxR;                             // [B]
-  int *s_owner = s_rstar + kMaxR;                           // [B]
-  int *s_usep = s_owner + kMaxR;                            // [B]
-  double *s_T = reinterpret_cast<double *>(s_usep + kMaxR); // [B]
-  double *s_red = s_T + kMaxR;                              // [kEpiWarps * 2]
+  int *s_ok = g_arg + kMaxR;                                // [R]
+  int *s_acc = s_ok + kMaxR;                                // [B]
+  int *s_rstar = s_acc + kMaxB;                             // [B]
+  int *s_owner = s_rstar + kMaxB;                           // [B]
+  int *s_usep = s_owner + kMaxB;                            // [B]
+  int *s_stoch = s_usep + kMaxB;                            // [B]
+  int *s_seg = s_stoch + kMaxB;                             // [2]: tile, quarter
+  double *s_T = reinterpret_cast<double *>(s_seg + 16);     // [B]
+  double *s_zw = s_T + kMaxB;                               // [B][kEpiWarps][2]
+  double *s_tw = s_zw + kMaxB * kEpiWarps * 2;              // [kMaxTilesPerCta][kEpiWarps]
+
   for (int n = warp; n < p.R; n += kThreads / 32) {
     float m = -INFINITY, s = 0.f;
     int idx = INT_MAX;
+#pragma unroll 4
     for (int cc = lane; cc < p.NC; cc += 32) {
       const float4 st = __ldcg(&p.pstat[static_cast<size_t>(cc) * p.R + n]);
-      const float M = fmaxf(m, st.x);
-      if (M != -INFINITY) s = s * expf(m - M) + st.y * expf(st.x - M);
-      int i2 = idx;
-      argmax_merge(m, i2, st.x, __float_as_int(st.z));
-      m = M;
-      idx = i2;
+      stat_merge(m, s, idx, st.x, st.y, __float_as_int(st.z));
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const float om = __shfl_xor_sync(0xffffffffu, m, o);
       const float os = __shfl_xor_sync(0xffffffffu, s, o);
       const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
-      const float M = fmaxf(m, om);
-      if (M != -INFINITY) s = s * expf(m - M) + os * expf(om - M);
-      int i2 = idx;
-      argmax_merge(m, i2, om, oi);
-      m = M;
-      idx = i2;
+      stat_merge(m, s, idx, om, os, oi);
     }
     if (lane == 0) { g_m[n] = m; g_s[n] = s; g_arg[n] = idx; }
+  }
+  for (int b = tid; b < p.B; b += kThreads) {
+    const int md = p.mode[b];
+    if (md != 0 && md != 1 && c == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
+    s_stoch[b] = (md == 1) && p.draft_probs != nullptr;
+  }
+  __syncthreads();
+  // Accept test of every draft row, all rows at once (the tests are independent;
+  // only the count of leading accepts depends on their order).
+  for (int n = tid; n < p.R; n += kThreads) {
+    const int b = s_seq[n];
+    int ok = 0;
+    if (b >= 0 && s_pos[n] < p.n_draft[b]) {
+      const int d = s_draft[n];
+      if (d < 0 || d >= p.V) {
+        if (c == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
+      } else if (!s_stoch[b]) {
+        ok = (d == g_arg[n]);
+      } else {
+        const float pd = expf(__ldcg(&p.ldraft[n]) - g_m[n]) / g_s[n];
+        const float qd = p.draft_probs[static_cast<size_t>(n - b) * p.V + d];
+        ok = (qd > 0.f) ? (p.uniforms[n] < pd / qd) : (pd > 0.f);
+      }
+    }
+    s_ok[n] = ok;
   }
   __syncthreads();
   for (int b = tid; b < p.B; b += kThreads) {
     const int r0 = p.cu_q[b], k = p.n_draft[b];
-    const int md = p.mode[b];
-    if (md != 0 && md != 1 && c == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
-    const bool stoch = (md == 1) && p.draft_probs != nullptr;
-    int a = 0;
+    int a = -1;
     if (r0 >= 0 && k >= 0 && p.cu_q[b + 1] - r0 == k + 1 && p.cu_q[b + 1] <= p.R) {
-      for (; a < k; ++a) {
-        const int n = r0 + a;
-        const int d = p.draft_tokens[r0 - b + a];
-        bool ok;
-        if (d < 0 || d >= p.V) {
-          if (c == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
-          ok = false;
-        } else if (!stoch) {
-          ok = (d == g_arg[n]);
-        } else {
-          const float pd = expf(__ldcg(&p.ldraft[n]) - g_m[n]) / g_s[n];
-          const float qd = p.draft_probs[static_cast<size_t>(r0 - b + a) * p.V + d];
-          ok = (qd > 0.f) ? (p.uniforms[n] < pd / qd) : (pd > 0.f);
-        }
-        if (!ok) break;
-      }
-    } else {
-      a = -1;
+      a = 0;
+      while (a < k && s_ok[r0 + a]) ++a;
     }
     s_acc[b] = a;
     s_rstar[b] = (a >= 0) ? r0 + a : -1;
-    if (a >= 0 && stoch) atomicOr(s_any_stoch, 1);
+    if (a < 0) s_stoch[b] = 0;
+    if (s_stoch[b]) atomicOr(s_any_stoch, 1);
     if (c == 0) {
       p.accepted_len[b] = a < 0 ? 0 : a;
       if (a < 0) p.next_token[b] = -1;
-      else if (!stoch) p.next_token[b] = g_arg[r0 + a];
+      else if (!s_stoch[b]) p.next_token[b] = g_arg[r0 + a];
     }
   }
   __syncthreads();
 
   if (*s_any_stoch) {
     // =================== phase C: slice masses of the sampled distribution ==
-    for (int b = 0; b < p.B; ++b) {
-      const bool stoch = (p.mode[b] == 1) && p.draft_probs != nullptr && s_acc[b] >= 0;
-      if (!stoch) continue;
-      if (warp >= 2) {
-        const int ew = warp - 2, q4 = warp & 3;
-        const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
+    if (warp >= 2) {
+      const int ew = warp - 2, q4 = warp & 3;
+      const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
+      for (int b = 0; b < p.B; ++b) {
+        if (!s_stoch[b]) continue;
         const int n = s_rstar[b];
         const int a = s_acc[b], k = p.n_draft[b];
-        const float *qrow = (a < k) ? p.draft_probs + static_cast<size_t>(p.cu_q[b] - b + a) * p.V : nullptr;
+        const float *qrow = (a < k) ? p.draft_probs + static_cast<size_t>(n - b) * p.V : nullptr;
         const float M = g_m[n], invS = 1.f / g_s[n];
         double z = 0.0, zp = 0.0;
-        for (int j = 0; j < ntiles; ++j) {
-          const int v = (t_lo + j) * kTileV + q4 * 32 + lane;
-          uint32_t raw;
-          tmem_ld1(tmem + lane_base + static_cast<uint32_t>(j * p.Rs + n), raw);
+        for (int j0 = 0; j0 < ntiles; j0 += 8) {
+          const int nj = min(8, ntiles - j0);
+          uint32_t raw[8];
+          float qv[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            if (j < nj) tmem_ld1(tmem + lane_base + static_cast<uint32_t>((j0 + j) * p.Rs + n), raw[j]);
+          }
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int v = (t_lo + j0 + j) * kTileV + q4 * 32 + lane;
+            qv[j] = (j < nj && qrow && v < p.V) ? qrow[v] : 0.f;
+          }
           tmem_wait_ld();
-          if (v < p.V) {
-            const double pv = static_cast<double>(expf(__uint_as_float(raw) - M) * invS);
-            zp += pv;
-            z += qrow ? fmax(0.0, pv - static_cast<double>(qrow[v])) : pv;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int v = (t_lo + j0 + j) * kTileV + q4 * 32 + lane;
+            if (j < nj && v < p.V) {
+              const double pv = static_cast<double>(expf(__uint_as_float(raw[j]) - M) * invS);
+              zp += pv;
+              z += qrow ? fmax(0.0, pv - static_cast<double>(qv[j])) : pv;
+            }
           }
         }
         z = warp_sum_d(z);
         zp = warp_sum_d(zp);
-        if (lane == 0) { s_red[ew * 2] = z; s_red[ew * 2 + 1] = zp; }
-        named_bar(1, kEpiWarps * 32);
-        if (ew == 0 && lane == 0) {
-          double zs = 0.0, zps = 0.0;
-          for (int w = 0; w < kEpiWarps; ++w) { zs += s_red[w * 2]; zps += s_red[w * 2 + 1]; }
-          __stcg(&p.zpart[static_cast<size_t>(c) * p.B + b], make_double2(zs, zps));
-        }
-        named_bar(1, kEpiWarps * 32);
+        if (lane == 0) { s_zw[(b * kEpiWarps + ew) * 2] = z; s_zw[(b * kEpiWarps + ew) * 2 + 1] = zp; }
       }
+    }
+    __syncthreads();
+    for (int b = tid; b < p.B; b += kThreads) {
+      if (!s_stoch[b]) continue;
+      double zs = 0.0, zps = 0.0;
+      for (int w = 0; w < kEpiWarps; ++w) { zs += s_zw[(b * kEpiWarps + w) * 2]; zps += s_zw[(b * kEpiWarps + w) * 2 + 1]; }
+      __stcg(&p.zpart[static_cast<size_t>(c) * p.B + b], make_double2(zs, zps));
     }
     if (!grid_barrier(p.bar, p.NC)) {
       atomicOr(p.status, SPADE_DEV_TIMEOUT);
@@ -482,8 +575,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     }
     // =================== phase D: owner slice of u*Z, in-slice scan =========
     for (int b = warp; b < p.B; b += kThreads / 32) {
-      const bool stoch = (p.mode[b] == 1) && p.draft_probs != nullptr && s_acc[b] >= 0;
-      if (!stoch) { if (lane == 0) s_owner[b] = -1; continue; }
+      if (!s_stoch[b]) { if (lane == 0) s_owner[b] = -1; continue; }
       double tot = 0.0, totp = 0.0;
       for (int cc = lane; cc < p.NC; cc += 32) {
         const double2 z = __ldcg(&p.zpart[static_cast<size_t>(cc) * p.B + b]);
@@ -497,9 +589,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       const int rk = p.cu_q[b] + p.n_draft[b];
       const double Tgt = static_cast<double>(p.uniforms[rk]) * Z;
       // First slice whose cumulative mass exceeds Tgt; else the last slice with mass.
-      double base = 0.0;
+      double base = 0.0, base_owner = 0.0, base_last = 0.0;
       int owner = -1, last_pos = -1;
-      double base_last = 0.0, base_owner = 0.0;
       for (int c0 = 0; c0 < p.NC && owner < 0; c0 += 32) {
         const int cc = c0 + lane;
         double z = 0.0;
@@ -529,13 +620,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       }
       if (lane == 0) {
         if (usep && c == 0) atomicOr(p.status, SPADE_DEV_FALLBACK);
-        if (owner >= 0) {
-          s_owner[b] = owner;
-          s_T[b] = Tgt - base_owner;
-        } else {
-          s_owner[b] = last_pos;
-          s_T[b] = Tgt - base_last;  // beyond the slice total: the scan clamps
-        }
+        s_owner[b] = owner >= 0 ? owner : last_pos;
+        s_T[b] = Tgt - (owner >= 0 ? base_owner : base_last);  // beyond the slice total: clamp
         s_usep[b] = usep;
       }
     }
@@ -544,26 +630,69 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       const int ew = warp - 2, q4 = warp & 3;
       const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
       for (int b = 0; b < p.B; ++b) {
-        if (s_owner[b] != c) continue;
+        if (!s_stoch[b] || s_owner[b] != c) continue;
         const int n = s_rstar[b];
         const int a = s_acc[b], k = p.n_draft[b];
         const bool usep = s_usep[b] != 0;
-        const float *qrow = (a < k && !usep)
-                                ? p.draft_probs + static_cast<size_t>(p.cu_q[b] - b + a) * p.V
-                                : nullptr;
+        const float *qrow = (a < k && !usep) ? p.draft_probs + static_cast<size_t>(n - b) * p.V : nullptr;
         const float M = g_m[n], invS = 1.f / g_s[n];
-        const double Tgt = s_T[b];
-        double run = 0.0;
-        int found = -1, last_pos = -1;
-        for (int j = 0; j < ntiles && found < 0; ++j) {
-          const int v = (t_lo + j) * kTileV + q4 * 32 + lane;
+        // (1) mass of every 32-entry segment (tile j, lane quarter q4) of the slice.
+        for (int j0 = 0; j0 < ntiles; j0 += 8) {
+          const int nj = min(8, ntiles - j0);
+          uint32_t raw[8];
+          float qv[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (j < nj) tmem_ld1(tmem + lane_base + static_cast<uint32_t>((j0 + j) * p.Rs + n), raw[j]);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int v = (t_lo + j0 + j) * kTileV + q4 * 32 + lane;
+            qv[j] = (j < nj && qrow && v < p.V) ? qrow[v] : 0.f;
+          }
+          tmem_wait_ld();
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int v = (t_lo + j0 + j) * kTileV + q4 * 32 + lane;
+            double rv = 0.0;
+            if (j < nj && v < p.V) {
+              const double pv = static_cast<double>(expf(__uint_as_float(raw[j]) - M) * invS);
+              rv = qrow ? fmax(0.0, pv - static_cast<double>(qv[j])) : pv;
+            }
+            rv = warp_sum_d(rv);
+            if (lane == 0 && j < nj) s_tw[(j0 + j) * kEpiWarps + q4] = rv;
+          }
+        }
+        named_bar(1, kEpiWarps * 32);
+        // (2) the segment holding the target, in vocabulary order.
+        if (ew == 0 && lane == 0) {
+          double run = 0.0, tgt = s_T[b];
+          int jt = -1, qt = -1, jl = -1, ql = -1;
+          for (int j = 0; j < ntiles && jt < 0; ++j) {
+            for (int q = 0; q < kEpiWarps; ++q) {
+              const double mseg = s_tw[j * kEpiWarps + q];
+              if (mseg > 0.0) { jl = j; ql = q; }
+              if (run + mseg > tgt && mseg > 0.0) { jt = j; qt = q; tgt -= run; break; }
+              run += mseg;
+            }
+          }
+          if (jt < 0) { jt = jl; qt = ql; tgt = 1e300; }  // rounding: clamp to the last mass
+          s_seg[0] = jt;
+          s_seg[1] = qt;
+          s_T[b] = tgt;
+        }
+        named_bar(1, kEpiWarps * 32);
+        // (3) the warp owning that segment scans its 32 entries.
+        const int jt = s_seg[0], qt = s_seg[1];
+        if (jt >= 0 && q4 == qt) {
           uint32_t raw;
-          tmem_ld1(tmem + lane_base + static_cast<uint32_t>(j * p.Rs + n), raw);
+          tmem_ld1(tmem + lane_base + static_cast<uint32_t>(jt * p.Rs + n), raw);
+          const int v = (t_lo + jt) * kTileV + q4 * 32 + lane;
+          const float qv = (qrow && v < p.V) ? qrow[v] : 0.f;
           tmem_wait_ld();
           double rv = 0.0;
           if (v < p.V) {
             const double pv = static_cast<double>(expf(__uint_as_float(raw) - M) * invS);
-            rv = qrow ? fmax(0.0, pv - static_cast<double>(qrow[v])) : pv;
+            rv = qrow ? fmax(0.0, pv - static_cast<double>(qv)) : pv;
           }
           double incl = rv;
 #pragma unroll
@@ -571,30 +700,16 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             const double t = __shfl_up_sync(0xffffffffu, incl, o);
             if (lane >= o) incl += t;
           }
-          const double wsum = __shfl_sync(0xffffffffu, incl, 31);
-          if (lane == 0) s_red[ew * 2] = wsum;
-          named_bar(1, kEpiWarps * 32);
-          double before = run;  // mass of this slice before this warp's 32 entries
-          for (int w = 0; w < q4; ++w) before += s_red[((w + 2) & 3) * 2];
-          double tile_tot = 0.0;
-          for (int w = 0; w < kEpiWarps; ++w) tile_tot += s_red[w * 2];
-          const unsigned hit = __ballot_sync(0xffffffffu, before + incl > Tgt && rv > 0.0);
+          const unsigned hit = __ballot_sync(0xffffffffu, incl > s_T[b] && rv > 0.0);
           const unsigned pos = __ballot_sync(0xffffffffu, rv > 0.0);
-          int my_found = hit ? v - lane + (__ffs(hit) - 1) : -1;
-          int my_last = pos ? v - lane + (31 - __clz(pos)) : -1;
-          named_bar(1, kEpiWarps * 32);
           if (lane == 0) {
-            reinterpret_cast<int *>(s_red)[2 * kEpiWarps * 2 + q4] = my_found;
-            reinterpret_cast<int *>(s_red)[2 * kEpiWarps * 2 + 4 + q4] = my_last;
+            const int l = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : 0);
+            p.next_token[b] = v + l;
           }
-          named_bar(1, kEpiWarps * 32);
-          const int *res = reinterpret_cast<const int *>(s_red) + 2 * kEpiWarps * 2;
-          for (int w = 0; w < 4 && found < 0; ++w) found = res[w];
-          for (int w = 0; w < 4; ++w) last_pos = res[4 + w] >= 0 ? res[4 + w] : last_pos;
-          run += tile_tot;
-          named_bar(1, kEpiWarps * 32);
+        } else if (jt < 0 && ew == 0 && lane == 0) {
+          p.next_token[b] = -1;
         }
-        if (ew == 0 && lane == 0) p.next_token[b] = found >= 0 ? found : last_pos;
+        named_bar(1, kEpiWarps * 32);
       }
     }
   }
@@ -643,11 +758,46 @@ static Plan make_plan(int R, int V, int sms) {
 }
 
 static size_t workspace_bytes_for(int B, int R, int NC) {
-  size_t off = 256;                                     // barrier words
+  size_t off = 256;                                        // barrier words
   off += round_up(static_cast<size_t>(NC) * R * 16, 256);  // pstat
-  off += round_up(static_cast<size_t>(R) * 4, 256);       // ldraft
-  off += round_up(static_cast<size_t>(NC) * B * 16, 256); // zpart
+  off += round_up(static_cast<size_t>(R) * 4, 256);        // ldraft
+  off += round_up(static_cast<size_t>(NC) * B * 16, 256);  // zpart
   return off;
+}
+
+// 3-D view of a row-major [rows, H] bf16 matrix: dims {64, rows, H/64},
+// strides {H*2, 128} bytes, box {64, box_rows, kg}; lands as [kg][box_rows][64]
+// with the 128-byte swizzle, i.e. kg canonical K-major tiles back to back.
+static bool encode_kslab_view(CUtensorMap *map, const void *base, int rows, int H, int box_rows,
+                              int kg) {
+  using EncodeFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+  static EncodeFn fn = nullptr;
+  if (!fn) {
+    void *f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess) {
+      fail(SPADE_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+      return false;
+    }
+    fn = reinterpret_cast<EncodeFn>(f);
+  }
+  cuuint64_t dims[3] = {64, static_cast<cuuint64_t>(rows), static_cast<cuuint64_t>(H / 64)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(H) * 2, 128};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(box_rows), static_cast<cuuint32_t>(kg)};
+  cuuint32_t es[3] = {1, 1, 1};
+  const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    fail(SPADE_ERR_CUDA, "cuTensorMapEncodeTiled (k-slab view) failed (%d)", static_cast<int>(r));
+    return false;
+  }
+  return true;
 }
 
 }  // namespace accept
@@ -679,6 +829,7 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
     return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept: bad sizes B=%d R=%d H=%d V=%d", B, R, H, V);
   if (H % 8) return fail(SPADE_ERR_SHAPE, "hidden size %d must be a multiple of 8", H);
   if (R > kMaxR) return fail(SPADE_ERR_SHAPE, "R = %d verify rows exceed %d per call", R, kMaxR);
+  if (B > kMaxB) return fail(SPADE_ERR_SHAPE, "B = %d sequences exceed %d per call", B, kMaxB);
   if (!aligned(hidden, 16) || !aligned(w_lm, 16))
     return fail(SPADE_ERR_INVALID_ARG, "hidden and w_lm must be 16-byte aligned");
   int sms = 0;
@@ -699,23 +850,30 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
   p.B = B; p.R = R; p.H = H; p.V = V;
   p.T = pl.T; p.NC = pl.NC; p.Ncols = pl.Ncols; p.Rs = pl.Rs;
   p.KC = (H + kKChunk - 1) / kKChunk;
+  p.KCF = H / kKChunk;
   const int tiles_max = (pl.T + pl.NC - 1) / pl.NC;
+  if (tiles_max > kMaxTilesPerCta)
+    return fail(SPADE_ERR_SHAPE, "vocabulary %d needs %d tiles per SM (max %d)", V, tiles_max, kMaxTilesPerCta);
   if (!plan_rounds(tiles_max, pl.Ncols, pl.Rs, p.round_tiles, &p.nrounds))
     return fail(SPADE_ERR_SHAPE,
                 "logits of %d rows x %d vocab do not fit on chip (%d tiles per SM, %d TMEM columns each)",
                 R, V, tiles_max, pl.Rs);
   p.idesc = idesc_bf16_f32(kTileV, pl.Ncols);
   p.tmem_cols = kTmemCols;
-  p.HS = 3;
-  p.WS = 2;
-  {
+  // Two k-chunks per stage (32 KB W boxes) while the rings fit in shared memory.
+  p.HS = 2;
+  p.KG = 2;
+  for (;;) {
     Params probe = p;
     probe.WS = 0;
     const int fixed = smem_layout(probe).total;
-    p.WS = (kSmemBudget - fixed) / kWSlotBytes;
-    if (p.WS > 12) p.WS = 12;
-    if (p.WS < 2) return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
+    p.WS = (kSmemBudget - fixed) / (p.KG * kWChunkBytes);
+    if (p.WS > 8) p.WS = 8;
+    if (p.WS >= 4 || p.KG == 1) break;
+    p.KG = 1;
   }
+  if (p.WS < 2) return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
+  p.NS = (p.KC + p.KG - 1) / p.KG;
   const size_t need = workspace_bytes_for(B, R, pl.NC);
   if (!workspace || workspace_bytes < need || !aligned(workspace, 256))
     return fail(SPADE_ERR_WORKSPACE, "accept workspace needs %zu bytes, 256-byte aligned (got %zu)",
@@ -729,10 +887,20 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
   off += round_up(static_cast<size_t>(R) * 4, 256);
   p.zpart = reinterpret_cast<double2 *>(ws + off);
 
-  CUtensorMap tw, th;
-  if (!encode_tmap_bf16_sw128(&tw, w_lm, H, V, static_cast<uint64_t>(H) * 2, kKChunk, kTileV) ||
-      !encode_tmap_bf16_sw128(&th, hidden, H, R, static_cast<uint64_t>(H) * 2, kKChunk, pl.Ncols))
+  // 2-D views (one k-chunk per box, zero fill past H) serve a ragged last
+  // k-chunk; 3-D views fetch KG full k-chunks per box.
+  CUtensorMap tw2, th2, tw3, th3;
+  if (!encode_tmap_bf16_sw128(&tw2, w_lm, H, V, static_cast<uint64_t>(H) * 2, kKChunk, kTileV) ||
+      !encode_tmap_bf16_sw128(&th2, hidden, H, R, static_cast<uint64_t>(H) * 2, kKChunk, pl.Ncols))
     return SPADE_ERR_CUDA;
+  if (p.KCF >= 1) {
+    if (!encode_kslab_view(&tw3, w_lm, V, H, kTileV, p.KG) ||
+        !encode_kslab_view(&th3, hidden, R, H, pl.Ncols, p.KG))
+      return SPADE_ERR_CUDA;
+  } else {
+    tw3 = tw2;  // never used: every stage takes the 2-D path
+    th3 = th2;
+  }
 
   const int smem = smem_layout(p).total;
   static bool configured = false;
@@ -742,6 +910,7 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(verify_accept)");
     configured = true;
   }
+  if (smem > kSmemBudget + 2048) return fail(SPADE_ERR_SHAPE, "shared memory plan too large (%d)", smem);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(pl.NC);
   cfg.blockDim = dim3(kThreads);
@@ -752,7 +921,7 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, verify_accept_kernel, p, tw, th);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, verify_accept_kernel, p, tw3, tw2, th3, th2);
   if (e != cudaSuccess) return cuda_fail(e, "verify_accept cooperative launch");
   return SPADE_OK;
 }
