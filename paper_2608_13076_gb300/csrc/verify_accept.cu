@@ -20,12 +20,13 @@
 //    MMAs from a single thread, warps 2-5 read accumulators back (tcgen05.ld)
 //    and reduce per-row max / sum-exp / argmax across the vocabulary (an
 //    8-row shared-memory transpose, then a 4-lane shuffle merge).
-//  * Two bounded device-wide barriers: after the first every CTA merges the
-//    per-slice statistics into p(d) and argmax for every row and takes the
-//    accept decisions; after the second the slice masses of the distribution
-//    to sample (residual or p, fp64) are known, and the CTA whose slice holds
-//    the point u*Z locates its 32-entry segment and scans it in vocabulary
-//    order to pick the token.
+//  * Bounded device-wide barriers separate the phases: after the first, CTA c
+//    merges the slice statistics of rows c, c + NC, ...; after the second every
+//    CTA holds max, sum-exp and argmax of every row and takes the accept
+//    decisions; after the third (only with stochastic sequences) the slice
+//    masses of the distribution to sample (residual or p, float-float sums)
+//    are known, and the CTA whose slice holds the point u*Z locates its
+//    32-entry segment and scans it in vocabulary order to pick the token.
 #include <cuda_bf16.h>
 
 #include <cfloat>
@@ -62,7 +63,8 @@ struct Params {
   unsigned *bar;     // [2]: arrival count, generation
   float4 *pstat;     // [NC][R]: slice max, slice sum-exp, slice argmax (bits), -
   float *ldraft;     // [R]: logit of the row's draft token
-  double2 *zpart;    // [NC][B]: slice mass of the distribution to sample, of p
+  float4 *gstat;     // [R]: merged row max, sum-exp, argmax (bits)
+  float4 *zpart;     // [NC][B]: slice mass of the sampled distribution and of p (float-float)
   int B, R, H, V, T, NC, Ncols, Rs;
   int KC;            // k-chunks of 64 (the last may be partial)
   int KCF;           // full k-chunks (H / 64)
@@ -71,6 +73,7 @@ struct Params {
   int nrounds;
   int round_tiles[kMaxRounds];
   int HS, WS;        // hidden / W ring slots
+  int BRS;           // box rows of the map used for a slice's last, partial tile
   uint32_t idesc;
   uint32_t tmem_cols;
 };
@@ -87,15 +90,23 @@ __host__ __device__ inline Smem smem_layout(const Params &p) {
   s.off_h = p.WS * s.w_slot;
   s.off_bar = s.off_h + p.HS * s.h_slot;
   s.off_misc = s.off_bar + (2 * p.WS + 2 * p.HS + 2) * 8;
-  s.off_rows = s.off_misc + 64;                     // int [3][kMaxR]: draft, seq, pos
-  s.off_wst = s.off_rows + 3 * kMaxR * 4;           // float4 [kEpiWarps][kMaxR]
-  s.off_tbuf = s.off_wst + kEpiWarps * kMaxR * 16;  // float [kEpiWarps][16][32]
+  s.off_rows = s.off_misc + 64;  // int/float [5][kMaxR] + int [3][kMaxB + 1]
+  s.off_wst = s.off_rows + 5 * kMaxR * 4 + 3 * (kMaxB + 1) * 4 + 4;  // float4 [kEpiWarps][R]
+  s.off_tbuf = s.off_wst + kEpiWarps * p.R * 16;    // float [kEpiWarps][16][32]
   s.total = s.off_tbuf + kEpiWarps * 16 * 32 * 4 + 1024;
   return s;
 }
 
+// bar.sync is the aligned form: every lane of a warp must arrive together.
+// Lanes that ran ahead of a divergent lane (a lane-0-only loop) reconverge
+// first, so no warp reaches the barrier before all of its lanes do.
 __device__ __forceinline__ void named_bar(int id, int threads) {
+  __syncwarp();
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+__device__ __forceinline__ void block_sync() {
+  __syncwarp();
+  __syncthreads();
 }
 
 __device__ __forceinline__ unsigned ld_acquire(const unsigned *p) {
@@ -118,25 +129,24 @@ __device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, i
 // poll the generation with a time limit.  Returns false if the wait expired.
 __device__ bool grid_barrier(unsigned *bar, int nctas) {
   __shared__ int s_ok;
-  __syncthreads();
+  block_sync();
   if (threadIdx.x == 0) {
     s_ok = 1;
     const unsigned gen = ld_acquire(bar + 1);
-    __threadfence();
-    const unsigned arrived = atomicAdd(bar, 1u);
+    unsigned arrived;
+    // The arrival releases this CTA's writes (ordered before it by bar.sync).
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(arrived) : "l"(bar) : "memory");
     if (arrived == static_cast<unsigned>(nctas) - 1) {
-      atomicExch(bar, 0u);
-      __threadfence();
-      atomicAdd(bar + 1, 1u);
+      asm volatile("st.relaxed.gpu.global.u32 [%0], 0;" ::"l"(bar) : "memory");
+      asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(bar + 1) : "memory");
     } else {
       const uint64_t t0 = globaltimer();
       while (ld_acquire(bar + 1) == gen) {
         if (globaltimer() - t0 > kWaitLimitNs) { s_ok = 0; break; }
       }
     }
-    __threadfence();
   }
-  __syncthreads();
+  block_sync();
   return s_ok != 0;
 }
 
@@ -152,16 +162,66 @@ __device__ __forceinline__ void stat_merge(float &m, float &s, int &i, float om,
   m = M;
 }
 
-__device__ __forceinline__ double warp_sum_d(double v) {
+// Float-float numbers (hi + lo, about 48 significant bits) for the sums that
+// place u*Z: GB300's fp64 rate is a small fraction of fp32, so the cumulative
+// masses use error-free fp32 transformations instead of doubles.
+struct ff2 {
+  float hi, lo;
+};
+// Knuth's TwoSum: s + e == a + b exactly.
+__device__ __forceinline__ ff2 two_sum(float a, float b) {
+  const float s = a + b;
+  const float bb = s - a;
+  const float e = (a - (s - bb)) + (b - bb);
+  return ff2{s, e};
+}
+__device__ __forceinline__ ff2 ff_norm(float hi, float lo) {
+  const float s = hi + lo;
+  return ff2{s, lo - (s - hi)};
+}
+__device__ __forceinline__ ff2 ff_add(ff2 a, ff2 b) {
+  const ff2 s = two_sum(a.hi, b.hi);
+  return ff_norm(s.hi, s.lo + a.lo + b.lo);
+}
+__device__ __forceinline__ ff2 ff_add_f(ff2 a, float b) {
+  const ff2 s = two_sum(a.hi, b);
+  return ff_norm(s.hi, s.lo + a.lo);
+}
+__device__ __forceinline__ ff2 ff_sub(ff2 a, ff2 b) { return ff_add(a, ff2{-b.hi, -b.lo}); }
+// a * b with the product's rounding error recovered by an fma.
+__device__ __forceinline__ ff2 ff_mul_f(ff2 a, float b) {
+  const float p = a.hi * b;
+  float e = fmaf(a.hi, b, -p);
+  e = fmaf(a.lo, b, e);
+  return ff_norm(p, e);
+}
+__device__ __forceinline__ bool ff_gt(ff2 a, ff2 b) {
+  const ff2 d = ff_sub(a, b);
+  return d.hi > 0.f || (d.hi == 0.f && d.lo > 0.f);
+}
+__device__ __forceinline__ ff2 ff_shfl(ff2 v, int src) {
+  return ff2{__shfl_sync(0xffffffffu, v.hi, src), __shfl_sync(0xffffffffu, v.lo, src)};
+}
+__device__ __forceinline__ ff2 warp_sum_ff(ff2 v) {
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  for (int o = 16; o > 0; o >>= 1)
+    v = ff_add(v, ff2{__shfl_xor_sync(0xffffffffu, v.hi, o), __shfl_xor_sync(0xffffffffu, v.lo, o)});
+  return ff_shfl(v, 0);  // one value for every lane
+}
+// Inclusive prefix sum over the warp's lanes.
+__device__ __forceinline__ ff2 warp_scan_ff(ff2 v, int lane) {
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const ff2 t{__shfl_up_sync(0xffffffffu, v.hi, o), __shfl_up_sync(0xffffffffu, v.lo, o)};
+    if (lane >= o) v = ff_add(t, v);
+  }
   return v;
 }
 
 // Per-row running statistics of one epilogue warp: the 8 rows c8*8..c8*8+7 of
 // the 32 vocab entries held in registers by the warp's lanes.
-__device__ __forceinline__ void reduce_rows8(const uint32_t *raw, int c8, int vlane0, int lane,
-                                             const Params &p, const int32_t *s_draft,
+__device__ __forceinline__ void reduce_rows8(const uint32_t *raw, int c8, int vlane0, int vlimit,
+                                             int lane, const Params &p, const int32_t *s_draft,
                                              float *tbuf, float4 *wst) {
 #pragma unroll
   for (int e = 0; e < 8; ++e) tbuf[e * 32 + lane] = __uint_as_float(raw[e]);
@@ -177,8 +237,8 @@ __device__ __forceinline__ void reduce_rows8(const uint32_t *raw, int c8, int vl
   int mi = INT_MAX;
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
-    if (v0 + i >= p.V) x[i] = -INFINITY;
-    if (v0 + i == d) p.ldraft[n] = x[i];
+    if (v0 + i >= vlimit) x[i] = -INFINITY;        // lanes past this CTA's slice
+    else if (v0 + i == d) p.ldraft[n] = x[i];      // only the slice owner writes
     if (x[i] > m) { m = x[i]; mi = v0 + i; }
   }
   float s = 0.f;
@@ -205,8 +265,8 @@ __device__ __forceinline__ void reduce_rows8(const uint32_t *raw, int c8, int vl
 
 __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tm_w3,
-    const __grid_constant__ CUtensorMap tm_w2, const __grid_constant__ CUtensorMap tm_h3,
-    const __grid_constant__ CUtensorMap tm_h2) {
+    const __grid_constant__ CUtensorMap tm_w2, const __grid_constant__ CUtensorMap tm_w2s,
+    const __grid_constant__ CUtensorMap tm_h3, const __grid_constant__ CUtensorMap tm_h2) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -225,14 +285,22 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   int32_t *s_draft = reinterpret_cast<int32_t *>(smem + L.off_rows);
   int32_t *s_seq = s_draft + kMaxR;
   int32_t *s_pos = s_seq + kMaxR;
+  float *s_u = reinterpret_cast<float *>(s_pos + kMaxR);   // uniforms[n]
+  float *s_qd = s_u + kMaxR;                              // q of the row's draft token
+  int32_t *s_cuq = reinterpret_cast<int32_t *>(s_qd + kMaxR);
+  int32_t *s_nd = s_cuq + kMaxB + 1;
+  int32_t *s_md = s_nd + kMaxB;
   float4 *s_wst = reinterpret_cast<float4 *>(smem + L.off_wst);
   float *s_tbuf = reinterpret_cast<float *>(smem + L.off_tbuf);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c = blockIdx.x;
-  const int t_lo = static_cast<int>(static_cast<int64_t>(c) * p.T / p.NC);
-  const int t_hi = static_cast<int>(static_cast<int64_t>(c + 1) * p.T / p.NC);
-  const int ntiles = t_hi - t_lo;
+  // This CTA's vocabulary slice [v_lo, v_hi): equal row counts (within one),
+  // cut into 128-row tiles; the last tile may be partial.
+  const int v_lo = static_cast<int>(static_cast<int64_t>(c) * p.V / p.NC);
+  const int v_hi = static_cast<int>(static_cast<int64_t>(c + 1) * p.V / p.NC);
+  const int ntiles = (v_hi - v_lo + kTileV - 1) / kTileV;
+  const bool short_last = (v_hi - v_lo) - (ntiles - 1) * kTileV <= p.BRS && p.BRS < kTileV;
 
   // ---- set-up: barriers, TMEM, per-row bookkeeping -------------------------
   if (tid == 0) {
@@ -249,8 +317,13 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     tmem_relinquish();
   }
   for (int n = tid; n < kMaxR; n += kThreads) { s_draft[n] = -1; s_seq[n] = -1; s_pos[n] = 0; }
-  __syncthreads();
+  block_sync();
   // Row n = cu_q[b] + i is position i of sequence b; it holds draft i for i < k_b.
+  for (int b = tid; b <= p.B; b += kThreads) s_cuq[b] = p.cu_q[b];
+  for (int b = tid; b < p.B; b += kThreads) {
+    s_nd[b] = p.n_draft[b];
+    s_md[b] = p.mode[b];
+  }
   for (int b = tid; b < p.B; b += kThreads) {
     const int r0 = p.cu_q[b], k = p.n_draft[b], r1 = p.cu_q[b + 1];
     if (r0 < 0 || k < 0 || r1 - r0 != k + 1 || r1 > p.R) {
@@ -264,7 +337,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     }
   }
   tc_fence_before();
-  __syncthreads();
+  block_sync();
   tc_fence_after();
   const uint32_t tmem = *s_tmem;
   int rounds_issued = 0;  // MMA thread: accumulator rounds committed
@@ -305,11 +378,18 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             mbar_wait(&w_empty[s], ((wi / p.WS) & 1) ^ 1, s_abort);
             if (!*s_abort) {
               uint8_t *dst = w_ring + s * L.w_slot;
-              const int row0 = (t_lo + tdone + j) * kTileV;
-              mbar_arrive_expect_tx(&w_full[s], nch * kWChunkBytes);
-              if (box3) {
+              const int row0 = v_lo + (tdone + j) * kTileV;
+              if (short_last && tdone + j == ntiles - 1) {
+                // Partial last tile: BRS-row boxes, one per k-chunk; the slot's
+                // remaining rows feed accumulator lanes that are never read.
+                mbar_arrive_expect_tx(&w_full[s], nch * p.BRS * 128);
+                for (int jj = 0; jj < nch; ++jj)
+                  tma_load_2d(dst + jj * kWChunkBytes, &tm_w2s, (c0 + jj) * kKChunk, row0, &w_full[s], pol_w);
+              } else if (box3) {
+                mbar_arrive_expect_tx(&w_full[s], nch * kWChunkBytes);
                 tma_load_3d(dst, &tm_w3, 0, row0, c0, &w_full[s], pol_w);
               } else {
+                mbar_arrive_expect_tx(&w_full[s], nch * kWChunkBytes);
                 for (int jj = 0; jj < nch; ++jj)
                   tma_load_2d(dst + jj * kWChunkBytes, &tm_w2, (c0 + jj) * kKChunk, row0, &w_full[s], pol_w);
               }
@@ -373,9 +453,18 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     const int ew = warp - 2;             // 0..3
     const int q4 = warp & 3;             // TMEM lane quarter this warp may access
     const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
-    float4 *wst = s_wst + ew * kMaxR;    // this warp's running stats per row
+    float4 *wst = s_wst + ew * p.R;      // this warp's running stats per row
     float *tbuf = s_tbuf + ew * 16 * 32;
     for (int n = lane; n < p.R; n += 32) wst[n] = make_float4(-INFINITY, 0.f, __int_as_float(INT_MAX), 0.f);
+    // While the first round accumulates: uniforms and q(draft) of every row.
+    for (int n = tid - 64; n < p.R; n += kEpiWarps * 32) {
+      s_u[n] = p.uniforms[n];
+      const int b = s_seq[n], d = s_draft[n];
+      float qd = 0.f;
+      if (b >= 0 && d >= 0 && d < p.V && s_md[b] == 1 && p.draft_probs != nullptr)
+        qd = p.draft_probs[static_cast<size_t>(n - b) * p.V + d];
+      s_qd[n] = qd;
+    }
     __syncwarp();
     int tdone = 0, used = 0;
     for (int r = 0; r < p.nrounds && tdone < ntiles; ++r) {
@@ -404,7 +493,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       if (lane == 0) mbar_arrive(acc_empty);
       for (int j = 0; j < nt; ++j) {
         const int t = tdone + j;
-        const int vlane0 = (t_lo + t) * kTileV + q4 * 32;  // vocab id of lane 0's row
+        const int vlane0 = v_lo + t * kTileV + q4 * 32;  // vocab id of lane 0's row
         const uint32_t col = tmem + lane_base + static_cast<uint32_t>(t * p.Rs);
         int c8 = 0;
         for (; (c8 + 1) * 8 < p.R; c8 += 2) {
@@ -412,14 +501,14 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           tmem_ld8(col + c8 * 8, raw);
           tmem_ld8(col + c8 * 8 + 8, raw + 8);
           tmem_wait_ld();
-          reduce_rows8(raw, c8, vlane0, lane, p, s_draft, tbuf, wst);
-          reduce_rows8(raw + 8, c8 + 1, vlane0, lane, p, s_draft, tbuf + 256, wst);
+          reduce_rows8(raw, c8, vlane0, v_hi, lane, p, s_draft, tbuf, wst);
+          reduce_rows8(raw + 8, c8 + 1, vlane0, v_hi, lane, p, s_draft, tbuf + 256, wst);
         }
         if (c8 * 8 < p.R) {
           uint32_t raw[8];
           tmem_ld8(col + c8 * 8, raw);
           tmem_wait_ld();
-          reduce_rows8(raw, c8, vlane0, lane, p, s_draft, tbuf, wst);
+          reduce_rows8(raw, c8, vlane0, v_hi, lane, p, s_draft, tbuf, wst);
         }
       }
       used += nt * p.Rs;
@@ -431,7 +520,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       float m = -INFINITY, s = 0.f;
       int idx = INT_MAX;
       for (int w = 0; w < kEpiWarps; ++w) {
-        const float4 st = s_wst[w * kMaxR + n];
+        const float4 st = s_wst[w * p.R + n];
         stat_merge(m, s, idx, st.x, st.y, __float_as_int(st.z));
       }
       __stcg(&p.pstat[static_cast<size_t>(c) * p.R + n], make_float4(m, s, __int_as_float(idx), 0.f));
@@ -440,6 +529,39 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   if (*s_abort) atomicOr(p.status, SPADE_DEV_TIMEOUT);
 
   // ======================= phase B: global row statistics, decisions =======
+  if (!grid_barrier(p.bar, p.NC)) {
+    atomicOr(p.status, SPADE_DEV_TIMEOUT);
+    *s_abort = 1;
+  }
+  // (1) Rows n = c, c + NC, ... are merged by this CTA, one warp per row, from
+  //     the NC slice partials (every CTA reading every partial would pile all
+  //     SMs onto the same L2 lines); the merged statistics go to the workspace.
+  {
+    constexpr int kChunksPerPass = 5;
+    for (int n = c + warp * p.NC; n < p.R; n += (kThreads / 32) * p.NC) {
+      float m = -INFINITY, sm = 0.f;
+      int idx = INT_MAX;
+      for (int cc0 = 0; cc0 < p.NC; cc0 += 32 * kChunksPerPass) {
+        float4 st[kChunksPerPass];
+#pragma unroll
+        for (int i = 0; i < kChunksPerPass; ++i) {
+          const int cc = cc0 + i * 32 + lane;
+          st[i] = cc < p.NC ? __ldcg(&p.pstat[static_cast<size_t>(cc) * p.R + n])
+                            : make_float4(-INFINITY, 0.f, __int_as_float(INT_MAX), 0.f);
+        }
+#pragma unroll
+        for (int i = 0; i < kChunksPerPass; ++i) stat_merge(m, sm, idx, st[i].x, st[i].y, __float_as_int(st[i].z));
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float om = __shfl_xor_sync(0xffffffffu, m, o);
+        const float os = __shfl_xor_sync(0xffffffffu, sm, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
+        stat_merge(m, sm, idx, om, os, oi);
+      }
+      if (lane == 0) __stcg(&p.gstat[n], make_float4(m, sm, __int_as_float(idx), 0.f));
+    }
+  }
   if (!grid_barrier(p.bar, p.NC)) {
     atomicOr(p.status, SPADE_DEV_TIMEOUT);
     *s_abort = 1;
@@ -455,39 +577,28 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   int *s_usep = s_owner + kMaxB;                            // [B]
   int *s_stoch = s_usep + kMaxB;                            // [B]
   int *s_seg = s_stoch + kMaxB;                             // [2]: tile, quarter
-  double *s_T = reinterpret_cast<double *>(s_seg + 16);     // [B]
-  double *s_zw = s_T + kMaxB;                               // [B][kEpiWarps][2]
-  double *s_tw = s_zw + kMaxB * kEpiWarps * 2;              // [kMaxTilesPerCta][kEpiWarps]
-
-  for (int n = warp; n < p.R; n += kThreads / 32) {
-    float m = -INFINITY, s = 0.f;
-    int idx = INT_MAX;
-#pragma unroll 4
-    for (int cc = lane; cc < p.NC; cc += 32) {
-      const float4 st = __ldcg(&p.pstat[static_cast<size_t>(cc) * p.R + n]);
-      stat_merge(m, s, idx, st.x, st.y, __float_as_int(st.z));
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float om = __shfl_xor_sync(0xffffffffu, m, o);
-      const float os = __shfl_xor_sync(0xffffffffu, s, o);
-      const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
-      stat_merge(m, s, idx, om, os, oi);
-    }
-    if (lane == 0) { g_m[n] = m; g_s[n] = s; g_arg[n] = idx; }
+  float2 *s_T = reinterpret_cast<float2 *>(s_seg + 16);     // [B] float-float
+  float4 *s_zw = reinterpret_cast<float4 *>(s_T + kMaxB);   // [B][kEpiWarps]
+  float2 *s_tw = reinterpret_cast<float2 *>(s_zw + kMaxB * kEpiWarps);  // [tiles][kEpiWarps]
+  // (2) Every CTA reads the merged statistics of all rows.
+  for (int n = tid; n < p.R; n += kThreads) {
+    const float4 g = __ldcg(&p.gstat[n]);
+    g_m[n] = g.x;
+    g_s[n] = g.y;
+    g_arg[n] = __float_as_int(g.z);
   }
   for (int b = tid; b < p.B; b += kThreads) {
-    const int md = p.mode[b];
+    const int md = s_md[b];
     if (md != 0 && md != 1 && c == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
     s_stoch[b] = (md == 1) && p.draft_probs != nullptr;
   }
-  __syncthreads();
-  // Accept test of every draft row, all rows at once (the tests are independent;
-  // only the count of leading accepts depends on their order).
+  block_sync();
+  // (3) Accept test of every draft row, all rows at once (the tests are
+  //     independent; only the count of leading accepts depends on their order).
   for (int n = tid; n < p.R; n += kThreads) {
     const int b = s_seq[n];
     int ok = 0;
-    if (b >= 0 && s_pos[n] < p.n_draft[b]) {
+    if (b >= 0 && s_pos[n] < s_nd[b]) {
       const int d = s_draft[n];
       if (d < 0 || d >= p.V) {
         if (c == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
@@ -495,17 +606,18 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         ok = (d == g_arg[n]);
       } else {
         const float pd = expf(__ldcg(&p.ldraft[n]) - g_m[n]) / g_s[n];
-        const float qd = p.draft_probs[static_cast<size_t>(n - b) * p.V + d];
-        ok = (qd > 0.f) ? (p.uniforms[n] < pd / qd) : (pd > 0.f);
+        const float qd = s_qd[n];
+        ok = (qd > 0.f) ? (s_u[n] < pd / qd) : (pd > 0.f);
       }
     }
     s_ok[n] = ok;
   }
-  __syncthreads();
+  block_sync();
+  // (4) Accepted length = leading accepts; the row that emits the next token.
   for (int b = tid; b < p.B; b += kThreads) {
-    const int r0 = p.cu_q[b], k = p.n_draft[b];
+    const int r0 = s_cuq[b], k = s_nd[b];
     int a = -1;
-    if (r0 >= 0 && k >= 0 && p.cu_q[b + 1] - r0 == k + 1 && p.cu_q[b + 1] <= p.R) {
+    if (r0 >= 0 && k >= 0 && s_cuq[b + 1] - r0 == k + 1 && s_cuq[b + 1] <= p.R) {
       a = 0;
       while (a < k && s_ok[r0 + a]) ++a;
     }
@@ -519,55 +631,90 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       else if (!s_stoch[b]) p.next_token[b] = g_arg[r0 + a];
     }
   }
-  __syncthreads();
+  block_sync();
 
   if (*s_any_stoch) {
     // =================== phase C: slice masses of the sampled distribution ==
+    // Terms are fp32; every sum is float-float, so the cumulative masses that
+    // place u*Z are as exact as the terms allow.
     if (warp >= 2) {
       const int ew = warp - 2, q4 = warp & 3;
       const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
-      for (int b = 0; b < p.B; ++b) {
-        if (!s_stoch[b]) continue;
-        const int n = s_rstar[b];
-        const int a = s_acc[b], k = p.n_draft[b];
-        const float *qrow = (a < k) ? p.draft_probs + static_cast<size_t>(n - b) * p.V : nullptr;
-        const float M = g_m[n], invS = 1.f / g_s[n];
-        double z = 0.0, zp = 0.0;
+      // Stochastic sequences in groups of kG: the TMEM reads and q loads of a
+      // whole group are in flight together.
+      constexpr int kG = 4;
+      for (int b0 = 0; b0 < p.B;) {
+        int bl[kG], nb = 0;
+        while (b0 < p.B && nb < kG) {
+          if (s_stoch[b0]) bl[nb++] = b0;
+          ++b0;
+        }
+        if (nb == 0) break;
+        const float *qrow[kG];
+        int nrow[kG];
+        float M[kG], invS[kG];
+        ff2 z[kG], zp[kG];
+#pragma unroll
+        for (int g = 0; g < kG; ++g) {
+          const int b = g < nb ? bl[g] : bl[0];
+          nrow[g] = s_rstar[b];
+          qrow[g] = (s_acc[b] < s_nd[b]) ? p.draft_probs + static_cast<size_t>(nrow[g] - b) * p.V : nullptr;
+          M[g] = g_m[nrow[g]];
+          invS[g] = 1.f / g_s[nrow[g]];
+          z[g] = ff2{0.f, 0.f};
+          zp[g] = ff2{0.f, 0.f};
+        }
         for (int j0 = 0; j0 < ntiles; j0 += 8) {
           const int nj = min(8, ntiles - j0);
-          uint32_t raw[8];
-          float qv[8];
+          uint32_t raw[kG][8];
+          float qv[kG][8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            if (j < nj) tmem_ld1(tmem + lane_base + static_cast<uint32_t>((j0 + j) * p.Rs + n), raw[j]);
+          for (int g = 0; g < kG; ++g) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              if (g < nb && j < nj)
+                tmem_ld1(tmem + lane_base + static_cast<uint32_t>((j0 + j) * p.Rs + nrow[g]), raw[g][j]);
           }
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int v = (t_lo + j0 + j) * kTileV + q4 * 32 + lane;
-            qv[j] = (j < nj && qrow && v < p.V) ? qrow[v] : 0.f;
+          for (int g = 0; g < kG; ++g) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
+              qv[g][j] = (g < nb && j < nj && qrow[g] && v < v_hi) ? qrow[g][v] : 0.f;
+            }
           }
           tmem_wait_ld();
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int v = (t_lo + j0 + j) * kTileV + q4 * 32 + lane;
-            if (j < nj && v < p.V) {
-              const double pv = static_cast<double>(expf(__uint_as_float(raw[j]) - M) * invS);
-              zp += pv;
-              z += qrow ? fmax(0.0, pv - static_cast<double>(qv[j])) : pv;
+          for (int g = 0; g < kG; ++g) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
+              if (g < nb && j < nj && v < v_hi) {
+                const float pv = expf(__uint_as_float(raw[g][j]) - M[g]) * invS[g];
+                zp[g] = ff_add_f(zp[g], pv);
+                z[g] = ff_add_f(z[g], qrow[g] ? fmaxf(0.f, pv - qv[g][j]) : pv);
+              }
             }
           }
         }
-        z = warp_sum_d(z);
-        zp = warp_sum_d(zp);
-        if (lane == 0) { s_zw[(b * kEpiWarps + ew) * 2] = z; s_zw[(b * kEpiWarps + ew) * 2 + 1] = zp; }
+#pragma unroll
+        for (int g = 0; g < kG; ++g) {
+          z[g] = warp_sum_ff(z[g]);
+          zp[g] = warp_sum_ff(zp[g]);
+          if (lane == 0 && g < nb) s_zw[bl[g] * kEpiWarps + ew] = make_float4(z[g].hi, z[g].lo, zp[g].hi, zp[g].lo);
+        }
       }
     }
-    __syncthreads();
+    block_sync();
     for (int b = tid; b < p.B; b += kThreads) {
       if (!s_stoch[b]) continue;
-      double zs = 0.0, zps = 0.0;
-      for (int w = 0; w < kEpiWarps; ++w) { zs += s_zw[(b * kEpiWarps + w) * 2]; zps += s_zw[(b * kEpiWarps + w) * 2 + 1]; }
-      __stcg(&p.zpart[static_cast<size_t>(c) * p.B + b], make_double2(zs, zps));
+      ff2 zs{0.f, 0.f}, zps{0.f, 0.f};
+      for (int w = 0; w < kEpiWarps; ++w) {
+        const float4 t = s_zw[b * kEpiWarps + w];
+        zs = ff_add(zs, ff2{t.x, t.y});
+        zps = ff_add(zps, ff2{t.z, t.w});
+      }
+      __stcg(&p.zpart[static_cast<size_t>(c) * p.B + b], make_float4(zs.hi, zs.lo, zps.hi, zps.lo));
     }
     if (!grid_barrier(p.bar, p.NC)) {
       atomicOr(p.status, SPADE_DEV_TIMEOUT);
@@ -576,63 +723,60 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     // =================== phase D: owner slice of u*Z, in-slice scan =========
     for (int b = warp; b < p.B; b += kThreads / 32) {
       if (!s_stoch[b]) { if (lane == 0) s_owner[b] = -1; continue; }
-      double tot = 0.0, totp = 0.0;
+      ff2 tot{0.f, 0.f}, totp{0.f, 0.f};
       for (int cc = lane; cc < p.NC; cc += 32) {
-        const double2 z = __ldcg(&p.zpart[static_cast<size_t>(cc) * p.B + b]);
-        tot += z.x;
-        totp += z.y;
+        const float4 z = __ldcg(&p.zpart[static_cast<size_t>(cc) * p.B + b]);
+        tot = ff_add(tot, ff2{z.x, z.y});
+        totp = ff_add(totp, ff2{z.z, z.w});
       }
-      tot = warp_sum_d(tot);
-      totp = warp_sum_d(totp);
-      const bool usep = !(tot > 0.0 && isfinite(tot));
-      const double Z = usep ? totp : tot;
-      const int rk = p.cu_q[b] + p.n_draft[b];
-      const double Tgt = static_cast<double>(p.uniforms[rk]) * Z;
+      tot = warp_sum_ff(tot);
+      totp = warp_sum_ff(totp);
+      const bool usep = !(tot.hi > 0.f && isfinite(tot.hi));
+      const ff2 Z = usep ? totp : tot;
+      const ff2 Tgt = ff_mul_f(Z, s_u[s_cuq[b] + s_nd[b]]);
       // First slice whose cumulative mass exceeds Tgt; else the last slice with mass.
-      double base = 0.0, base_owner = 0.0, base_last = 0.0;
+      ff2 base{0.f, 0.f}, base_owner{0.f, 0.f}, base_last{0.f, 0.f};
       int owner = -1, last_pos = -1;
       for (int c0 = 0; c0 < p.NC && owner < 0; c0 += 32) {
         const int cc = c0 + lane;
-        double z = 0.0;
+        ff2 z{0.f, 0.f};
         if (cc < p.NC) {
-          const double2 zz = __ldcg(&p.zpart[static_cast<size_t>(cc) * p.B + b]);
-          z = usep ? zz.y : zz.x;
+          const float4 zz = __ldcg(&p.zpart[static_cast<size_t>(cc) * p.B + b]);
+          z = usep ? ff2{zz.z, zz.w} : ff2{zz.x, zz.y};
         }
-        double incl = z;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const double t = __shfl_up_sync(0xffffffffu, incl, o);
-          if (lane >= o) incl += t;
-        }
-        const unsigned hit = __ballot_sync(0xffffffffu, cc < p.NC && base + incl > Tgt);
-        const unsigned pos = __ballot_sync(0xffffffffu, cc < p.NC && z > 0.0);
+        const ff2 incl = warp_scan_ff(z, lane);
+        const ff2 reach = ff_add(base, incl);
+        const ff2 before = ff_add(base, ff_sub(incl, z));  // mass of the slices before cc
+        const unsigned hit = __ballot_sync(0xffffffffu, cc < p.NC && ff_gt(reach, Tgt));
+        const unsigned pos = __ballot_sync(0xffffffffu, cc < p.NC && z.hi > 0.f);
         if (hit) {
           const int l = __ffs(hit) - 1;
           owner = c0 + l;
-          base_owner = base + __shfl_sync(0xffffffffu, incl - z, l);
+          base_owner = ff_shfl(before, l);
         }
         if (pos) {
           const int l = 31 - __clz(pos);
           last_pos = c0 + l;
-          base_last = base + __shfl_sync(0xffffffffu, incl - z, l);
+          base_last = ff_shfl(before, l);
         }
-        base += __shfl_sync(0xffffffffu, incl, 31);
+        base = ff_shfl(reach, 31);
       }
       if (lane == 0) {
         if (usep && c == 0) atomicOr(p.status, SPADE_DEV_FALLBACK);
         s_owner[b] = owner >= 0 ? owner : last_pos;
-        s_T[b] = Tgt - (owner >= 0 ? base_owner : base_last);  // beyond the slice total: clamp
+        const ff2 t = ff_sub(Tgt, owner >= 0 ? base_owner : base_last);  // past the total: clamp
+        s_T[b] = make_float2(t.hi, t.lo);
         s_usep[b] = usep;
       }
     }
-    __syncthreads();
+    block_sync();
     if (warp >= 2) {
       const int ew = warp - 2, q4 = warp & 3;
       const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
       for (int b = 0; b < p.B; ++b) {
         if (!s_stoch[b] || s_owner[b] != c) continue;
         const int n = s_rstar[b];
-        const int a = s_acc[b], k = p.n_draft[b];
+        const int a = s_acc[b], k = s_nd[b];
         const bool usep = s_usep[b] != 0;
         const float *qrow = (a < k && !usep) ? p.draft_probs + static_cast<size_t>(n - b) * p.V : nullptr;
         const float M = g_m[n], invS = 1.f / g_s[n];
@@ -646,39 +790,42 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             if (j < nj) tmem_ld1(tmem + lane_base + static_cast<uint32_t>((j0 + j) * p.Rs + n), raw[j]);
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
-            const int v = (t_lo + j0 + j) * kTileV + q4 * 32 + lane;
-            qv[j] = (j < nj && qrow && v < p.V) ? qrow[v] : 0.f;
+            const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
+            qv[j] = (j < nj && qrow && v < v_hi) ? qrow[v] : 0.f;
           }
           tmem_wait_ld();
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
-            const int v = (t_lo + j0 + j) * kTileV + q4 * 32 + lane;
-            double rv = 0.0;
-            if (j < nj && v < p.V) {
-              const double pv = static_cast<double>(expf(__uint_as_float(raw[j]) - M) * invS);
-              rv = qrow ? fmax(0.0, pv - static_cast<double>(qv[j])) : pv;
+            const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
+            float rv = 0.f;
+            if (j < nj && v < v_hi) {
+              const float pv = expf(__uint_as_float(raw[j]) - M) * invS;
+              rv = qrow ? fmaxf(0.f, pv - qv[j]) : pv;
             }
-            rv = warp_sum_d(rv);
-            if (lane == 0 && j < nj) s_tw[(j0 + j) * kEpiWarps + q4] = rv;
+            const ff2 seg = warp_sum_ff(ff2{rv, 0.f});
+            if (lane == 0 && j < nj) s_tw[(j0 + j) * kEpiWarps + q4] = make_float2(seg.hi, seg.lo);
           }
         }
         named_bar(1, kEpiWarps * 32);
         // (2) the segment holding the target, in vocabulary order.
         if (ew == 0 && lane == 0) {
-          double run = 0.0, tgt = s_T[b];
+          ff2 run{0.f, 0.f};
+          const ff2 tgt0{s_T[b].x, s_T[b].y};
+          ff2 tgt = tgt0;
           int jt = -1, qt = -1, jl = -1, ql = -1;
           for (int j = 0; j < ntiles && jt < 0; ++j) {
             for (int q = 0; q < kEpiWarps; ++q) {
-              const double mseg = s_tw[j * kEpiWarps + q];
-              if (mseg > 0.0) { jl = j; ql = q; }
-              if (run + mseg > tgt && mseg > 0.0) { jt = j; qt = q; tgt -= run; break; }
-              run += mseg;
+              const ff2 mseg{s_tw[j * kEpiWarps + q].x, s_tw[j * kEpiWarps + q].y};
+              if (mseg.hi > 0.f) { jl = j; ql = q; }
+              const ff2 reach = ff_add(run, mseg);
+              if (mseg.hi > 0.f && ff_gt(reach, tgt0)) { jt = j; qt = q; tgt = ff_sub(tgt0, run); break; }
+              run = reach;
             }
           }
-          if (jt < 0) { jt = jl; qt = ql; tgt = 1e300; }  // rounding: clamp to the last mass
+          if (jt < 0) { jt = jl; qt = ql; tgt = ff2{INFINITY, 0.f}; }  // rounding: clamp to the last mass
           s_seg[0] = jt;
           s_seg[1] = qt;
-          s_T[b] = tgt;
+          s_T[b] = make_float2(tgt.hi, tgt.lo);
         }
         named_bar(1, kEpiWarps * 32);
         // (3) the warp owning that segment scans its 32 entries.
@@ -686,22 +833,18 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         if (jt >= 0 && q4 == qt) {
           uint32_t raw;
           tmem_ld1(tmem + lane_base + static_cast<uint32_t>(jt * p.Rs + n), raw);
-          const int v = (t_lo + jt) * kTileV + q4 * 32 + lane;
-          const float qv = (qrow && v < p.V) ? qrow[v] : 0.f;
+          const int v = v_lo + jt * kTileV + q4 * 32 + lane;
+          const float qv = (qrow && v < v_hi) ? qrow[v] : 0.f;
           tmem_wait_ld();
-          double rv = 0.0;
-          if (v < p.V) {
-            const double pv = static_cast<double>(expf(__uint_as_float(raw) - M) * invS);
-            rv = qrow ? fmax(0.0, pv - static_cast<double>(qv)) : pv;
+          float rv = 0.f;
+          if (v < v_hi) {
+            const float pv = expf(__uint_as_float(raw) - M) * invS;
+            rv = qrow ? fmaxf(0.f, pv - qv) : pv;
           }
-          double incl = rv;
-#pragma unroll
-          for (int o = 1; o < 32; o <<= 1) {
-            const double t = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += t;
-          }
-          const unsigned hit = __ballot_sync(0xffffffffu, incl > s_T[b] && rv > 0.0);
-          const unsigned pos = __ballot_sync(0xffffffffu, rv > 0.0);
+          const ff2 incl = warp_scan_ff(ff2{rv, 0.f}, lane);
+          const ff2 tgt{s_T[b].x, s_T[b].y};
+          const unsigned hit = __ballot_sync(0xffffffffu, rv > 0.f && ff_gt(incl, tgt));
+          const unsigned pos = __ballot_sync(0xffffffffu, rv > 0.f);
           if (lane == 0) {
             const int l = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : 0);
             p.next_token[b] = v + l;
@@ -716,7 +859,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
 
   // ---- teardown: every TMEM access above has completed --------------------
   tc_fence_before();
-  __syncthreads();
+  block_sync();
   if (warp == 1) {
     // No MMA may still write TMEM when it is released (matters only after an
     // expired wait; otherwise the epilogue already consumed the last round).
@@ -757,10 +900,25 @@ static Plan make_plan(int R, int V, int sms) {
   return pl;
 }
 
+// Slices are V/NC rows (floor or ceil); returns the tiles of the longest slice
+// and the box rows (multiple of 8, < 128) that cover every partial last tile,
+// or 128 when no slice ends in a tile short enough to be worth a short box.
+static void slice_shape(int V, int NC, int *tiles_max, int *brs) {
+  const int lmin = V / NC, lmax = lmin + (V % NC ? 1 : 0);
+  *tiles_max = (lmax + kTileV - 1) / kTileV;
+  int last = 0;
+  for (int L : {lmin, lmax}) {
+    const int rows = L - ((L + kTileV - 1) / kTileV - 1) * kTileV;
+    if (rows < kTileV && rows > last) last = rows;
+  }
+  *brs = last == 0 ? kTileV : (last + 7) / 8 * 8;
+}
+
 static size_t workspace_bytes_for(int B, int R, int NC) {
   size_t off = 256;                                        // barrier words
   off += round_up(static_cast<size_t>(NC) * R * 16, 256);  // pstat
   off += round_up(static_cast<size_t>(R) * 4, 256);        // ldraft
+  off += round_up(static_cast<size_t>(R) * 16, 256);       // gstat
   off += round_up(static_cast<size_t>(NC) * B * 16, 256);  // zpart
   return off;
 }
@@ -851,7 +1009,8 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
   p.T = pl.T; p.NC = pl.NC; p.Ncols = pl.Ncols; p.Rs = pl.Rs;
   p.KC = (H + kKChunk - 1) / kKChunk;
   p.KCF = H / kKChunk;
-  const int tiles_max = (pl.T + pl.NC - 1) / pl.NC;
+  int tiles_max = 0;
+  slice_shape(V, pl.NC, &tiles_max, &p.BRS);
   if (tiles_max > kMaxTilesPerCta)
     return fail(SPADE_ERR_SHAPE, "vocabulary %d needs %d tiles per SM (max %d)", V, tiles_max, kMaxTilesPerCta);
   if (!plan_rounds(tiles_max, pl.Ncols, pl.Rs, p.round_tiles, &p.nrounds))
@@ -861,7 +1020,7 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
   p.idesc = idesc_bf16_f32(kTileV, pl.Ncols);
   p.tmem_cols = kTmemCols;
   // Two k-chunks per stage (32 KB W boxes) while the rings fit in shared memory.
-  p.HS = 2;
+  p.HS = 3;
   p.KG = 2;
   for (;;) {
     Params probe = p;
@@ -885,12 +1044,15 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
   off += round_up(static_cast<size_t>(pl.NC) * R * 16, 256);
   p.ldraft = reinterpret_cast<float *>(ws + off);
   off += round_up(static_cast<size_t>(R) * 4, 256);
-  p.zpart = reinterpret_cast<double2 *>(ws + off);
+  p.gstat = reinterpret_cast<float4 *>(ws + off);
+  off += round_up(static_cast<size_t>(R) * 16, 256);
+  p.zpart = reinterpret_cast<float4 *>(ws + off);
 
   // 2-D views (one k-chunk per box, zero fill past H) serve a ragged last
   // k-chunk; 3-D views fetch KG full k-chunks per box.
-  CUtensorMap tw2, th2, tw3, th3;
+  CUtensorMap tw2, tw2s, th2, tw3, th3;
   if (!encode_tmap_bf16_sw128(&tw2, w_lm, H, V, static_cast<uint64_t>(H) * 2, kKChunk, kTileV) ||
+      !encode_tmap_bf16_sw128(&tw2s, w_lm, H, V, static_cast<uint64_t>(H) * 2, kKChunk, p.BRS) ||
       !encode_tmap_bf16_sw128(&th2, hidden, H, R, static_cast<uint64_t>(H) * 2, kKChunk, pl.Ncols))
     return SPADE_ERR_CUDA;
   if (p.KCF >= 1) {
@@ -921,7 +1083,7 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, verify_accept_kernel, p, tw3, tw2, th3, th2);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, verify_accept_kernel, p, tw3, tw2, tw2s, th3, th2);
   if (e != cudaSuccess) return cuda_fail(e, "verify_accept cooperative launch");
   return SPADE_OK;
 }

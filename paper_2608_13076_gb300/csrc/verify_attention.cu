@@ -138,8 +138,16 @@ __device__ __forceinline__ Seg locate(const Sched &s, int64_t x) {
   return g;
 }
 
+// bar.sync is the aligned form: every lane of a warp must arrive together.
+// Lanes that ran ahead of a divergent lane (a lane-0-only loop) reconverge
+// first, so no warp reaches the barrier before all of its lanes do.
 __device__ __forceinline__ void named_bar(int id, int threads) {
+  __syncwarp();
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+__device__ __forceinline__ void block_sync() {
+  __syncwarp();
+  __syncthreads();
 }
 
 // Byte offset of 16-byte chunk `c` (0..D/8-1) of row `r` inside a K/V stage
@@ -181,7 +189,7 @@ __global__ void __launch_bounds__(Layout<D, MT>::THREADS, 1)
     s_ctx[b] = c;
     s_kd[b] = bad ? -1 : k;
   }
-  __syncthreads();
+  block_sync();
   Sched sc;
   sc.pref = s_pref; sc.ctx = s_ctx; sc.kd = s_kd;
   sc.B = p.B; sc.Hkv = p.Hkv; sc.G = p.G; sc.RB = p.RB; sc.num_ctas = p.num_ctas;
@@ -213,7 +221,7 @@ __global__ void __launch_bounds__(Layout<D, MT>::THREADS, 1)
     }
     fence_mbar_init();
   }
-  __syncthreads();
+  block_sync();
   sc.total = s_pref[p.B];
   if (sc.total == 0) return;
   // Never more CTAs than chunks: every CTA kept has a non-empty range, so the
