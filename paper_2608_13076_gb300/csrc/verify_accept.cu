@@ -80,7 +80,7 @@ struct Params {
 
 struct Smem {
   int w_slot, h_slot;
-  int off_h, off_bar, off_misc, off_rows, off_wst, off_tbuf, total;
+  int off_h, off_bar, off_misc, off_rows, off_tbuf, total;
 };
 
 __host__ __device__ inline Smem smem_layout(const Params &p) {
@@ -91,9 +91,10 @@ __host__ __device__ inline Smem smem_layout(const Params &p) {
   s.off_bar = s.off_h + p.HS * s.h_slot;
   s.off_misc = s.off_bar + (2 * p.WS + 2 * p.HS + 2) * 8;
   s.off_rows = s.off_misc + 64;  // int/float [5][kMaxR] + int [3][kMaxB + 1]
-  s.off_wst = s.off_rows + 5 * kMaxR * 4 + 3 * (kMaxB + 1) * 4 + 4;  // float4 [kEpiWarps][R]
-  s.off_tbuf = s.off_wst + kEpiWarps * p.R * 16;    // float [kEpiWarps][16][32]
-  s.total = s.off_tbuf + kEpiWarps * 16 * 32 * 4 + 1024;
+  // Per epilogue warp a 32 x 33 float transpose buffer; after the last round
+  // the same bytes hold the warps' per-row statistics (float4 [kEpiWarps][R]).
+  s.off_tbuf = s.off_rows + 5 * kMaxR * 4 + 3 * (kMaxB + 1) * 4 + 4;
+  s.total = s.off_tbuf + kEpiWarps * 32 * 33 * 4 + 1024;
   return s;
 }
 
@@ -218,51 +219,6 @@ __device__ __forceinline__ ff2 warp_scan_ff(ff2 v, int lane) {
   return v;
 }
 
-// Per-row running statistics of one epilogue warp: the 8 rows c8*8..c8*8+7 of
-// the 32 vocab entries held in registers by the warp's lanes.
-__device__ __forceinline__ void reduce_rows8(const uint32_t *raw, int c8, int vlane0, int vlimit,
-                                             int lane, const Params &p, const int32_t *s_draft,
-                                             float *tbuf, float4 *wst) {
-#pragma unroll
-  for (int e = 0; e < 8; ++e) tbuf[e * 32 + lane] = __uint_as_float(raw[e]);
-  __syncwarp();
-  const int r = lane >> 2, part = lane & 3;
-  const int n = c8 * 8 + r;
-  const float4 lo = *reinterpret_cast<const float4 *>(tbuf + r * 32 + part * 8);
-  const float4 hi = *reinterpret_cast<const float4 *>(tbuf + r * 32 + part * 8 + 4);
-  float x[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
-  const int v0 = vlane0 + part * 8;  // vocab id of x[0]
-  const int d = (n < p.R) ? s_draft[n] : -1;
-  float m = -INFINITY;
-  int mi = INT_MAX;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    if (v0 + i >= vlimit) x[i] = -INFINITY;        // lanes past this CTA's slice
-    else if (v0 + i == d) p.ldraft[n] = x[i];      // only the slice owner writes
-    if (x[i] > m) { m = x[i]; mi = v0 + i; }
-  }
-  float s = 0.f;
-  if (m != -INFINITY) {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) s += ex2((x[i] - m) * kLog2e);
-  }
-#pragma unroll
-  for (int o = 1; o <= 2; o <<= 1) {
-    const float om = __shfl_xor_sync(0xffffffffu, m, o);
-    const float os = __shfl_xor_sync(0xffffffffu, s, o);
-    const int oi = __shfl_xor_sync(0xffffffffu, mi, o);
-    stat_merge(m, s, mi, om, os, oi);
-  }
-  __syncwarp();
-  if (part == 0 && n < p.R) {
-    float4 st = wst[n];
-    int si = __float_as_int(st.z);
-    stat_merge(st.x, st.y, si, m, s, mi);
-    st.z = __int_as_float(si);
-    wst[n] = st;
-  }
-}
-
 __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tm_w3,
     const __grid_constant__ CUtensorMap tm_w2, const __grid_constant__ CUtensorMap tm_w2s,
@@ -290,8 +246,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   int32_t *s_cuq = reinterpret_cast<int32_t *>(s_qd + kMaxR);
   int32_t *s_nd = s_cuq + kMaxB + 1;
   int32_t *s_md = s_nd + kMaxB;
-  float4 *s_wst = reinterpret_cast<float4 *>(smem + L.off_wst);
   float *s_tbuf = reinterpret_cast<float *>(smem + L.off_tbuf);
+  float4 *s_wst = reinterpret_cast<float4 *>(smem + L.off_tbuf);  // after the last round
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c = blockIdx.x;
@@ -453,9 +409,12 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     const int ew = warp - 2;             // 0..3
     const int q4 = warp & 3;             // TMEM lane quarter this warp may access
     const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
-    float4 *wst = s_wst + ew * p.R;      // this warp's running stats per row
-    float *tbuf = s_tbuf + ew * 16 * 32;
-    for (int n = lane; n < p.R; n += 32) wst[n] = make_float4(-INFINITY, 0.f, __int_as_float(INT_MAX), 0.f);
+    float *T = s_tbuf + ew * (32 * 33);  // this warp's transpose buffer
+    // Running statistics of rows lane + 32 * j over this warp's vocab entries.
+    float rm[8], rs[8];
+    int ri[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) { rm[j] = -INFINITY; rs[j] = 0.f; ri[j] = INT_MAX; }
     // While the first round accumulates: uniforms and q(draft) of every row.
     for (int n = tid - 64; n < p.R; n += kEpiWarps * 32) {
       s_u[n] = p.uniforms[n];
@@ -479,11 +438,22 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           const uint32_t src = tmem + lane_base + static_cast<uint32_t>(used + j * p.Ncols);
           const uint32_t dst = tmem + lane_base + static_cast<uint32_t>(used + j * p.Rs);
           if (src == dst) continue;
-          for (int c8 = 0; c8 < p.Rs / 8; ++c8) {
-            uint32_t raw[8];
-            tmem_ld8(src + c8 * 8, raw);
+          // 32-column steps, each as four 8-column accesses (TMEM addresses here
+          // are only 8-column aligned) behind one wait.
+          int cc = 0;
+          for (; cc + 32 <= p.Rs; cc += 32) {
+            uint32_t raw[32];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) tmem_ld8(src + cc + 8 * q, raw + 8 * q);
             tmem_wait_ld();
-            tmem_st8(dst + c8 * 8, raw);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) tmem_st8(dst + cc + 8 * q, raw + 8 * q);
+          }
+          for (; cc < p.Rs; cc += 8) {
+            uint32_t raw[8];
+            tmem_ld8(src + cc, raw);
+            tmem_wait_ld();
+            tmem_st8(dst + cc, raw);
           }
         }
         tmem_wait_st();
@@ -491,30 +461,63 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(acc_empty);
+      // Statistics of this round's tiles, 32 rows at a time: one TMEM load gives
+      // each lane (one vocab entry) 32 rows; a 32 x 33 shared-memory transpose
+      // gives each lane one row over the warp's 32 vocab entries, reduced
+      // serially -- no shuffles.
       for (int j = 0; j < nt; ++j) {
         const int t = tdone + j;
         const int vlane0 = v_lo + t * kTileV + q4 * 32;  // vocab id of lane 0's row
+        const bool my_valid = vlane0 + lane < v_hi;       // lanes past the slice are masked
         const uint32_t col = tmem + lane_base + static_cast<uint32_t>(t * p.Rs);
-        int c8 = 0;
-        for (; (c8 + 1) * 8 < p.R; c8 += 2) {
-          uint32_t raw[16];
-          tmem_ld8(col + c8 * 8, raw);
-          tmem_ld8(col + c8 * 8 + 8, raw + 8);
-          tmem_wait_ld();
-          reduce_rows8(raw, c8, vlane0, v_hi, lane, p, s_draft, tbuf, wst);
-          reduce_rows8(raw + 8, c8 + 1, vlane0, v_hi, lane, p, s_draft, tbuf + 256, wst);
-        }
-        if (c8 * 8 < p.R) {
-          uint32_t raw[8];
-          tmem_ld8(col + c8 * 8, raw);
-          tmem_wait_ld();
-          reduce_rows8(raw, c8, vlane0, v_hi, lane, p, s_draft, tbuf, wst);
+#pragma unroll
+        for (int cj = 0; cj < 8; ++cj) {
+          const int r0 = cj * 32;
+          if (r0 < p.R) {
+            const int nc = min(32, p.Rs - r0);  // columns of this chunk (multiple of 8)
+            uint32_t raw[32];
+            // Four 8-column loads (8-column aligned addresses) behind one wait.
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              if (8 * q < nc) tmem_ld8(col + r0 + 8 * q, raw + 8 * q);
+            tmem_wait_ld();
+#pragma unroll
+            for (int rr = 0; rr < 32; ++rr)
+              if (rr < nc) T[lane * 33 + rr] = my_valid ? __uint_as_float(raw[rr]) : -INFINITY;
+            __syncwarp();
+            const int n = r0 + lane;
+            if (lane < nc && n < p.R) {
+              float x[32];
+              float m = -INFINITY;
+              int mi = 0;
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                x[i] = T[i * 33 + lane];
+                if (x[i] > m) { m = x[i]; mi = i; }
+              }
+              float sm = 0.f;
+              if (m != -INFINITY) {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) sm += ex2((x[i] - m) * kLog2e);
+              }
+              stat_merge(rm[cj], rs[cj], ri[cj], m, sm, m == -INFINITY ? INT_MAX : vlane0 + mi);
+              const int d = s_draft[n];
+              if (d >= vlane0 && d < vlane0 + 32 && d < v_hi) p.ldraft[n] = T[(d - vlane0) * 33 + lane];
+            }
+            __syncwarp();
+          }
         }
       }
       used += nt * p.Rs;
       tdone += nt;
     }
     // Merge the four warps' statistics and publish this CTA's slice partials.
+    named_bar(1, kEpiWarps * 32);  // every warp is done with its transpose buffer
+#pragma unroll
+    for (int cj = 0; cj < 8; ++cj) {
+      const int n = cj * 32 + lane;
+      if (n < p.R) s_wst[ew * p.R + n] = make_float4(rm[cj], rs[cj], __int_as_float(ri[cj]), 0.f);
+    }
     named_bar(1, kEpiWarps * 32);
     for (int n = tid - 64; n < p.R; n += kEpiWarps * 32) {
       float m = -INFINITY, s = 0.f;
