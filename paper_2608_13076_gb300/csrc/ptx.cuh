@@ -112,6 +112,16 @@ SPADE_DEVICE void tma_load_2d(void *dst, const CUtensorMap *map, int32_t x, int3
       : "memory");
 }
 
+// 3-D tiled load of box {x, y, z} at coordinates (x, y, z); see tma_load_2d.
+SPADE_DEVICE void tma_load_3d(void *dst, const CUtensorMap *map, int32_t x, int32_t y, int32_t z,
+                              uint64_t *bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+
 // ---------------------------------------------------------------- warp MMA
 SPADE_DEVICE void ldmatrix_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
                               uint32_t &r3) {

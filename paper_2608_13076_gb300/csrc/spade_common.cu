@@ -97,6 +97,36 @@ bool encode_tmap_bf16_sw128(CUtensorMap *map, const void *base, uint64_t inner, 
   return true;
 }
 
+bool encode_tmap_rows_by_slab(CUtensorMap *map, const void *base, uint64_t rows, uint32_t cols,
+                              uint32_t box_rows) {
+  std::call_once(g_encode_once, [] {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<EncodeFn>(fn);
+  });
+  if (!g_encode) {
+    fail(SPADE_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+    return false;
+  }
+  cuuint64_t dims[3] = {64, rows, cols / 64};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(cols) * 2, 128};
+  cuuint32_t box[3] = {64, box_rows, cols / 64};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    fail(SPADE_ERR_CUDA, "cuTensorMapEncodeTiled (row slabs) failed (%d) for [%llu x %u]",
+         static_cast<int>(r), (unsigned long long)rows, cols);
+    return false;
+  }
+  return true;
+}
+
 }  // namespace spade
 
 extern "C" {

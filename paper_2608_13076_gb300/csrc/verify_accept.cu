@@ -116,14 +116,6 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned *p) {
   return v;
 }
 
-__device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, int32_t x,
-                                            int32_t y, int32_t z, uint64_t *bar, uint64_t pol) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "l"(pol)
-      : "memory");
-}
 
 // Device-wide barrier among the NC co-resident CTAs (cooperative launch).  The
 // last CTA to arrive resets the count and bumps the generation; the others

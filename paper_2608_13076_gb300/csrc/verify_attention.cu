@@ -251,11 +251,9 @@ __global__ void __launch_bounds__(Layout<D, MT>::THREADS, 1)
           uint8_t *kt = smem + s * L::STAGE_BYTES;
           uint8_t *vt = kt + L::TILE_BYTES;
           mbar_arrive_expect_tx(&full_bar[s], L::STAGE_BYTES);
-#pragma unroll
-          for (int bx = 0; bx < L::BOXES; ++bx) {
-            tma_load_2d(kt + bx * kChunk * 128, &tm_k, bx * 64, row0 + ci * kChunk, &full_bar[s], pol);
-            tma_load_2d(vt + bx * kChunk * 128, &tm_v, bx * 64, row0 + ci * kChunk, &full_bar[s], pol);
-          }
+          // One box per tile: 64 keys x all of D, landing as [D/64][64 keys][64].
+          tma_load_3d(kt, &tm_k, 0, row0 + ci * kChunk, 0, &full_bar[s], pol);
+          tma_load_3d(vt, &tm_v, 0, row0 + ci * kChunk, 0, &full_bar[s], pol);
           issued = it + 1;
         }
       }
@@ -679,8 +677,8 @@ extern "C" spade_status spade_verify_attention(
 
   CUtensorMap tk, tv;
   const uint64_t rows = static_cast<uint64_t>(B) * Hkv * cap;
-  if (!encode_tmap_bf16_sw128(&tk, k_cache, D, rows, static_cast<uint64_t>(D) * 2, 64, attn::kChunk) ||
-      !encode_tmap_bf16_sw128(&tv, v_cache, D, rows, static_cast<uint64_t>(D) * 2, 64, attn::kChunk))
+  if (!encode_tmap_rows_by_slab(&tk, k_cache, rows, D, attn::kChunk) ||
+      !encode_tmap_rows_by_slab(&tv, v_cache, rows, D, attn::kChunk))
     return SPADE_ERR_CUDA;
 
   const int mt = (G * (max_k + 1) >= attn::kRowBlock) ? 4 : (G * (max_k + 1) + 15) / 16;
