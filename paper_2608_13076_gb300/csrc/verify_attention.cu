@@ -553,42 +553,84 @@ __global__ void __launch_bounds__(Layout<D, MT>::THREADS, 1)
       named_bar(1, NT);
       if (*s_last) {
         // This CTA finished the unit last: merge every partial by log-sum-exp.
+        // Online merge, two rows per warp step, the loads of up to kBatch
+        // partials per row in flight together.
         const int64_t slot0 = c_first + unit;
         constexpr int PER = D / 32;
-        for (int rl = cw; rl < nrow; rl += L::NW) {
-          float M = -INFINITY;
-          for (int s2 = 0; s2 < nparts; ++s2)
-            M = fmaxf(M, __ldcg(p.partials + (slot0 + s2) * slot_floats(D) + kRowBlock * D + rl));
-          const float U = (M == -INFINITY) ? 0.f : M;
-          float acc[PER];
+        constexpr int kBatch = 4;
+        for (int rl0 = 2 * cw; rl0 < nrow; rl0 += 2 * L::NW) {
+          float M[2] = {-INFINITY, -INFINITY}, Lsum[2] = {0.f, 0.f};
+          float acc[2][PER];
 #pragma unroll
-          for (int e = 0; e < PER; ++e) acc[e] = 0.f;
-          float Lsum = 0.f;
-          for (int s2 = 0; s2 < nparts; ++s2) {
-            const float *ps = p.partials + (slot0 + s2) * slot_floats(D);
-            const float w = ex2(__ldcg(ps + kRowBlock * D + rl) - U);
-            Lsum += w * __ldcg(ps + kRowBlock * D + kRowBlock + rl);
-            if constexpr (PER == 4) {
-              const float4 v = __ldcg(reinterpret_cast<const float4 *>(ps + rl * D + lane * 4));
-              acc[0] += w * v.x; acc[1] += w * v.y; acc[2] += w * v.z; acc[3] += w * v.w;
-            } else {
-              const float2 v = __ldcg(reinterpret_cast<const float2 *>(ps + rl * D + lane * 2));
-              acc[0] += w * v.x; acc[1] += w * v.y;
+          for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int e = 0; e < PER; ++e) acc[h][e] = 0.f;
+          for (int s0 = 0; s0 < nparts; s0 += kBatch) {
+            float mv[2][kBatch], lv[2][kBatch], ov[2][kBatch][PER];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const int rl = min(rl0 + h, nrow - 1);
+#pragma unroll
+              for (int j = 0; j < kBatch; ++j) {
+                if (s0 + j < nparts) {
+                  const float *ps = p.partials + (slot0 + s0 + j) * slot_floats(D);
+                  mv[h][j] = __ldcg(ps + kRowBlock * D + rl);
+                  lv[h][j] = __ldcg(ps + kRowBlock * D + kRowBlock + rl);
+                  if constexpr (PER == 4) {
+                    const float4 v = __ldcg(reinterpret_cast<const float4 *>(ps + rl * D + lane * 4));
+                    ov[h][j][0] = v.x; ov[h][j][1] = v.y; ov[h][j][2] = v.z; ov[h][j][3] = v.w;
+                  } else {
+                    const float2 v = __ldcg(reinterpret_cast<const float2 *>(ps + rl * D + lane * 2));
+                    ov[h][j][0] = v.x; ov[h][j][1] = v.y;
+                  }
+                } else {
+                  mv[h][j] = -INFINITY;
+                  lv[h][j] = 0.f;
+#pragma unroll
+                  for (int e = 0; e < PER; ++e) ov[h][j][e] = 0.f;
+                }
+              }
+            }
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              float Mn = M[h];
+#pragma unroll
+              for (int j = 0; j < kBatch; ++j) Mn = fmaxf(Mn, mv[h][j]);
+              const float U = (Mn == -INFINITY) ? 0.f : Mn;
+              const float f = ex2(M[h] - U);
+              Lsum[h] *= f;
+#pragma unroll
+              for (int e = 0; e < PER; ++e) acc[h][e] *= f;
+#pragma unroll
+              for (int j = 0; j < kBatch; ++j) {
+                const float w = ex2(mv[h][j] - U);
+                Lsum[h] += w * lv[h][j];
+#pragma unroll
+                for (int e = 0; e < PER; ++e) acc[h][e] += w * ov[h][j][e];
+              }
+              M[h] = Mn;
             }
           }
-          const int row = kRowBlock * g.rb + rl;
-          const int i = row / p.G, gh = row % p.G;
-          const size_t orow = static_cast<size_t>(q_row0 + i) * p.Hq + g.kvh * p.G + gh;
-          const float inv = 1.f / Lsum;
-          if constexpr (PER == 4) {
-            uint2 v;
-            v.x = pack_bf16(acc[0] * inv, acc[1] * inv);
-            v.y = pack_bf16(acc[2] * inv, acc[3] * inv);
-            *reinterpret_cast<uint2 *>(p.out + orow * D + lane * 4) = v;
-          } else {
-            *reinterpret_cast<uint32_t *>(p.out + orow * D + lane * 2) = pack_bf16(acc[0] * inv, acc[1] * inv);
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int rl = rl0 + h;
+            if (rl < nrow) {
+              const int row = kRowBlock * g.rb + rl;
+              const int i = row / p.G, gh = row % p.G;
+              const size_t orow = static_cast<size_t>(q_row0 + i) * p.Hq + g.kvh * p.G + gh;
+              const float inv = 1.f / Lsum[h];
+              if constexpr (PER == 4) {
+                uint2 v;
+                v.x = pack_bf16(acc[h][0] * inv, acc[h][1] * inv);
+                v.y = pack_bf16(acc[h][2] * inv, acc[h][3] * inv);
+                *reinterpret_cast<uint2 *>(p.out + orow * D + lane * 4) = v;
+              } else {
+                *reinterpret_cast<uint32_t *>(p.out + orow * D + lane * 2) =
+                    pack_bf16(acc[h][0] * inv, acc[h][1] * inv);
+              }
+              if (p.lse && lane == 0) p.lse[orow] = (M[h] + log2f(Lsum[h])) * 0.69314718055994531f;
+            }
           }
-          if (p.lse && lane == 0) p.lse[orow] = (M + log2f(Lsum)) * 0.69314718055994531f;
         }
         if (ctid == 0) p.counters[unit] = 0;  // every part has arrived: reset for the next call
       }
