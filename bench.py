@@ -49,6 +49,20 @@ def _peaks():
         return 6800.0, 1900.0, 1700.0, "fallback"
 
 
+def _traffic(kernel, workload):
+    """ncu DRAM bytes per launch for this kernel and workload, if the kernel source is unchanged."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            rec = json.load(f)[kernel][workload]
+        with open(os.path.join(ROOT, rec["source"]), "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest()[:16] != rec["sha256_16"]:
+                return None
+        return rec["bytes"]
+    except Exception:
+        return None
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -250,11 +264,13 @@ def run_spade(args, ws, rank, local):
     m_acc = statistics.mean(t_acc)
     m_attn = statistics.mean(t_attn)
     roof_lm = {"kernel": "verify_accept_kernel", "bound": "hbm", "achieved": lm_bytes / m_acc / 1e9,
-               "peak": hbm, "unit": "GB/s", "frac": lm_bytes / m_acc / 1e9 / hbm, "traffic": None,
+               "peak": hbm, "unit": "GB/s", "frac": lm_bytes / m_acc / 1e9 / hbm,
+               "traffic": _traffic("verify_accept_kernel", args.workload),
                "algorithmic_bytes": lm_bytes, "peak_source": peak_src,
                "tensor_tflops": lm_flop / m_acc / 1e12, "tensor_frac_of_bf16_peak": lm_flop / m_acc / 1e12 / bf16}
     roof_attn = {"kernel": "verify_attention_kernel", "bound": "hbm", "achieved": attn_bytes / m_attn / 1e9,
-                 "peak": hbm, "unit": "GB/s", "frac": attn_bytes / m_attn / 1e9 / hbm, "traffic": None,
+                 "peak": hbm, "unit": "GB/s", "frac": attn_bytes / m_attn / 1e9 / hbm,
+                 "traffic": _traffic("verify_attention_kernel", args.workload),
                  "algorithmic_bytes": attn_bytes, "peak_source": peak_src,
                  "tflops": attn_flop / m_attn / 1e12}
     dominant = roof_lm if m_acc >= m_attn else roof_attn
