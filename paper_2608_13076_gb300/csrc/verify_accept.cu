@@ -41,12 +41,20 @@ constexpr int kTileV = 128;    // vocab rows per tile (MMA M)
 constexpr int kKChunk = 64;    // K elements per 128-byte swizzle row
 constexpr int kEpiWarps = 4;
 constexpr int kThreads = 32 * (2 + kEpiWarps);
-constexpr int kMaxR = 256;     // verify rows per call on the resident path (MMA N <= 256)
+constexpr int kMaxRes = 256;   // rows kept resident in TMEM (MMA N <= 256)
+constexpr int kMaxR = 512;     // verify rows per call (two-pass path above kMaxRes)
 constexpr int kMaxB = 256;
-constexpr int kMaxRounds = 8;
+constexpr int kMaxRounds = 32;
+// Kernel kinds.  kResident: the whole step in one launch, logits resident in
+// TMEM.  kStatsOnly: first pass for more rows than TMEM holds -- statistics and
+// accept decisions only; the rows to sample are gathered into the workspace.
+// kPresampled: second pass, resident, on the gathered rows with the decisions
+// already taken.
+constexpr int kResident = 0, kStatsOnly = 1, kPresampled = 2;
 constexpr int kMaxTilesPerCta = 32;
 constexpr int kTmemCols = 512;
-constexpr int kSmemBudget = 216 * 1024;
+constexpr int kSmemBudget = 220 * 1024;
+constexpr int kSmemMax = 225 * 1024;  // opt-in limit (227 KB) minus static shared memory
 constexpr int kWChunkBytes = kTileV * kKChunk * 2;  // 16 KB: one tile x one k-chunk
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -65,6 +73,16 @@ struct Params {
   float *ldraft;     // [R]: logit of the row's draft token
   float4 *gstat;     // [R]: merged row max, sum-exp, argmax (bits)
   float4 *zpart;     // [NC][B]: slice mass of the sampled distribution and of p (float-float)
+  int4 *samp;        // [B]: sample specs written by kStatsOnly, read by kPresampled:
+                     //      draft_probs row (-1: sample p), uniform bits, output index, row
+  int *samp_count;   // number of specs
+  __nv_bfloat16 *hidden_s;      // [B, H]: gathered hidden rows of the samples
+  const __nv_bfloat16 *hidden;  // the call's hidden rows (gather source)
+  int kind;
+  int nchunks;       // MMA N-chunks per tile (2 when Ncols > 256)
+  int n0w;           // width of the first N-chunk
+  uint32_t idesc1;   // instruction descriptor of the second N-chunk
+  int h_box_rows, h_boxes;  // hidden rows per TMA box, boxes per k-chunk
   int B, R, H, V, T, NC, Ncols, Rs;
   int KC;            // k-chunks of 64 (the last may be partial)
   int KCF;           // full k-chunks (H / 64)
@@ -86,7 +104,7 @@ struct Smem {
 __host__ __device__ inline Smem smem_layout(const Params &p) {
   Smem s;
   s.w_slot = p.KG * kWChunkBytes;
-  s.h_slot = p.KG * p.Ncols * 128;
+  s.h_slot = p.KG * p.h_boxes * p.h_box_rows * 128;
   s.off_h = p.WS * s.w_slot;
   s.off_bar = s.off_h + p.HS * s.h_slot;
   s.off_misc = s.off_bar + (2 * p.WS + 2 * p.HS + 2) * 8;
@@ -94,7 +112,8 @@ __host__ __device__ inline Smem smem_layout(const Params &p) {
   // Per epilogue warp a 32 x 33 float transpose buffer; after the last round
   // the same bytes hold the warps' per-row statistics (float4 [kEpiWarps][R]).
   s.off_tbuf = s.off_rows + 5 * kMaxR * 4 + 3 * (kMaxB + 1) * 4 + 4;
-  s.total = s.off_tbuf + kEpiWarps * 32 * 33 * 4 + 1024;
+  const int tbuf = kEpiWarps * 32 * 33 * 4, wst = kEpiWarps * p.R * 16;
+  s.total = s.off_tbuf + (tbuf > wst ? tbuf : wst) + 1024;
   return s;
 }
 
@@ -249,6 +268,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   const int v_hi = static_cast<int>(static_cast<int64_t>(c + 1) * p.V / p.NC);
   const int ntiles = (v_hi - v_lo + kTileV - 1) / kTileV;
   const bool short_last = (v_hi - v_lo) - (ntiles - 1) * kTileV <= p.BRS && p.BRS < kTileV;
+  // Second pass with nothing to sample: the whole grid leaves before any set-up.
+  if (p.kind == kPresampled && *p.samp_count == 0) return;
 
   // ---- set-up: barriers, TMEM, per-row bookkeeping -------------------------
   if (tid == 0) {
@@ -267,6 +288,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   for (int n = tid; n < kMaxR; n += kThreads) { s_draft[n] = -1; s_seq[n] = -1; s_pos[n] = 0; }
   block_sync();
   // Row n = cu_q[b] + i is position i of sequence b; it holds draft i for i < k_b.
+  if (p.kind != kPresampled) {
   for (int b = tid; b <= p.B; b += kThreads) s_cuq[b] = p.cu_q[b];
   for (int b = tid; b < p.B; b += kThreads) {
     s_nd[b] = p.n_draft[b];
@@ -283,6 +305,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       s_pos[r0 + i] = i;
       if (i < k) s_draft[r0 + i] = p.draft_tokens[r0 - b + i];
     }
+  }
   }
   tc_fence_before();
   block_sync();
@@ -310,12 +333,15 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             mbar_wait(&h_empty[s], ((hi / p.HS) & 1) ^ 1, s_abort);
             if (!*s_abort) {
               uint8_t *dst = h_ring + s * L.h_slot;
-              mbar_arrive_expect_tx(&h_full[s], nch * p.Ncols * 128);
-              if (box3) {
+              const int hk = p.h_boxes * p.h_box_rows * 128;  // bytes per k-chunk
+              mbar_arrive_expect_tx(&h_full[s], nch * hk);
+              if (box3 && p.h_boxes == 1) {
                 tma_load_3d(dst, &tm_h3, 0, 0, c0, &h_full[s], pol_h);
               } else {
                 for (int j = 0; j < nch; ++j)
-                  tma_load_2d(dst + j * p.Ncols * 128, &tm_h2, (c0 + j) * kKChunk, 0, &h_full[s], pol_h);
+                  for (int bi = 0; bi < p.h_boxes; ++bi)
+                    tma_load_2d(dst + j * hk + bi * p.h_box_rows * 128, &tm_h2, (c0 + j) * kKChunk,
+                                bi * p.h_box_rows, &h_full[s], pol_h);
               }
               h_issued = hi + 1;
             }
@@ -376,12 +402,17 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             tc_fence_after();
             const uint32_t w_addr = smem_u32(w_ring + ws * L.w_slot);
             const uint32_t d_tmem = tmem + static_cast<uint32_t>(used + j * p.Ncols);
+            const int hk = p.h_boxes * p.h_box_rows * 128;
             for (int jj = 0; jj < nch; ++jj) {
+              for (int ci = 0; ci < p.nchunks; ++ci) {
+                // N-chunk ci: TMEM columns and hidden rows from noff on.
+                const uint32_t noff = ci ? static_cast<uint32_t>(p.n0w) : 0u;
 #pragma unroll
-              for (int k16 = 0; k16 < kKChunk / 16; ++k16) {
-                tc_mma_f16(d_tmem, smem_desc_sw128(w_addr + jj * kWChunkBytes + 32 * k16),
-                           smem_desc_sw128(h_addr + jj * p.Ncols * 128 + 32 * k16), p.idesc,
-                           (ks | jj | k16) != 0);
+                for (int k16 = 0; k16 < kKChunk / 16; ++k16) {
+                  tc_mma_f16(d_tmem + noff, smem_desc_sw128(w_addr + jj * kWChunkBytes + 32 * k16),
+                             smem_desc_sw128(h_addr + jj * hk + noff * 128 + 32 * k16),
+                             ci ? p.idesc1 : p.idesc, (ks | jj | k16) != 0);
+                }
               }
             }
             tc_commit(&w_empty[ws]);
@@ -392,7 +423,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         }
         tc_commit(acc_full);
         ++rounds_issued;
-        used += nt * p.Rs;
+        if (p.kind != kStatsOnly) used += nt * p.Rs;  // statistics-only: one slot, reused
         tdone += nt;
       }
     }
@@ -403,12 +434,13 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
     float *T = s_tbuf + ew * (32 * 33);  // this warp's transpose buffer
     // Running statistics of rows lane + 32 * j over this warp's vocab entries.
-    float rm[8], rs[8];
-    int ri[8];
+    constexpr int kRC = kMaxR / 32;  // 32-row chunks
+    float rm[kRC], rs[kRC];
+    int ri[kRC];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) { rm[j] = -INFINITY; rs[j] = 0.f; ri[j] = INT_MAX; }
+    for (int j = 0; j < kRC; ++j) { rm[j] = -INFINITY; rs[j] = 0.f; ri[j] = INT_MAX; }
     // While the first round accumulates: uniforms and q(draft) of every row.
-    for (int n = tid - 64; n < p.R; n += kEpiWarps * 32) {
+    for (int n = tid - 64; p.kind != kPresampled && n < p.R; n += kEpiWarps * 32) {
       s_u[n] = p.uniforms[n];
       const int b = s_seq[n], d = s_draft[n];
       float qd = 0.f;
@@ -425,7 +457,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       // Compaction: this round's tiles move from stride Ncols to stride Rs, so
       // tile t of the slice ends at column t * Rs and the next round's MMAs
       // may start at once in the columns after it.
-      if (p.Ncols != p.Rs) {
+      if (p.kind != kStatsOnly && p.Ncols != p.Rs) {
         for (int j = 0; j < nt; ++j) {
           const uint32_t src = tmem + lane_base + static_cast<uint32_t>(used + j * p.Ncols);
           const uint32_t dst = tmem + lane_base + static_cast<uint32_t>(used + j * p.Rs);
@@ -450,9 +482,11 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         }
         tmem_wait_st();
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(acc_empty);
+      if (p.kind != kStatsOnly) {
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acc_empty);
+      }
       // Statistics of this round's tiles, 32 rows at a time: one TMEM load gives
       // each lane (one vocab entry) 32 rows; a 32 x 33 shared-memory transpose
       // gives each lane one row over the warp's 32 vocab entries, reduced
@@ -461,9 +495,9 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         const int t = tdone + j;
         const int vlane0 = v_lo + t * kTileV + q4 * 32;  // vocab id of lane 0's row
         const bool my_valid = vlane0 + lane < v_hi;       // lanes past the slice are masked
-        const uint32_t col = tmem + lane_base + static_cast<uint32_t>(t * p.Rs);
+        const uint32_t col = tmem + lane_base + static_cast<uint32_t>(p.kind == kStatsOnly ? 0 : t * p.Rs);
 #pragma unroll
-        for (int cj = 0; cj < 8; ++cj) {
+        for (int cj = 0; cj < kRC; ++cj) {
           const int r0 = cj * 32;
           if (r0 < p.R) {
             const int nc = min(32, p.Rs - r0);  // columns of this chunk (multiple of 8)
@@ -500,13 +534,20 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           }
         }
       }
-      used += nt * p.Rs;
+      if (p.kind == kStatsOnly) {
+        // The accumulator slot is read: the next tile may overwrite it.
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acc_empty);
+      } else {
+        used += nt * p.Rs;
+      }
       tdone += nt;
     }
     // Merge the four warps' statistics and publish this CTA's slice partials.
     named_bar(1, kEpiWarps * 32);  // every warp is done with its transpose buffer
 #pragma unroll
-    for (int cj = 0; cj < 8; ++cj) {
+    for (int cj = 0; cj < kRC; ++cj) {
       const int n = cj * 32 + lane;
       if (n < p.R) s_wst[ew * p.R + n] = make_float4(rm[cj], rs[cj], __int_as_float(ri[cj]), 0.f);
     }
@@ -571,7 +612,10 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   int *s_owner = s_rstar + kMaxB;                           // [B]
   int *s_usep = s_owner + kMaxB;                            // [B]
   int *s_stoch = s_usep + kMaxB;                            // [B]
-  int *s_seg = s_stoch + kMaxB;                             // [2]: tile, quarter
+  int *s_qidx = s_stoch + kMaxB;                            // [B] draft_probs row, -1: p
+  float *s_usmp = reinterpret_cast<float *>(s_qidx + kMaxB); // [B] sampling uniform
+  int *s_outb = reinterpret_cast<int *>(s_usmp + kMaxB);    // [B] next_token index
+  int *s_seg = s_outb + kMaxB;                              // [2]: tile, quarter; [4]: count
   float2 *s_T = reinterpret_cast<float2 *>(s_seg + 16);     // [B] float-float
   float4 *s_zw = reinterpret_cast<float4 *>(s_T + kMaxB);   // [B][kEpiWarps]
   float2 *s_tw = reinterpret_cast<float2 *>(s_zw + kMaxB * kEpiWarps);  // [tiles][kEpiWarps]
@@ -582,12 +626,13 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     g_s[n] = g.y;
     g_arg[n] = __float_as_int(g.z);
   }
-  for (int b = tid; b < p.B; b += kThreads) {
+  for (int b = tid; p.kind != kPresampled && b < p.B; b += kThreads) {
     const int md = s_md[b];
     if (md != 0 && md != 1 && c == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
     s_stoch[b] = (md == 1) && p.draft_probs != nullptr;
   }
   block_sync();
+  if (p.kind != kPresampled) {
   // (3) Accept test of every draft row, all rows at once (the tests are
   //     independent; only the count of leading accepts depends on their order).
   for (int n = tid; n < p.R; n += kThreads) {
@@ -620,15 +665,57 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     s_rstar[b] = (a >= 0) ? r0 + a : -1;
     if (a < 0) s_stoch[b] = 0;
     if (s_stoch[b]) atomicOr(s_any_stoch, 1);
+    // What to sample: the residual against q of draft a (a < k) or p (bonus).
+    s_qidx[b] = (a >= 0 && a < k) ? r0 - b + a : -1;
+    s_usmp[b] = (a >= 0) ? s_u[r0 + k] : 0.f;
+    s_outb[b] = b;
     if (c == 0) {
       p.accepted_len[b] = a < 0 ? 0 : a;
       if (a < 0) p.next_token[b] = -1;
       else if (!s_stoch[b]) p.next_token[b] = g_arg[r0 + a];
     }
   }
+  } else {
+    // Second pass: row j holds sample j, decided by the first pass.
+    const int ns = *p.samp_count;
+    for (int j = tid; j < p.B; j += kThreads) {
+      s_stoch[j] = j < ns;
+      s_rstar[j] = j;
+      if (j < ns) {
+        const int4 sp = p.samp[j];
+        s_qidx[j] = sp.x;
+        s_usmp[j] = __int_as_float(sp.y);
+        s_outb[j] = sp.z;
+      }
+    }
+    if (tid == 0) *s_any_stoch = ns > 0;
+  }
   block_sync();
 
-  if (*s_any_stoch) {
+  if (p.kind == kStatsOnly) {
+    // First pass of the two-pass path: publish one sample spec per sequence
+    // that needs a draw and gather its hidden row for the second pass.
+    if (tid == 0) {
+      int ns = 0;
+      for (int b = 0; b < p.B; ++b) s_owner[b] = s_stoch[b] ? ns++ : -1;
+      s_seg[4] = ns;
+    }
+    block_sync();
+    if (c == 0) {
+      for (int b = tid; b < p.B; b += kThreads)
+        if (s_owner[b] >= 0)
+          p.samp[s_owner[b]] = make_int4(s_qidx[b], __float_as_int(s_usmp[b]), s_outb[b], s_rstar[b]);
+      if (tid == 0) *p.samp_count = s_seg[4];
+    }
+    const int hv = p.H / 8;  // 16-byte vectors per hidden row
+    for (int b = 0; b < p.B; ++b) {
+      const int j = s_owner[b];
+      if (j < 0 || j % p.NC != c) continue;
+      const uint4 *src = reinterpret_cast<const uint4 *>(p.hidden + static_cast<size_t>(s_rstar[b]) * p.H);
+      uint4 *dst = reinterpret_cast<uint4 *>(p.hidden_s + static_cast<size_t>(j) * p.H);
+      for (int e = tid; e < hv; e += kThreads) dst[e] = src[e];
+    }
+  } else if (*s_any_stoch) {
     // =================== phase C: slice masses of the sampled distribution ==
     // Terms are fp32; every sum is float-float, so the cumulative masses that
     // place u*Z are as exact as the terms allow.
@@ -653,7 +740,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         for (int g = 0; g < kG; ++g) {
           const int b = g < nb ? bl[g] : bl[0];
           nrow[g] = s_rstar[b];
-          qrow[g] = (s_acc[b] < s_nd[b]) ? p.draft_probs + static_cast<size_t>(nrow[g] - b) * p.V : nullptr;
+          qrow[g] = s_qidx[b] >= 0 ? p.draft_probs + static_cast<size_t>(s_qidx[b]) * p.V : nullptr;
           M[g] = g_m[nrow[g]];
           invS[g] = 1.f / g_s[nrow[g]];
           z[g] = ff2{0.f, 0.f};
@@ -728,7 +815,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       totp = warp_sum_ff(totp);
       const bool usep = !(tot.hi > 0.f && isfinite(tot.hi));
       const ff2 Z = usep ? totp : tot;
-      const ff2 Tgt = ff_mul_f(Z, s_u[s_cuq[b] + s_nd[b]]);
+      const ff2 Tgt = ff_mul_f(Z, s_usmp[b]);
       // First slice whose cumulative mass exceeds Tgt; else the last slice with mass.
       ff2 base{0.f, 0.f}, base_owner{0.f, 0.f}, base_last{0.f, 0.f};
       int owner = -1, last_pos = -1;
@@ -771,9 +858,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       for (int b = 0; b < p.B; ++b) {
         if (!s_stoch[b] || s_owner[b] != c) continue;
         const int n = s_rstar[b];
-        const int a = s_acc[b], k = s_nd[b];
         const bool usep = s_usep[b] != 0;
-        const float *qrow = (a < k && !usep) ? p.draft_probs + static_cast<size_t>(n - b) * p.V : nullptr;
+        const float *qrow = (s_qidx[b] >= 0 && !usep) ? p.draft_probs + static_cast<size_t>(s_qidx[b]) * p.V : nullptr;
         const float M = g_m[n], invS = 1.f / g_s[n];
         // (1) mass of every 32-entry segment (tile j, lane quarter q4) of the slice.
         for (int j0 = 0; j0 < ntiles; j0 += 8) {
@@ -842,10 +928,10 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           const unsigned pos = __ballot_sync(0xffffffffu, rv > 0.f);
           if (lane == 0) {
             const int l = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : 0);
-            p.next_token[b] = v + l;
+            p.next_token[s_outb[b]] = v + l;
           }
         } else if (jt < 0 && ew == 0 && lane == 0) {
-          p.next_token[b] = -1;
+          p.next_token[s_outb[b]] = -1;
         }
         named_bar(1, kEpiWarps * 32);
       }
@@ -909,13 +995,59 @@ static void slice_shape(int V, int NC, int *tiles_max, int *brs) {
   *brs = last == 0 ? kTileV : (last + 7) / 8 * 8;
 }
 
-static size_t workspace_bytes_for(int B, int R, int NC) {
-  size_t off = 256;                                        // barrier words
-  off += round_up(static_cast<size_t>(NC) * R * 16, 256);  // pstat
-  off += round_up(static_cast<size_t>(R) * 4, 256);        // ldraft
-  off += round_up(static_cast<size_t>(R) * 16, 256);       // gstat
-  off += round_up(static_cast<size_t>(NC) * B * 16, 256);  // zpart
-  return off;
+// Scratch of one launch: slice partials, draft logits, merged statistics, slice masses.
+struct WsRegion {
+  size_t pstat, ldraft, gstat, zpart, end;
+};
+static WsRegion ws_region(size_t off, int B, int R, int NC) {
+  WsRegion w;
+  w.pstat = off;
+  off += round_up(static_cast<size_t>(NC) * R * 16, 256);
+  w.ldraft = off;
+  off += round_up(static_cast<size_t>(R) * 4, 256);
+  w.gstat = off;
+  off += round_up(static_cast<size_t>(R) * 16, 256);
+  w.zpart = off;
+  off += round_up(static_cast<size_t>(NC) * B * 16, 256);
+  w.end = off;
+  return w;
+}
+
+// Whole workspace.  One launch: [barrier words][region].  Two passes:
+// [barrier words][pass-1 region][sample specs][count][gathered hidden][pass-2 region].
+struct WsLayout {
+  bool two_pass;
+  WsRegion r1, r2;
+  size_t samp, count, hidden_s, end;
+};
+
+static bool resident_fits(int R, int V, int NC) {
+  if (R > kMaxRes) return false;
+  int tiles = 0, brs = 0, rt[kMaxRounds], nr = 0;
+  slice_shape(V, NC, &tiles, &brs);
+  const Plan pl = make_plan(R, V, NC);
+  return tiles <= kMaxTilesPerCta && plan_rounds(tiles, pl.Ncols, pl.Rs, rt, &nr);
+}
+
+static WsLayout ws_layout(int B, int R, int H, int V, int sms) {
+  WsLayout L{};
+  const int NC = make_plan(R, V, sms).NC;
+  L.two_pass = !resident_fits(R, V, NC);
+  L.r1 = ws_region(256, B, R, NC);
+  if (!L.two_pass) {
+    L.end = L.r1.end;
+    return L;
+  }
+  size_t off = L.r1.end;
+  L.samp = off;
+  off += round_up(static_cast<size_t>(B) * 16, 256);
+  L.count = off;
+  off += 256;
+  L.hidden_s = off;
+  off += round_up(static_cast<size_t>(B) * H * 2, 256);
+  L.r2 = ws_region(off, B, B, NC);
+  L.end = L.r2.end;
+  return L;
 }
 
 // 3-D view of a row-major [rows, H] bf16 matrix: dims {64, rows, H/64},
@@ -953,6 +1085,118 @@ static bool encode_kslab_view(CUtensorMap *map, const void *base, int rows, int 
   return true;
 }
 
+struct Maps {
+  CUtensorMap w3, w2, w2s, h3, h2;
+};
+
+// Fills the plan-dependent fields of `p` for a launch of kind `kind` over the
+// rows of `hidden` ([R, H]) and encodes its tensor maps.
+static spade_status prepare(Params &p, int kind, const void *hidden, const void *w_lm, int R,
+                            int sms, Maps &m) {
+  const Plan pl = make_plan(R, p.V, sms);
+  p.kind = kind;
+  p.R = R;
+  p.T = pl.T;
+  p.NC = pl.NC;
+  p.Ncols = pl.Ncols;
+  p.Rs = pl.Rs;
+  p.KC = (p.H + kKChunk - 1) / kKChunk;
+  p.KCF = p.H / kKChunk;
+  int tiles_max = 0;
+  slice_shape(p.V, pl.NC, &tiles_max, &p.BRS);
+  if (tiles_max > kMaxTilesPerCta)
+    return fail(SPADE_ERR_SHAPE, "vocabulary %d needs %d tiles per SM (max %d)", p.V, tiles_max,
+                kMaxTilesPerCta);
+  p.tmem_cols = kTmemCols;
+  if (kind == kStatsOnly) {
+    // One tile per round in one accumulator slot; rows beyond 256 take a
+    // second MMA N-chunk.  Hidden rows arrive in <= 256-row boxes.
+    if (pl.Ncols > kTmemCols) return fail(SPADE_ERR_SHAPE, "R = %d rows exceed %d", R, kTmemCols);
+    p.nrounds = tiles_max;
+    for (int r = 0; r < tiles_max; ++r) p.round_tiles[r] = 1;
+    p.nchunks = pl.Ncols > 256 ? 2 : 1;
+    p.n0w = p.nchunks == 2 ? ((pl.Ncols / 2 + 15) / 16 * 16) : pl.Ncols;
+    p.idesc = idesc_bf16_f32(kTileV, p.n0w);
+    p.idesc1 = idesc_bf16_f32(kTileV, p.nchunks == 2 ? pl.Ncols - p.n0w : 16);
+    p.h_boxes = p.nchunks;
+    p.h_box_rows = p.nchunks == 2 ? 256 : pl.Ncols;
+    p.HS = 2;
+    p.KG = 1;
+  } else {
+    if (!plan_rounds(tiles_max, pl.Ncols, pl.Rs, p.round_tiles, &p.nrounds))
+      return fail(SPADE_ERR_SHAPE,
+                  "logits of %d rows x %d vocab do not fit on chip (%d tiles per SM, %d TMEM columns each)",
+                  R, p.V, tiles_max, pl.Rs);
+    p.nchunks = 1;
+    p.n0w = pl.Ncols;
+    p.idesc = idesc_bf16_f32(kTileV, pl.Ncols);
+    p.idesc1 = p.idesc;
+    p.h_boxes = 1;
+    p.h_box_rows = pl.Ncols;
+    p.HS = 3;
+    p.KG = 2;  // two k-chunks per stage (32 KB W boxes) while the rings fit
+  }
+  for (;;) {
+    Params probe = p;
+    probe.WS = 0;
+    const int fixed = smem_layout(probe).total;
+    p.WS = (kSmemBudget - fixed) / (p.KG * kWChunkBytes);
+    if (p.WS > 8) p.WS = 8;
+    if (p.WS >= 4 || p.KG == 1) break;
+    p.KG = 1;
+  }
+  if (p.WS < 2) return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
+  p.NS = (p.KC + p.KG - 1) / p.KG;
+  if (smem_layout(p).total > kSmemMax) return fail(SPADE_ERR_SHAPE, "shared memory plan too large");
+
+  // 2-D views (one k-chunk per box, zero fill past H) serve a ragged last
+  // k-chunk and row boxes of the first pass; 3-D views fetch KG full k-chunks.
+  const uint64_t pitch = static_cast<uint64_t>(p.H) * 2;
+  if (!encode_tmap_bf16_sw128(&m.w2, w_lm, p.H, p.V, pitch, kKChunk, kTileV) ||
+      !encode_tmap_bf16_sw128(&m.w2s, w_lm, p.H, p.V, pitch, kKChunk, p.BRS) ||
+      !encode_tmap_bf16_sw128(&m.h2, hidden, p.H, R, pitch, kKChunk, p.h_box_rows))
+    return SPADE_ERR_CUDA;
+  if (p.KCF >= 1) {
+    if (!encode_kslab_view(&m.w3, w_lm, p.V, p.H, kTileV, p.KG) ||
+        !encode_kslab_view(&m.h3, hidden, R, p.H, pl.Ncols < 256 ? pl.Ncols : 256, p.KG))
+      return SPADE_ERR_CUDA;
+  } else {
+    m.w3 = m.w2;  // never used: every stage takes the 2-D path
+    m.h3 = m.h2;
+  }
+  return SPADE_OK;
+}
+
+static spade_status launch(const Params &p, const Maps &m, cudaStream_t stream) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(verify_accept_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(verify_accept)");
+    configured = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.NC);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem_layout(p).total;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, verify_accept_kernel, p, m.w3, m.w2, m.w2s, m.h3, m.h2);
+  if (e != cudaSuccess) return cuda_fail(e, "verify_accept cooperative launch");
+  return SPADE_OK;
+}
+
+static void set_region(Params &p, uint8_t *ws, const WsRegion &r) {
+  p.pstat = reinterpret_cast<float4 *>(ws + r.pstat);
+  p.ldraft = reinterpret_cast<float *>(ws + r.ldraft);
+  p.gstat = reinterpret_cast<float4 *>(ws + r.gstat);
+  p.zpart = reinterpret_cast<float4 *>(ws + r.zpart);
+}
+
 }  // namespace accept
 }  // namespace spade
 
@@ -962,8 +1206,7 @@ extern "C" size_t spade_accept_workspace_size(int32_t B, int32_t R, int32_t H, i
   if (B <= 0 || R < B || H <= 0 || V <= 0) return 0;
   int sms = 0;
   if (device_info(&sms, nullptr) != SPADE_OK) return 0;
-  const accept::Plan pl = accept::make_plan(R, V, sms);
-  return accept::workspace_bytes_for(B, R, pl.NC);
+  return accept::ws_layout(B, R, H, V, sms).end;
 }
 
 extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm,
@@ -989,7 +1232,13 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
   spade_status st = device_info(&sms, nullptr);
   if (st != SPADE_OK) return st;
 
-  const Plan pl = make_plan(R, V, sms);
+  const WsLayout L = ws_layout(B, R, H, V, sms);
+  if (!workspace || workspace_bytes < L.end || !aligned(workspace, 256))
+    return fail(SPADE_ERR_WORKSPACE, "accept workspace needs %zu bytes, 256-byte aligned (got %zu)",
+                L.end, workspace_bytes);
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+
   Params p{};
   p.draft_tokens = draft_tokens;
   p.draft_probs = draft_probs;
@@ -1000,85 +1249,30 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
   p.accepted_len = accepted_len;
   p.next_token = next_token;
   p.status = status;
-  p.B = B; p.R = R; p.H = H; p.V = V;
-  p.T = pl.T; p.NC = pl.NC; p.Ncols = pl.Ncols; p.Rs = pl.Rs;
-  p.KC = (H + kKChunk - 1) / kKChunk;
-  p.KCF = H / kKChunk;
-  int tiles_max = 0;
-  slice_shape(V, pl.NC, &tiles_max, &p.BRS);
-  if (tiles_max > kMaxTilesPerCta)
-    return fail(SPADE_ERR_SHAPE, "vocabulary %d needs %d tiles per SM (max %d)", V, tiles_max, kMaxTilesPerCta);
-  if (!plan_rounds(tiles_max, pl.Ncols, pl.Rs, p.round_tiles, &p.nrounds))
-    return fail(SPADE_ERR_SHAPE,
-                "logits of %d rows x %d vocab do not fit on chip (%d tiles per SM, %d TMEM columns each)",
-                R, V, tiles_max, pl.Rs);
-  p.idesc = idesc_bf16_f32(kTileV, pl.Ncols);
-  p.tmem_cols = kTmemCols;
-  // Two k-chunks per stage (32 KB W boxes) while the rings fit in shared memory.
-  p.HS = 3;
-  p.KG = 2;
-  for (;;) {
-    Params probe = p;
-    probe.WS = 0;
-    const int fixed = smem_layout(probe).total;
-    p.WS = (kSmemBudget - fixed) / (p.KG * kWChunkBytes);
-    if (p.WS > 8) p.WS = 8;
-    if (p.WS >= 4 || p.KG == 1) break;
-    p.KG = 1;
-  }
-  if (p.WS < 2) return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
-  p.NS = (p.KC + p.KG - 1) / p.KG;
-  const size_t need = workspace_bytes_for(B, R, pl.NC);
-  if (!workspace || workspace_bytes < need || !aligned(workspace, 256))
-    return fail(SPADE_ERR_WORKSPACE, "accept workspace needs %zu bytes, 256-byte aligned (got %zu)",
-                need, workspace_bytes);
-  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  p.B = B;
+  p.H = H;
+  p.V = V;
+  p.hidden = static_cast<const __nv_bfloat16 *>(hidden);
   p.bar = reinterpret_cast<unsigned *>(ws);
-  size_t off = 256;
-  p.pstat = reinterpret_cast<float4 *>(ws + off);
-  off += round_up(static_cast<size_t>(pl.NC) * R * 16, 256);
-  p.ldraft = reinterpret_cast<float *>(ws + off);
-  off += round_up(static_cast<size_t>(R) * 4, 256);
-  p.gstat = reinterpret_cast<float4 *>(ws + off);
-  off += round_up(static_cast<size_t>(R) * 16, 256);
-  p.zpart = reinterpret_cast<float4 *>(ws + off);
-
-  // 2-D views (one k-chunk per box, zero fill past H) serve a ragged last
-  // k-chunk; 3-D views fetch KG full k-chunks per box.
-  CUtensorMap tw2, tw2s, th2, tw3, th3;
-  if (!encode_tmap_bf16_sw128(&tw2, w_lm, H, V, static_cast<uint64_t>(H) * 2, kKChunk, kTileV) ||
-      !encode_tmap_bf16_sw128(&tw2s, w_lm, H, V, static_cast<uint64_t>(H) * 2, kKChunk, p.BRS) ||
-      !encode_tmap_bf16_sw128(&th2, hidden, H, R, static_cast<uint64_t>(H) * 2, kKChunk, pl.Ncols))
-    return SPADE_ERR_CUDA;
-  if (p.KCF >= 1) {
-    if (!encode_kslab_view(&tw3, w_lm, V, H, kTileV, p.KG) ||
-        !encode_kslab_view(&th3, hidden, R, H, pl.Ncols, p.KG))
-      return SPADE_ERR_CUDA;
-  } else {
-    tw3 = tw2;  // never used: every stage takes the 2-D path
-    th3 = th2;
+  set_region(p, ws, L.r1);
+  Maps m;
+  if (!L.two_pass) {
+    st = prepare(p, kResident, hidden, w_lm, R, sms, m);
+    if (st != SPADE_OK) return st;
+    return launch(p, m, s);
   }
-
-  const int smem = smem_layout(p).total;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(verify_accept_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget + 2048);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(verify_accept)");
-    configured = true;
-  }
-  if (smem > kSmemBudget + 2048) return fail(SPADE_ERR_SHAPE, "shared memory plan too large (%d)", smem);
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(pl.NC);
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = reinterpret_cast<cudaStream_t>(stream);
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeCooperative;
-  attr[0].val.cooperative = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, verify_accept_kernel, p, tw3, tw2, tw2s, th3, th2);
-  if (e != cudaSuccess) return cuda_fail(e, "verify_accept cooperative launch");
-  return SPADE_OK;
+  // More rows than TMEM holds: a statistics-and-decisions pass over all rows,
+  // then a resident pass over the gathered rows that need a draw.
+  p.samp = reinterpret_cast<int4 *>(ws + L.samp);
+  p.samp_count = reinterpret_cast<int *>(ws + L.count);
+  p.hidden_s = reinterpret_cast<__nv_bfloat16 *>(ws + L.hidden_s);
+  st = prepare(p, kStatsOnly, hidden, w_lm, R, sms, m);
+  if (st != SPADE_OK) return st;
+  st = launch(p, m, s);
+  if (st != SPADE_OK) return st;
+  Params p2 = p;
+  set_region(p2, ws, L.r2);
+  st = prepare(p2, kPresampled, p.hidden_s, w_lm, B, sms, m);
+  if (st != SPADE_OK) return st;
+  return launch(p2, m, s);
 }

@@ -28,6 +28,11 @@ SMALL = {
                                  ctx=(20000, 20000), k=(6, 6), mode="greedy", match_prob=0.9, seed=15),
     "many_rows": W.WorkloadSpec("many_rows", B=16, Hq=16, Hkv=2, D=128, H=384, V=5000, ctx=(30, 900),
                                 k=(1, 8), mode="mixed", seed=16),
+    # More verify rows than TMEM keeps resident: the two-pass LM head.
+    "two_pass_mixed": W.WorkloadSpec("two_pass_mixed", B=40, Hq=8, Hkv=2, D=128, H=320, V=9000,
+                                     ctx=(5, 300), k=(4, 10), mode="mixed", seed=17),
+    "two_pass_stochastic": W.WorkloadSpec("two_pass_stochastic", B=48, Hq=4, Hkv=4, D=64, H=256,
+                                          V=40000, ctx=(1, 64), k=(6, 9), mode="stochastic", seed=18),
 }
 
 
@@ -109,7 +114,7 @@ def test_repeat_calls_reuse_workspace(dev):
 
 # ---------------------------------------------------------------------------
 # Benchmark workloads at full size (the launch configuration bench.py times).
-FULL = ["tiny", "llama2_7b_greedy", "llama2_7b_stochastic", "llama3_8b", "long_70b"]
+FULL = ["tiny", "llama2_7b_greedy", "llama2_7b_stochastic", "llama3_8b", "long_70b", "ragged"]
 
 
 def _sample_pairs(wl, n, seed):
