@@ -268,9 +268,10 @@ def run_spade(args, ws, rank, local):
                "traffic": _traffic("verify_accept_kernel", args.workload),
                "algorithmic_bytes": lm_bytes, "peak_source": peak_src,
                "tensor_tflops": lm_flop / m_acc / 1e12, "tensor_frac_of_bf16_peak": lm_flop / m_acc / 1e12 / bf16}
-    roof_attn = {"kernel": "verify_attention_kernel", "bound": "hbm", "achieved": attn_bytes / m_attn / 1e9,
+    attn_kernel = "verify_attention_tc_kernel" if wl["D"] == 128 else "verify_attention_kernel"
+    roof_attn = {"kernel": attn_kernel, "bound": "hbm", "achieved": attn_bytes / m_attn / 1e9,
                  "peak": hbm, "unit": "GB/s", "frac": attn_bytes / m_attn / 1e9 / hbm,
-                 "traffic": _traffic("verify_attention_kernel", args.workload),
+                 "traffic": _traffic(attn_kernel, args.workload),
                  "algorithmic_bytes": attn_bytes, "peak_source": peak_src,
                  "tflops": attn_flop / m_attn / 1e12}
     dominant = roof_lm if m_acc >= m_attn else roof_attn

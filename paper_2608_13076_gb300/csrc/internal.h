@@ -25,10 +25,11 @@ bool encode_tmap_bf16_sw128(CUtensorMap *map, const void *base, uint64_t inner, 
 
 // Encodes a 3-D view of a row-major bf16 matrix [rows, cols] (cols a multiple
 // of 64): dims {64, rows, cols/64}, strides {cols*2, 128} bytes, box
-// {64, box_rows, cols/64}, 128-byte swizzle.  One box fetches box_rows whole
-// rows and lands them as cols/64 slabs of [box_rows][64], back to back.
+// {64, box_rows, box_slabs}, 128-byte swizzle.  One box fetches box_rows rows
+// and lands them as box_slabs slabs of [box_rows][64], back to back; box_slabs
+// = 0 means all cols/64 slabs (whole rows).
 bool encode_tmap_rows_by_slab(CUtensorMap *map, const void *base, uint64_t rows, uint32_t cols,
-                              uint32_t box_rows);
+                              uint32_t box_rows, uint32_t box_slabs = 0);
 
 inline bool aligned(const void *p, uintptr_t a) {
   return (reinterpret_cast<uintptr_t>(p) % a) == 0;

@@ -98,7 +98,7 @@ bool encode_tmap_bf16_sw128(CUtensorMap *map, const void *base, uint64_t inner, 
 }
 
 bool encode_tmap_rows_by_slab(CUtensorMap *map, const void *base, uint64_t rows, uint32_t cols,
-                              uint32_t box_rows) {
+                              uint32_t box_rows, uint32_t box_slabs) {
   std::call_once(g_encode_once, [] {
     void *fn = nullptr;
     cudaDriverEntryPointQueryResult q;
@@ -113,7 +113,7 @@ bool encode_tmap_rows_by_slab(CUtensorMap *map, const void *base, uint64_t rows,
   }
   cuuint64_t dims[3] = {64, rows, cols / 64};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(cols) * 2, 128};
-  cuuint32_t box[3] = {64, box_rows, cols / 64};
+  cuuint32_t box[3] = {64, box_rows, box_slabs ? box_slabs : cols / 64};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims,
                         strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,

@@ -1,8 +1,10 @@
 // verify_attention.cu -- attention of the k+1 verify positions of every sequence
 // against its bf16 KV cache (the verifier's single forward pass over the draft
-// block: Sec. III-B "Verification Stage", Algorithm 1 cloud step).
+// block: Sec. III-B "Verification Stage", Algorithm 1 cloud step).  This file
+// holds the C-ABI entry points (head dim 128 dispatches to the tensor-memory
+// kernel in verify_attention_tc.cu) and the warp-MMA kernel used for head dim 64.
 //
-// Design (GB300):
+// Warp-MMA kernel design (GB300):
 //  * Work unit = (sequence b, KV head, block of <= 64 query rows).  The G query
 //    heads of a KV head times the k_b+1 positions form the rows, so every K/V
 //    tile fetched from HBM is used by all of them (GQA grouping).
@@ -13,42 +15,19 @@
 //    finishes a unit last (atomic counter) merges them by log-sum-exp.
 //  * One producer warp streams K/V chunks with TMA (128B-swizzled boxes) into a
 //    multi-stage ring guarded by mbarriers; consumer warps run the QK^T and PV
-//    products on bf16 tensor-core MMAs with fp32 accumulators and an online
-//    softmax whose row statistics are merged with warp shuffles.
+//    products on bf16 warp MMAs with fp32 accumulators and an online softmax
+//    whose row statistics are merged with warp shuffles.
 //  * The causal mask is applied only to chunks that reach past ctx_b, i.e.
 //    inside the draft block; cache slots beyond ctx_b + k_b are zeroed in the
 //    value fragments so whatever they hold cannot reach the result.
-#include <cuda_bf16.h>
-
-#include <cfloat>
 #include <mutex>
 
-#include "internal.h"
-#include "ptx.cuh"
+#include "attn_common.cuh"
 
 namespace spade {
 namespace attn {
 
-constexpr int kChunk = 64;     // keys per pipeline stage
-constexpr int kRowBlock = 64;  // query rows per work unit
-constexpr int kMaxB = 512;     // sequences per call (per-CTA schedule lives in smem)
 constexpr int kSmemBudget = 220 * 1024;
-
-struct Params {
-  const __nv_bfloat16 *q;
-  __nv_bfloat16 *out;
-  float *lse;
-  const int32_t *ctx_lens;
-  const int32_t *n_draft;
-  const int32_t *cu_q;
-  int32_t *counters;  // [units], zero between calls
-  float *partials;    // [(num_ctas + units) slots][kRowBlock * D + 2 * kRowBlock]
-  int32_t *status;
-  int B, Hq, Hkv, G, cap, max_k, R, RB, num_ctas;
-  float scale_log2;  // log2(e) / sqrt(D)
-};
-
-constexpr int round_up_c(int x, int a) { return (x + a - 1) / a * a; }
 
 template <int D, int MT>
 struct Layout {
@@ -77,78 +56,6 @@ struct Layout {
   static constexpr int OFF_MISC = OFF_BAR + 2 * STAGES * 8;
   static constexpr int SMEM = OFF_MISC + 64 + 1024;  // + slack for 1024-byte alignment
 };
-
-__host__ __device__ constexpr int slot_floats(int D) { return kRowBlock * D + 2 * kRowBlock; }
-
-// Per-CTA view of the schedule.
-struct Sched {
-  const int64_t *pref;  // [B+1] chunk prefix over sequences
-  const int32_t *ctx;   // [B]
-  const int32_t *kd;    // [B]  (-1 marks an invalid sequence: no work)
-  int B, Hkv, G, RB;
-  int64_t total;
-  int num_ctas;
-
-  __device__ int rows_of(int b) const { return G * (kd[b] + 1); }
-  __device__ int rb_count(int b) const {
-    return kd[b] < 0 ? 0 : (rows_of(b) + kRowBlock - 1) / kRowBlock;
-  }
-  __device__ int chunks(int b, int rb) const {
-    const int m = rows_of(b);
-    const int last_row = min(kRowBlock * (rb + 1), m) - 1;
-    const int i_hi = last_row / G;
-    return (ctx[b] + i_hi + 1 + kChunk - 1) / kChunk;
-  }
-  __device__ int64_t owner(int64_t x) const {
-    return ((x + 1) * num_ctas + total - 1) / total - 1;
-  }
-};
-
-struct Seg {
-  int b, kvh, rb;
-  int ci;        // first chunk (within the unit) of this segment
-  int nch;       // chunks of the unit
-  int64_t ust;   // global index of the unit's first chunk
-};
-
-__device__ __forceinline__ Seg locate(const Sched &s, int64_t x) {
-  int lo = 0, hi = s.B - 1;  // largest b with pref[b] <= x
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (s.pref[mid] <= x) lo = mid; else hi = mid - 1;
-  }
-  Seg g;
-  g.b = lo;
-  g.nch = 0;
-  const int nrb = s.rb_count(lo);
-  int span = 0;
-  for (int rb = 0; rb < nrb; ++rb) span += s.chunks(lo, rb);
-  int64_t o = x - s.pref[lo];
-  g.kvh = static_cast<int>(o / span);
-  int o2 = static_cast<int>(o - static_cast<int64_t>(g.kvh) * span);
-  int cum = 0;
-  g.rb = 0;
-  for (int rb = 0; rb < nrb; ++rb) {
-    const int c = s.chunks(lo, rb);
-    if (o2 < cum + c) { g.rb = rb; g.nch = c; break; }
-    cum += c;
-  }
-  g.ci = o2 - cum;
-  g.ust = s.pref[lo] + static_cast<int64_t>(g.kvh) * span + cum;
-  return g;
-}
-
-// bar.sync is the aligned form: every lane of a warp must arrive together.
-// Lanes that ran ahead of a divergent lane (a lane-0-only loop) reconverge
-// first, so no warp reaches the barrier before all of its lanes do.
-__device__ __forceinline__ void named_bar(int id, int threads) {
-  __syncwarp();
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
-}
-__device__ __forceinline__ void block_sync() {
-  __syncwarp();
-  __syncthreads();
-}
 
 // Byte offset of 16-byte chunk `c` (0..D/8-1) of row `r` inside a K/V stage
 // tile written by TMA with 128-byte swizzle (box = 64 rows x 128 bytes).
@@ -179,41 +86,13 @@ __global__ void __launch_bounds__(Layout<D, MT>::THREADS, 1)
 
   // ---- per-sequence validation and chunk counts ---------------------------
   if (tid == 0) { *s_abort = 0; *s_last = 0; }
-  for (int b = tid; b < p.B; b += blockDim.x) {
-    const int c = p.ctx_lens[b], k = p.n_draft[b];
-    const int q0 = p.cu_q[b], q1 = p.cu_q[b + 1];
-    int bad = 0;
-    if (c < 0 || k < 0 || k > p.max_k || q0 < 0 || q1 > p.R || q1 - q0 != k + 1) bad = SPADE_DEV_BAD_INDEX;
-    else if (static_cast<int64_t>(c) + k + 1 > p.cap) bad = SPADE_DEV_CAPACITY;
-    if (bad && blockIdx.x == 0) atomicOr(p.status, bad);
-    s_ctx[b] = c;
-    s_kd[b] = bad ? -1 : k;
-  }
+  sched_validate(p, s_ctx, s_kd, tid, blockDim.x);
   block_sync();
   Sched sc;
   sc.pref = s_pref; sc.ctx = s_ctx; sc.kd = s_kd;
   sc.B = p.B; sc.Hkv = p.Hkv; sc.G = p.G; sc.RB = p.RB; sc.num_ctas = p.num_ctas;
   if (warp == 0) {
-    // Warp-level scan of W_b = Hkv * sum_rb chunks(b, rb).
-    int64_t carry = 0;
-    for (int b0 = 0; b0 < p.B; b0 += 32) {
-      const int b = b0 + lane;
-      int64_t w = 0;
-      if (b < p.B) {
-        const int nrb = sc.rb_count(b);
-        int span = 0;
-        for (int rb = 0; rb < nrb; ++rb) span += sc.chunks(b, rb);
-        w = static_cast<int64_t>(p.Hkv) * span;
-      }
-      int64_t incl = w;
-      for (int o = 1; o < 32; o <<= 1) {
-        const int64_t v = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += v;
-      }
-      if (b < p.B) s_pref[b] = carry + incl - w;
-      carry += __shfl_sync(0xffffffffu, incl, 31);
-    }
-    if (lane == 0) s_pref[p.B] = carry;
+    sched_scan(p, sc, s_pref, lane);
   } else if (warp == 1 && lane == 0) {
     for (int s = 0; s < L::STAGES; ++s) {
       mbar_init(&full_bar[s], 1);
@@ -542,96 +421,13 @@ __global__ void __launch_bounds__(Layout<D, MT>::THREADS, 1)
             __stcg(part + kRowBlock * D + kRowBlock + rl, h ? l1 : l0);
           }
         }
-        __threadfence();
       }
       named_bar(1, NT);
-      if (ctid == 0) {
-        const int old = atomicAdd(&p.counters[unit], 1);
-        __threadfence();
-        *s_last = (old == nparts - 1);
-      }
+      if (ctid == 0) *s_last = arrive_part(&p.counters[unit], nparts);
       named_bar(1, NT);
       if (*s_last) {
         // This CTA finished the unit last: merge every partial by log-sum-exp.
-        // Online merge, two rows per warp step, the loads of up to kBatch
-        // partials per row in flight together.
-        const int64_t slot0 = c_first + unit;
-        constexpr int PER = D / 32;
-        constexpr int kBatch = 4;
-        for (int rl0 = 2 * cw; rl0 < nrow; rl0 += 2 * L::NW) {
-          float M[2] = {-INFINITY, -INFINITY}, Lsum[2] = {0.f, 0.f};
-          float acc[2][PER];
-#pragma unroll
-          for (int h = 0; h < 2; ++h)
-#pragma unroll
-            for (int e = 0; e < PER; ++e) acc[h][e] = 0.f;
-          for (int s0 = 0; s0 < nparts; s0 += kBatch) {
-            float mv[2][kBatch], lv[2][kBatch], ov[2][kBatch][PER];
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              const int rl = min(rl0 + h, nrow - 1);
-#pragma unroll
-              for (int j = 0; j < kBatch; ++j) {
-                if (s0 + j < nparts) {
-                  const float *ps = p.partials + (slot0 + s0 + j) * slot_floats(D);
-                  mv[h][j] = __ldcg(ps + kRowBlock * D + rl);
-                  lv[h][j] = __ldcg(ps + kRowBlock * D + kRowBlock + rl);
-                  if constexpr (PER == 4) {
-                    const float4 v = __ldcg(reinterpret_cast<const float4 *>(ps + rl * D + lane * 4));
-                    ov[h][j][0] = v.x; ov[h][j][1] = v.y; ov[h][j][2] = v.z; ov[h][j][3] = v.w;
-                  } else {
-                    const float2 v = __ldcg(reinterpret_cast<const float2 *>(ps + rl * D + lane * 2));
-                    ov[h][j][0] = v.x; ov[h][j][1] = v.y;
-                  }
-                } else {
-                  mv[h][j] = -INFINITY;
-                  lv[h][j] = 0.f;
-#pragma unroll
-                  for (int e = 0; e < PER; ++e) ov[h][j][e] = 0.f;
-                }
-              }
-            }
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              float Mn = M[h];
-#pragma unroll
-              for (int j = 0; j < kBatch; ++j) Mn = fmaxf(Mn, mv[h][j]);
-              const float U = (Mn == -INFINITY) ? 0.f : Mn;
-              const float f = ex2(M[h] - U);
-              Lsum[h] *= f;
-#pragma unroll
-              for (int e = 0; e < PER; ++e) acc[h][e] *= f;
-#pragma unroll
-              for (int j = 0; j < kBatch; ++j) {
-                const float w = ex2(mv[h][j] - U);
-                Lsum[h] += w * lv[h][j];
-#pragma unroll
-                for (int e = 0; e < PER; ++e) acc[h][e] += w * ov[h][j][e];
-              }
-              M[h] = Mn;
-            }
-          }
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int rl = rl0 + h;
-            if (rl < nrow) {
-              const int row = kRowBlock * g.rb + rl;
-              const int i = row / p.G, gh = row % p.G;
-              const size_t orow = static_cast<size_t>(q_row0 + i) * p.Hq + g.kvh * p.G + gh;
-              const float inv = 1.f / Lsum[h];
-              if constexpr (PER == 4) {
-                uint2 v;
-                v.x = pack_bf16(acc[h][0] * inv, acc[h][1] * inv);
-                v.y = pack_bf16(acc[h][2] * inv, acc[h][3] * inv);
-                *reinterpret_cast<uint2 *>(p.out + orow * D + lane * 4) = v;
-              } else {
-                *reinterpret_cast<uint32_t *>(p.out + orow * D + lane * 2) =
-                    pack_bf16(acc[h][0] * inv, acc[h][1] * inv);
-              }
-              if (p.lse && lane == 0) p.lse[orow] = (M[h] + log2f(Lsum[h])) * 0.69314718055994531f;
-            }
-          }
-        }
+        merge_partials<D>(p, c_first + unit, nparts, nrow, g.rb, g.kvh, q_row0, cw, L::NW, lane);
         if (ctid == 0) p.counters[unit] = 0;  // every part has arrived: reset for the next call
       }
     }
@@ -717,23 +513,26 @@ extern "C" spade_status spade_verify_attention(
   const int64_t max_chunks = static_cast<int64_t>(units) * ((cap + attn::kChunk - 1) / attn::kChunk);
   p.num_ctas = static_cast<int>(max_chunks < sms ? max_chunks : sms);
 
-  CUtensorMap tk, tv;
   const uint64_t rows = static_cast<uint64_t>(B) * Hkv * cap;
-  if (!encode_tmap_rows_by_slab(&tk, k_cache, rows, D, attn::kChunk) ||
-      !encode_tmap_rows_by_slab(&tv, v_cache, rows, D, attn::kChunk))
-    return SPADE_ERR_CUDA;
-
-  const int mt = (G * (max_k + 1) >= attn::kRowBlock) ? 4 : (G * (max_k + 1) + 15) / 16;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e;
   if (D == 128) {
-    switch (mt) {
-      case 1: e = attn::launch<128, 1>(p, tk, tv, s); break;
-      case 2: e = attn::launch<128, 2>(p, tk, tv, s); break;
-      case 3: e = attn::launch<128, 3>(p, tk, tv, s); break;
-      default: e = attn::launch<128, 4>(p, tk, tv, s); break;
-    }
+    // Tensor-memory kernel: 128-key boxes of both 64-dim slabs, and 64-key
+    // boxes of one slab for a segment's last odd slice.
+    CUtensorMap k2, v2, k1, v1;
+    if (!encode_tmap_rows_by_slab(&k2, k_cache, rows, D, 128) ||
+        !encode_tmap_rows_by_slab(&v2, v_cache, rows, D, 128) ||
+        !encode_tmap_rows_by_slab(&k1, k_cache, rows, D, attn::kChunk, 1) ||
+        !encode_tmap_rows_by_slab(&v1, v_cache, rows, D, attn::kChunk, 1))
+      return SPADE_ERR_CUDA;
+    const int rows_max = G * (max_k + 1) < attn::kRowBlock ? G * (max_k + 1) : attn::kRowBlock;
+    e = attn::launch_tc(p, k2, v2, k1, v1, (rows_max + 15) / 16 * 16, s);
   } else {
+    CUtensorMap tk, tv;
+    if (!encode_tmap_rows_by_slab(&tk, k_cache, rows, D, attn::kChunk) ||
+        !encode_tmap_rows_by_slab(&tv, v_cache, rows, D, attn::kChunk))
+      return SPADE_ERR_CUDA;
+    const int mt = (G * (max_k + 1) >= attn::kRowBlock) ? 4 : (G * (max_k + 1) + 15) / 16;
     switch (mt) {
       case 1: e = attn::launch<64, 1>(p, tk, tv, s); break;
       case 2: e = attn::launch<64, 2>(p, tk, tv, s); break;
