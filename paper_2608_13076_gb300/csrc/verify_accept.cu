@@ -52,6 +52,7 @@ constexpr int kMaxRounds = 32;
 // already taken.
 constexpr int kResident = 0, kStatsOnly = 1, kPresampled = 2;
 constexpr int kMaxTilesPerCta = 32;
+constexpr int kMaxNC = 256;  // CTAs (vocabulary slices) per launch
 constexpr int kTmemCols = 512;
 constexpr int kSmemBudget = 220 * 1024;
 constexpr int kSmemMax = 225 * 1024;  // opt-in limit (227 KB) minus static shared memory
@@ -68,7 +69,7 @@ struct Params {
   int32_t *accepted_len;
   int32_t *next_token;
   int32_t *status;
-  unsigned *bar;     // [2]: arrival count, generation
+  unsigned *bar;     // [0]: arrival count, [kGenWord]: generation
   float4 *pstat;     // [NC][R]: slice max, slice sum-exp, slice argmax (bits), -
   float *ldraft;     // [R]: logit of the row's draft token
   float4 *gstat;     // [R]: merged row max, sum-exp, argmax (bits)
@@ -129,33 +130,43 @@ __device__ __forceinline__ void block_sync() {
   __syncthreads();
 }
 
-__device__ __forceinline__ unsigned ld_acquire(const unsigned *p) {
+__device__ __forceinline__ unsigned ld_relaxed(const unsigned *p) {
   unsigned v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
 
+// Word offset of the grid barrier's generation counter: its own 128-byte line,
+// apart from the arrival count, so the waiting CTAs' polls do not queue behind
+// the arrival atomics on one L2 line.
+constexpr int kGenWord = 32;
+static_assert(kGenWord * 4 + 4 <= 256, "barrier words live in the workspace's first 256 bytes");
 
 // Device-wide barrier among the NC co-resident CTAs (cooperative launch).  The
 // last CTA to arrive resets the count and bumps the generation; the others
-// poll the generation with a time limit.  Returns false if the wait expired.
+// poll the generation (relaxed loads with a short back-off, then an acquire
+// fence) with a time limit.  Returns false if the wait expired.
 __device__ bool grid_barrier(unsigned *bar, int nctas) {
   __shared__ int s_ok;
   block_sync();
   if (threadIdx.x == 0) {
     s_ok = 1;
-    const unsigned gen = ld_acquire(bar + 1);
+    unsigned *gen_p = bar + kGenWord;
+    // Read before arriving (the arrival's release orders this load first).
+    const unsigned gen = ld_relaxed(gen_p);
     unsigned arrived;
     // The arrival releases this CTA's writes (ordered before it by bar.sync).
     asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(arrived) : "l"(bar) : "memory");
     if (arrived == static_cast<unsigned>(nctas) - 1) {
       asm volatile("st.relaxed.gpu.global.u32 [%0], 0;" ::"l"(bar) : "memory");
-      asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(bar + 1) : "memory");
+      asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(gen_p) : "memory");
     } else {
       const uint64_t t0 = globaltimer();
-      while (ld_acquire(bar + 1) == gen) {
+      while (ld_relaxed(gen_p) == gen) {
         if (globaltimer() - t0 > kWaitLimitNs) { s_ok = 0; break; }
+        __nanosleep(20);
       }
+      asm volatile("fence.acq_rel.gpu;" ::: "memory");
     }
   }
   block_sync();
@@ -717,14 +728,16 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     }
   } else if (*s_any_stoch) {
     // =================== phase C: slice masses of the sampled distribution ==
-    // Terms are fp32; every sum is float-float, so the cumulative masses that
-    // place u*Z are as exact as the terms allow.
+    // Terms are fp32 (p = 2^((l - m) log2 e) / Z on the SFU, the same formula
+    // here and in phase D, so the slice and segment masses agree); every sum is
+    // float-float, so the cumulative masses that place u*Z are as exact as the
+    // terms allow.
     if (warp >= 2) {
       const int ew = warp - 2, q4 = warp & 3;
       const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
       // Stochastic sequences in groups of kG: the TMEM reads and q loads of a
       // whole group are in flight together.
-      constexpr int kG = 4;
+      constexpr int kG = 8;
       for (int b0 = 0; b0 < p.B;) {
         int bl[kG], nb = 0;
         while (b0 < p.B && nb < kG) {
@@ -772,7 +785,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             for (int j = 0; j < 8; ++j) {
               const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
               if (g < nb && j < nj && v < v_hi) {
-                const float pv = expf(__uint_as_float(raw[g][j]) - M[g]) * invS[g];
+                const float pv = ex2((__uint_as_float(raw[g][j]) - M[g]) * kLog2e) * invS[g];
                 zp[g] = ff_add_f(zp[g], pv);
                 z[g] = ff_add_f(z[g], qrow[g] ? fmaxf(0.f, pv - qv[g][j]) : pv);
               }
@@ -803,13 +816,24 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       *s_abort = 1;
     }
     // =================== phase D: owner slice of u*Z, in-slice scan =========
+    // One warp per sequence: all NC slice masses in registers (one round of
+    // loads), their total, then a chunked prefix scan for the first slice whose
+    // cumulative mass passes u*Z.
+    constexpr int kZC = kMaxNC / 32;
     for (int b = warp; b < p.B; b += kThreads / 32) {
       if (!s_stoch[b]) { if (lane == 0) s_owner[b] = -1; continue; }
+      float4 zz[kZC];
+#pragma unroll
+      for (int i = 0; i < kZC; ++i) {
+        const int cc = i * 32 + lane;
+        zz[i] = (i * 32 < p.NC && cc < p.NC) ? __ldcg(&p.zpart[static_cast<size_t>(cc) * p.B + b])
+                                            : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
       ff2 tot{0.f, 0.f}, totp{0.f, 0.f};
-      for (int cc = lane; cc < p.NC; cc += 32) {
-        const float4 z = __ldcg(&p.zpart[static_cast<size_t>(cc) * p.B + b]);
-        tot = ff_add(tot, ff2{z.x, z.y});
-        totp = ff_add(totp, ff2{z.z, z.w});
+#pragma unroll
+      for (int i = 0; i < kZC; ++i) {
+        tot = ff_add(tot, ff2{zz[i].x, zz[i].y});
+        totp = ff_add(totp, ff2{zz[i].z, zz[i].w});
       }
       tot = warp_sum_ff(tot);
       totp = warp_sum_ff(totp);
@@ -819,13 +843,11 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       // First slice whose cumulative mass exceeds Tgt; else the last slice with mass.
       ff2 base{0.f, 0.f}, base_owner{0.f, 0.f}, base_last{0.f, 0.f};
       int owner = -1, last_pos = -1;
-      for (int c0 = 0; c0 < p.NC && owner < 0; c0 += 32) {
-        const int cc = c0 + lane;
-        ff2 z{0.f, 0.f};
-        if (cc < p.NC) {
-          const float4 zz = __ldcg(&p.zpart[static_cast<size_t>(cc) * p.B + b]);
-          z = usep ? ff2{zz.z, zz.w} : ff2{zz.x, zz.y};
-        }
+#pragma unroll
+      for (int i = 0; i < kZC; ++i) {
+        if (i * 32 >= p.NC || owner >= 0) break;
+        const int cc = i * 32 + lane;
+        const ff2 z = usep ? ff2{zz[i].z, zz[i].w} : ff2{zz[i].x, zz[i].y};
         const ff2 incl = warp_scan_ff(z, lane);
         const ff2 reach = ff_add(base, incl);
         const ff2 before = ff_add(base, ff_sub(incl, z));  // mass of the slices before cc
@@ -833,12 +855,12 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         const unsigned pos = __ballot_sync(0xffffffffu, cc < p.NC && z.hi > 0.f);
         if (hit) {
           const int l = __ffs(hit) - 1;
-          owner = c0 + l;
+          owner = i * 32 + l;
           base_owner = ff_shfl(before, l);
         }
         if (pos) {
           const int l = 31 - __clz(pos);
-          last_pos = c0 + l;
+          last_pos = i * 32 + l;
           base_last = ff_shfl(before, l);
         }
         base = ff_shfl(reach, 31);
@@ -880,7 +902,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
             float rv = 0.f;
             if (j < nj && v < v_hi) {
-              const float pv = expf(__uint_as_float(raw[j]) - M) * invS;
+              const float pv = ex2((__uint_as_float(raw[j]) - M) * kLog2e) * invS;
               rv = qrow ? fmaxf(0.f, pv - qv[j]) : pv;
             }
             const ff2 seg = warp_sum_ff(ff2{rv, 0.f});
@@ -919,7 +941,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           tmem_wait_ld();
           float rv = 0.f;
           if (v < v_hi) {
-            const float pv = expf(__uint_as_float(raw) - M) * invS;
+            const float pv = ex2((__uint_as_float(raw) - M) * kLog2e) * invS;
             rv = qrow ? fmaxf(0.f, pv - qv) : pv;
           }
           const ff2 incl = warp_scan_ff(ff2{rv, 0.f}, lane);
@@ -976,6 +998,7 @@ static Plan make_plan(int R, int V, int sms) {
   Plan pl;
   pl.T = (V + kTileV - 1) / kTileV;
   pl.NC = pl.T < sms ? pl.T : sms;
+  if (pl.NC > kMaxNC) pl.NC = kMaxNC;
   pl.Ncols = (R + 15) / 16 * 16;
   pl.Rs = (R + 7) / 8 * 8;
   return pl;
