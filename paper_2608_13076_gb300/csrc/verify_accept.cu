@@ -737,7 +737,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
       // Stochastic sequences in groups of kG: the TMEM reads and q loads of a
       // whole group are in flight together.
-      constexpr int kG = 8;
+      constexpr int kG = 4;
       for (int b0 = 0; b0 < p.B;) {
         int bl[kG], nb = 0;
         while (b0 < p.B && nb < kG) {
