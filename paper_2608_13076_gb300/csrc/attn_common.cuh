@@ -18,6 +18,7 @@ namespace attn {
 constexpr int kChunk = 64;     // keys per schedule slice (and per warp-MMA stage)
 constexpr int kRowBlock = 64;  // query rows per work unit
 constexpr int kMaxB = 512;     // sequences per call (per-CTA schedule lives in smem)
+constexpr int kUnitCostTc = 5; // virtual slices per unit in the tensor-memory kernel's schedule
 
 struct Params {
   const __nv_bfloat16 *q;
@@ -30,6 +31,7 @@ struct Params {
   float *partials;    // [(num_ctas + units) slots][kRowBlock * D + 2 * kRowBlock]
   int32_t *status;
   int B, Hq, Hkv, G, cap, max_k, R, RB, num_ctas;
+  int unit_cost;     // virtual slices charged at each unit's start (the schedule's cost model)
   float scale_log2;  // log2(e) / sqrt(D)
 };
 
@@ -37,12 +39,15 @@ constexpr int round_up_c(int x, int a) { return (x + a - 1) / a * a; }
 
 __host__ __device__ constexpr int slot_floats(int D) { return kRowBlock * D + 2 * kRowBlock; }
 
-// Per-CTA view of the schedule.
+// Per-CTA view of the schedule.  The units' key slices are laid end to end in
+// a cost space where every unit also carries E virtual slices at its start
+// (its epilogue and pipeline restart), and the cost space is cut into one equal
+// range per CTA; E = 0 is the plain stream-K split over slices.
 struct Sched {
-  const int64_t *pref;  // [B+1] chunk prefix over sequences
+  const int64_t *pref;  // [B+1] cost prefix over sequences
   const int32_t *ctx;   // [B]
   const int32_t *kd;    // [B]  (-1 marks an invalid sequence: no work)
-  int B, Hkv, G, RB;
+  int B, Hkv, G, RB, E;
   int64_t total;
   int num_ctas;
 
@@ -56,6 +61,8 @@ struct Sched {
     const int i_hi = last_row / G;
     return (ctx[b] + i_hi + 1 + kChunk - 1) / kChunk;
   }
+  __device__ int cost(int b, int rb) const { return chunks(b, rb) + E; }
+  // CTA whose range holds cost position x.
   __device__ int64_t owner(int64_t x) const {
     return ((x + 1) * num_ctas + total - 1) / total - 1;
   }
@@ -63,9 +70,9 @@ struct Sched {
 
 struct Seg {
   int b, kvh, rb;
-  int ci;        // first chunk (within the unit) of this segment
-  int nch;       // chunks of the unit
-  int64_t ust;   // global index of the unit's first chunk
+  int ci;        // cost offset of the position within the unit (0 .. E + nch - 1)
+  int nch;       // key slices of the unit
+  int64_t ust;   // cost position of the unit's start (its first real slice is at ust + E)
 };
 
 __device__ __forceinline__ Seg locate(const Sched &s, int64_t x) {
@@ -79,15 +86,15 @@ __device__ __forceinline__ Seg locate(const Sched &s, int64_t x) {
   g.nch = 0;
   const int nrb = s.rb_count(lo);
   int span = 0;
-  for (int rb = 0; rb < nrb; ++rb) span += s.chunks(lo, rb);
+  for (int rb = 0; rb < nrb; ++rb) span += s.cost(lo, rb);
   int64_t o = x - s.pref[lo];
   g.kvh = static_cast<int>(o / span);
   int o2 = static_cast<int>(o - static_cast<int64_t>(g.kvh) * span);
   int cum = 0;
   g.rb = 0;
   for (int rb = 0; rb < nrb; ++rb) {
-    const int c = s.chunks(lo, rb);
-    if (o2 < cum + c) { g.rb = rb; g.nch = c; break; }
+    const int c = s.cost(lo, rb);
+    if (o2 < cum + c) { g.rb = rb; g.nch = c - s.E; break; }
     cum += c;
   }
   g.ci = o2 - cum;
@@ -123,8 +130,8 @@ __device__ __forceinline__ void sched_validate(const Params &p, int32_t *s_ctx, 
   }
 }
 
-// Exclusive prefix over sequences of their chunk counts (one warp):
-// W_b = Hkv * sum over row blocks of chunks(b, rb).
+// Exclusive prefix over sequences of their costs (one warp):
+// W_b = Hkv * sum over row blocks of (chunks(b, rb) + E).
 __device__ __forceinline__ void sched_scan(const Params &p, const Sched &sc, int64_t *s_pref,
                                            int lane) {
   int64_t carry = 0;
@@ -134,7 +141,7 @@ __device__ __forceinline__ void sched_scan(const Params &p, const Sched &sc, int
     if (b < p.B) {
       const int nrb = sc.rb_count(b);
       int span = 0;
-      for (int rb = 0; rb < nrb; ++rb) span += sc.chunks(b, rb);
+      for (int rb = 0; rb < nrb; ++rb) span += sc.cost(b, rb);
       w = static_cast<int64_t>(p.Hkv) * span;
     }
     int64_t incl = w;

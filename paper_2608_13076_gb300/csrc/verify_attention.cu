@@ -90,7 +90,7 @@ __global__ void __launch_bounds__(Layout<D, MT>::THREADS, 1)
   block_sync();
   Sched sc;
   sc.pref = s_pref; sc.ctx = s_ctx; sc.kd = s_kd;
-  sc.B = p.B; sc.Hkv = p.Hkv; sc.G = p.G; sc.RB = p.RB; sc.num_ctas = p.num_ctas;
+  sc.B = p.B; sc.Hkv = p.Hkv; sc.G = p.G; sc.RB = p.RB; sc.E = p.unit_cost; sc.num_ctas = p.num_ctas;
   if (warp == 0) {
     sched_scan(p, sc, s_pref, lane);
   } else if (warp == 1 && lane == 0) {
@@ -379,8 +379,8 @@ __global__ void __launch_bounds__(Layout<D, MT>::THREADS, 1)
 
     // ---- emit: final output, or a partial for the cross-CTA merge ---------
     const int unit = (g.b * p.Hkv + g.kvh) * p.RB + g.rb;
-    const int64_t c_first = sc.owner(g.ust);
-    const int64_t c_last = sc.owner(g.ust + g.nch - 1);
+    const int64_t c_first = sc.owner(g.ust + sc.E);
+    const int64_t c_last = sc.owner(g.ust + sc.E + g.nch - 1);
     const int nparts = static_cast<int>(c_last - c_first + 1);
     const bool writer = (ks == 0) && active;
     if (nparts == 1) {
@@ -509,6 +509,10 @@ extern "C" spade_status spade_verify_attention(
   p.status = status;
   p.B = B; p.Hq = Hq; p.Hkv = Hkv; p.G = G; p.cap = cap; p.max_k = max_k; p.R = R; p.RB = RB;
   p.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(D));
+  // The tensor-memory kernel charges each unit's epilogue and pipeline restart
+  // to the CTA that starts it (about five slices' worth); the warp-MMA kernel
+  // keeps the plain split.
+  p.unit_cost = (D == 128) ? attn::kUnitCostTc : 0;
   // One CTA per SM, never more CTAs than key chunks could exist.
   const int64_t max_chunks = static_cast<int64_t>(units) * ((cap + attn::kChunk - 1) / attn::kChunk);
   p.num_ctas = static_cast<int>(max_chunks < sms ? max_chunks : sms);

@@ -142,19 +142,30 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-// One segment of a CTA's range: consecutive slices [x, seg_end) of one unit.
+// One segment of a CTA's range: the part of one unit's cost span in
+// [x, seg_end); its real key slices are g.ci .. g.ci + n_here - 1.
 struct SegInfo {
   Seg g;
   int64_t seg_end;
-  int n_here;   // slices in this segment
+  int n_here;   // key slices in this segment (0: only the unit's virtual start)
   int nchunk;   // MMA chunks (pairs of slices, the last one possibly single)
 };
 __device__ __forceinline__ SegInfo seg_at(const Sched &sc, int64_t x, int64_t x_end) {
   SegInfo s;
   s.g = locate(sc, x);
-  s.seg_end = min(x_end, s.g.ust + s.g.nch);
-  s.n_here = static_cast<int>(s.seg_end - x);
+  s.seg_end = min(x_end, s.g.ust + sc.E + s.g.nch);
+  const int lo = max(0, static_cast<int>(x - s.g.ust) - sc.E);
+  const int hi = max(0, static_cast<int>(s.seg_end - s.g.ust) - sc.E);
+  s.g.ci = lo;
+  s.n_here = hi - lo;
   s.nchunk = (s.n_here + 1) / 2;
+  return s;
+}
+// The first segment at or after cost position x that holds key slices (all
+// roles skip the same empty ones); n_here == 0 when the range has none left.
+__device__ __forceinline__ SegInfo next_seg(const Sched &sc, int64_t x, int64_t x_end) {
+  SegInfo s = seg_at(sc, x, x_end);
+  while (s.n_here == 0 && s.seg_end < x_end) s = seg_at(sc, s.seg_end, x_end);
   return s;
 }
 
@@ -190,7 +201,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   block_sync();
   Sched sc;
   sc.pref = s_pref; sc.ctx = s_ctx; sc.kd = s_kd;
-  sc.B = p.B; sc.Hkv = p.Hkv; sc.G = p.G; sc.RB = p.RB; sc.num_ctas = p.num_ctas;
+  sc.B = p.B; sc.Hkv = p.Hkv; sc.G = p.G; sc.RB = p.RB; sc.E = p.unit_cost; sc.num_ctas = p.num_ctas;
   if (warp == 0) {
     sched_scan(p, sc, s_pref, lane);
   } else if (warp == 1 && lane == 0) {
@@ -240,7 +251,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t it = 0, k_issued = 0, v_issued = 0;
       bool expired = false;
       for (int64_t x = x_begin; x < x_end;) {
-        const SegInfo si = seg_at(sc, x, x_end);
+        const SegInfo si = next_seg(sc, x, x_end);
+        if (si.n_here == 0) break;
         const int row0 = (si.g.b * p.Hkv + si.g.kvh) * p.cap;
         for (int c = 0; c < si.nchunk; ++c, ++it) {
           const int st = it % kStages;
@@ -311,7 +323,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (last) tc_commit(&bars[kBarOFinal]);
       };
       for (int64_t x = x_begin; x < x_end;) {
-        const SegInfo si = seg_at(sc, x, x_end);
+        const SegInfo si = next_seg(sc, x, x_end);
+        if (si.n_here == 0) break;
         if (!mbar_wait(&bars[kBarSeg], seg & 1, s_abort)) expired = true;  // Q staged, O^T free
         tc_fence_after();
         const uint32_t q_addr = smem_base + Smem::Q + (seg & 1) * 2 * kQSlab;
@@ -368,15 +381,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     };
 
-    SegInfo si = seg_at(sc, x_begin, x_end);
-    prefetch_q(si, 0);
+    SegInfo si = next_seg(sc, x_begin, x_end);
+    if (si.n_here > 0) prefetch_q(si, 0);
     cp_async_commit();
-    for (int64_t x = x_begin; x < x_end;) {
+    for (int64_t x = x_begin; x < x_end && si.n_here > 0;) {
       const Seg g = si.g;
       SegInfo si_next = si;
+      si_next.n_here = 0;
       if (si.seg_end < x_end) {
-        si_next = seg_at(sc, si.seg_end, x_end);
-        prefetch_q(si_next, (seg + 1) & 1);  // that buffer's last reader (unit seg-1) is done
+        si_next = next_seg(sc, si.seg_end, x_end);
+        if (si_next.n_here > 0) prefetch_q(si_next, (seg + 1) & 1);  // that buffer's last reader (unit seg-1) is done
       }
       cp_async_commit();
       const int ctx = s_ctx[g.b];
@@ -550,8 +564,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait(&bars[kBarOFinal], seg & 1, s_abort)) expired = true;
       tc_fence_after();
       const int unit = (g.b * p.Hkv + g.kvh) * p.RB + g.rb;
-      const int64_t c_first = sc.owner(g.ust);
-      const int64_t c_last = sc.owner(g.ust + g.nch - 1);
+      const int64_t c_first = sc.owner(g.ust + sc.E);
+      const int64_t c_last = sc.owner(g.ust + sc.E + g.nch - 1);
       const int nparts = static_cast<int>(c_last - c_first + 1);
       if (nparts == 1) {
 #pragma unroll
