@@ -178,13 +178,22 @@ def run_spade(args, ws, rank, local):
                                      workspace=ws_attn, status=status)
         if evs:
             evs[1].record(stream)
-        spade.spade_verify_accept(inputs["hidden"], wl["w_lm"], inputs["draft_tokens"], inputs["draft_probs"],
-                                  inputs["uniforms"], inputs["mode"], inputs["cu_q"], inputs["n_draft"], acc,
-                                  tok, workspace=ws_acc, status=status)
-        if evs:
-            evs[2].record(stream)
-        spade.spade_kv_commit(wl["k_cache"], wl["v_cache"], inputs["ctx_lens"], acc, inputs["n_draft"],
-                              status=status)
+        if args.separate_commit:
+            spade.spade_verify_accept(inputs["hidden"], wl["w_lm"], inputs["draft_tokens"],
+                                      inputs["draft_probs"], inputs["uniforms"], inputs["mode"], inputs["cu_q"],
+                                      inputs["n_draft"], acc, tok, workspace=ws_acc, status=status)
+            if evs:
+                evs[2].record(stream)
+            spade.spade_kv_commit(wl["k_cache"], wl["v_cache"], inputs["ctx_lens"], acc, inputs["n_draft"],
+                                  status=status)
+        else:
+            # Accept + KV commit in one launch (the commit runs inside the LM-head kernel).
+            spade.spade_verify_accept_commit(inputs["hidden"], wl["w_lm"], inputs["draft_tokens"],
+                                             inputs["draft_probs"], inputs["uniforms"], inputs["mode"],
+                                             inputs["cu_q"], inputs["n_draft"], acc, tok, wl["k_cache"],
+                                             wl["v_cache"], inputs["ctx_lens"], workspace=ws_acc, status=status)
+            if evs:
+                evs[2].record(stream)
         if evs:
             evs[3].record(stream)
 
@@ -285,10 +294,11 @@ def run_spade(args, ws, rank, local):
                    "l2": "flushed between steps" if flush else f"working set {work_set / 1e9:.2f} GB > L2"},
         "tokens_per_step": tokens_per_step,
         "accepted_len": acc.tolist(),
-        "kernels_us": {"verify_attention": m_attn * 1e6, "verify_accept": m_acc * 1e6,
-                       "kv_commit": statistics.mean(t_com) * 1e6},
+        "kernels_us": ({"verify_attention": m_attn * 1e6, "verify_accept": m_acc * 1e6,
+                        "kv_commit": statistics.mean(t_com) * 1e6} if args.separate_commit else
+                       {"verify_attention": m_attn * 1e6, "verify_accept_commit": m_acc * 1e6}),
         "roofline": dominant, "roofline_attention": roof_attn, "roofline_lm_head": roof_lm,
-        "e2e": e2e, "gpu_launches": 3 * args.steps, "wall_s_timed_loop": t_wall,
+        "e2e": e2e, "gpu_launches": (3 if args.separate_commit else 2) * args.steps, "wall_s_timed_loop": t_wall,
         "clocks": clk.summary(),
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -375,6 +385,8 @@ def main():
     ap.add_argument("--workload", default="llama3_8b", choices=sorted(W.SPECS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--separate-commit", action="store_true",
+                    help="run the KV commit as its own launch instead of inside the LM-head kernel")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3) if args.impl == "spade" else args.warmup
     ws, rank, local = _dist()

@@ -15,6 +15,7 @@
  *                           sampling from norm(max(0, p - q)) (Sec. III-C)
  *   spade_kv_commit         context update m <- m + a + 1 (Algorithm 1) on the
  *                           KV cache: keep accepted slots, clear rejected ones
+ *   spade_verify_accept_commit  the two calls above fused into one launch
  *
  * Conventions shared by every call
  *  - Every pointer argument is a DEVICE pointer owned by the caller; the
@@ -179,6 +180,32 @@ spade_status spade_verify_accept(const void *hidden, const void *w_lm,
 
 /* Bytes of workspace spade_verify_accept needs (0 on invalid sizes). */
 size_t spade_accept_workspace_size(int32_t B, int32_t R, int32_t H, int32_t V);
+
+/*
+ * spade_verify_accept followed by spade_kv_commit, in one launch: once the
+ * accept decisions are taken on the device, the same kernel clears the
+ * rejected draft slots [ctx_b + a_b + 1, ctx_b + n_draft[b]] of k_cache and
+ * v_cache (every KV head) and advances ctx_lens[b] by a_b + 1, exactly as
+ * spade_kv_commit does (Algorithm 1's context update), so a verify step needs
+ * one launch fewer.  Arguments are those of the two calls:
+ *   k_cache, v_cache bf16 [B, Hkv, cap, D], 16-byte aligned, D % 8 == 0,
+ *                    updated in place
+ *   ctx_lens         int32 [B], read and updated in place
+ * Sequences with an invalid verify block are left untouched and reported in
+ * `status` (SPADE_DEV_BAD_INDEX / SPADE_DEV_CAPACITY), as by spade_kv_commit.
+ * The caller must not have another kernel reading the caches or ctx_lens
+ * concurrently (the step's attention is ordered before this call on `stream`).
+ */
+spade_status spade_verify_accept_commit(const void *hidden, const void *w_lm,
+                                        const int32_t *draft_tokens, const float *draft_probs,
+                                        const float *uniforms, const int32_t *mode,
+                                        const int32_t *cu_q, const int32_t *n_draft,
+                                        int32_t *accepted_len, int32_t *next_token,
+                                        void *k_cache, void *v_cache, int32_t *ctx_lens,
+                                        int32_t B, int32_t R, int32_t H, int32_t V, int32_t Hkv,
+                                        int32_t D, int32_t cap, void *workspace,
+                                        size_t workspace_bytes, int32_t *status,
+                                        spade_stream_t stream);
 
 /* ------------------------------------------------------------------------ */
 /* KV commit (Algorithm 1 context update)                                    */

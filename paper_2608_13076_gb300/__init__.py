@@ -77,6 +77,8 @@ def load():
     lib.spade_attn_workspace_size.argtypes = [_i32] * 6
     lib.spade_verify_accept.restype = _i32
     lib.spade_verify_accept.argtypes = [_vp] * 10 + [_i32] * 4 + [_vp, _sz, _vp, _vp]
+    lib.spade_verify_accept_commit.restype = _i32
+    lib.spade_verify_accept_commit.argtypes = [_vp] * 13 + [_i32] * 7 + [_vp, _sz, _vp, _vp]
     lib.spade_accept_workspace_size.restype = _sz
     lib.spade_accept_workspace_size.argtypes = [_i32] * 4
     lib.spade_kv_commit.restype = _i32
@@ -227,6 +229,41 @@ def spade_verify_accept(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode,
         _ptr(hidden), _ptr(w_lm), _ptr(draft_tokens), _ptr(draft_probs), _ptr(uniforms), _ptr(mode),
         _ptr(cu_q), _ptr(n_draft), _ptr(accepted_len), _ptr(next_token), B, R, H, V,
         _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream))
+    _check_rc(rc)
+    return accepted_len, next_token
+
+
+def spade_verify_accept_commit(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
+                               accepted_len, next_token, k_cache, v_cache, ctx_lens, *, workspace,
+                               status, stream=None):
+    """spade_verify_accept followed by spade_kv_commit in one launch (see include/spade.h)."""
+    _need(hidden, "hidden", torch.bfloat16, 2)
+    _need(w_lm, "w_lm", torch.bfloat16, 2)
+    _need(uniforms, "uniforms", torch.float32, 1)
+    for t, n in ((draft_tokens, "draft_tokens"), (mode, "mode"), (cu_q, "cu_q"), (n_draft, "n_draft"),
+                 (accepted_len, "accepted_len"), (next_token, "next_token"), (status, "status"),
+                 (ctx_lens, "ctx_lens")):
+        _need(t, n, torch.int32, 1)
+    if draft_probs is not None:
+        _need(draft_probs, "draft_probs", torch.float32, 2)
+    _need(workspace, "workspace", torch.uint8, 1)
+    _need(k_cache, "k_cache", torch.bfloat16, 4)
+    _need(v_cache, "v_cache", torch.bfloat16, 4)
+    R, H = hidden.shape
+    V, H2 = w_lm.shape
+    B = n_draft.numel()
+    Bc, Hkv, cap, D = k_cache.shape
+    if H2 != H or uniforms.numel() != R or draft_tokens.numel() != R - B or cu_q.numel() != B + 1 \
+            or mode.numel() != B or accepted_len.numel() != B or next_token.numel() != B \
+            or Bc != B or tuple(v_cache.shape) != tuple(k_cache.shape) or ctx_lens.numel() != B:
+        raise ValueError("inconsistent accept/commit shapes")
+    if draft_probs is not None and tuple(draft_probs.shape) != (R - B, V):
+        raise ValueError("draft_probs must be [R - B, V]")
+    rc = load().spade_verify_accept_commit(
+        _ptr(hidden), _ptr(w_lm), _ptr(draft_tokens), _ptr(draft_probs), _ptr(uniforms), _ptr(mode),
+        _ptr(cu_q), _ptr(n_draft), _ptr(accepted_len), _ptr(next_token), _ptr(k_cache), _ptr(v_cache),
+        _ptr(ctx_lens), B, R, H, V, Hkv, D, cap, _ptr(workspace), workspace.numel(), _ptr(status),
+        _stream(stream))
     _check_rc(rc)
     return accepted_len, next_token
 

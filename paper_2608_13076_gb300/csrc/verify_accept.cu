@@ -79,6 +79,11 @@ struct Params {
   int *samp_count;   // number of specs
   __nv_bfloat16 *hidden_s;      // [B, H]: gathered hidden rows of the samples
   const __nv_bfloat16 *hidden;  // the call's hidden rows (gather source)
+  // Fused KV commit (null kc: not requested): clear the rejected draft slots of
+  // the caches [B, Hkv, cap, Dk] and advance ctx_lens once the decisions exist.
+  uint4 *kc, *vc;
+  int32_t *ctx_lens;
+  int Hkv, Dk, cap;
   int kind;
   int nchunks;       // MMA N-chunks per tile (2 when Ncols > 256)
   int n0w;           // width of the first N-chunk
@@ -703,6 +708,37 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   }
   block_sync();
 
+  // ---- fused KV commit (Algorithm 1 context update) -----------------------
+  // The decisions are known: sequence b (b = c, c + NC, ...) keeps slots
+  // [0, ctx_b + a_b] and its rejected drafts' slots [ctx_b + a_b + 1, ctx_b +
+  // k_b] are cleared; ctx_lens[b] advances by a_b + 1.  Warps 0-1 do it (they
+  // are idle in phase C); this step's attention has finished with the cache.
+  if (p.kc != nullptr && p.kind != kPresampled && warp < 2) {
+    for (int b = c; b < p.B; b += p.NC) {
+      const int a = s_acc[b];
+      if (a < 0) continue;  // invalid sequence: reported, left untouched
+      const int k = s_nd[b];
+      const int ctx = p.ctx_lens[b];
+      if (ctx < 0 || static_cast<int64_t>(ctx) + k + 1 > p.cap) {
+        if (tid == 0) atomicOr(p.status, ctx < 0 ? SPADE_DEV_BAD_INDEX : SPADE_DEV_CAPACITY);
+        continue;
+      }
+      const int lo = ctx + a + 1;
+      const int vec = p.Dk / 8;  // 16-byte vectors per slot
+      const int per_head = (k - a) * vec;
+      const int total = p.Hkv * per_head;
+      const uint4 z = make_uint4(0, 0, 0, 0);
+      for (int e = tid; e < total; e += 64) {
+        const int h = e / per_head;
+        const size_t off = ((static_cast<size_t>(b) * p.Hkv + h) * p.cap + lo) * vec + (e - h * per_head);
+        p.kc[off] = z;
+        p.vc[off] = z;
+      }
+      named_bar(2, 64);  // every thread has read ctx_lens[b] before it changes
+      if (tid == 0) p.ctx_lens[b] = lo;
+    }
+  }
+
   if (p.kind == kStatsOnly) {
     // First pass of the two-pass path: publish one sample spec per sequence
     // that needs a draw and gather its hidden row for the second pass.
@@ -1232,14 +1268,21 @@ extern "C" size_t spade_accept_workspace_size(int32_t B, int32_t R, int32_t H, i
   return accept::ws_layout(B, R, H, V, sms).end;
 }
 
-extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm,
-                                            const int32_t *draft_tokens, const float *draft_probs,
-                                            const float *uniforms, const int32_t *mode,
-                                            const int32_t *cu_q, const int32_t *n_draft,
-                                            int32_t *accepted_len, int32_t *next_token, int32_t B,
-                                            int32_t R, int32_t H, int32_t V, void *workspace,
-                                            size_t workspace_bytes, int32_t *status,
-                                            spade_stream_t stream) {
+namespace spade {
+namespace accept {
+struct CommitArgs {
+  void *k_cache, *v_cache;
+  int32_t *ctx_lens;
+  int Hkv, D, cap;
+};
+static spade_status verify_accept_impl(const void *hidden, const void *w_lm,
+                                       const int32_t *draft_tokens, const float *draft_probs,
+                                       const float *uniforms, const int32_t *mode,
+                                       const int32_t *cu_q, const int32_t *n_draft,
+                                       int32_t *accepted_len, int32_t *next_token, int32_t B,
+                                       int32_t R, int32_t H, int32_t V, void *workspace,
+                                       size_t workspace_bytes, int32_t *status,
+                                       spade_stream_t stream, const CommitArgs *cm) {
   using namespace accept;
   if (!hidden || !w_lm || !uniforms || !mode || !cu_q || !n_draft || !accepted_len ||
       !next_token || !status || (R > B && !draft_tokens))
@@ -1277,6 +1320,14 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
   p.V = V;
   p.hidden = static_cast<const __nv_bfloat16 *>(hidden);
   p.bar = reinterpret_cast<unsigned *>(ws);
+  if (cm) {
+    p.kc = static_cast<uint4 *>(cm->k_cache);
+    p.vc = static_cast<uint4 *>(cm->v_cache);
+    p.ctx_lens = cm->ctx_lens;
+    p.Hkv = cm->Hkv;
+    p.Dk = cm->D;
+    p.cap = cm->cap;
+  }
   set_region(p, ws, L.r1);
   Maps m;
   if (!L.two_pass) {
@@ -1294,8 +1345,43 @@ extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm
   st = launch(p, m, s);
   if (st != SPADE_OK) return st;
   Params p2 = p;
+  p2.kc = p2.vc = nullptr;  // the first pass committed
   set_region(p2, ws, L.r2);
   st = prepare(p2, kPresampled, p.hidden_s, w_lm, B, sms, m);
   if (st != SPADE_OK) return st;
   return launch(p2, m, s);
+}
+}  // namespace accept
+}  // namespace spade
+
+extern "C" spade_status spade_verify_accept(const void *hidden, const void *w_lm,
+                                            const int32_t *draft_tokens, const float *draft_probs,
+                                            const float *uniforms, const int32_t *mode,
+                                            const int32_t *cu_q, const int32_t *n_draft,
+                                            int32_t *accepted_len, int32_t *next_token, int32_t B,
+                                            int32_t R, int32_t H, int32_t V, void *workspace,
+                                            size_t workspace_bytes, int32_t *status,
+                                            spade_stream_t stream) {
+  return accept::verify_accept_impl(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q,
+                                    n_draft, accepted_len, next_token, B, R, H, V, workspace,
+                                    workspace_bytes, status, stream, nullptr);
+}
+
+extern "C" spade_status spade_verify_accept_commit(
+    const void *hidden, const void *w_lm, const int32_t *draft_tokens, const float *draft_probs,
+    const float *uniforms, const int32_t *mode, const int32_t *cu_q, const int32_t *n_draft,
+    int32_t *accepted_len, int32_t *next_token, void *k_cache, void *v_cache, int32_t *ctx_lens,
+    int32_t B, int32_t R, int32_t H, int32_t V, int32_t Hkv, int32_t D, int32_t cap,
+    void *workspace, size_t workspace_bytes, int32_t *status, spade_stream_t stream) {
+  if (!k_cache || !v_cache || !ctx_lens)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_commit: null cache or ctx_lens pointer");
+  if (Hkv <= 0 || D <= 0 || cap <= 0)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_commit: non-positive cache size");
+  if (D % 8) return fail(SPADE_ERR_SHAPE, "spade_verify_accept_commit: D = %d must be a multiple of 8", D);
+  if (!aligned(k_cache, 16) || !aligned(v_cache, 16))
+    return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_commit: caches must be 16-byte aligned");
+  const accept::CommitArgs cm{k_cache, v_cache, ctx_lens, Hkv, D, cap};
+  return accept::verify_accept_impl(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q,
+                                    n_draft, accepted_len, next_token, B, R, H, V, workspace,
+                                    workspace_bytes, status, stream, &cm);
 }

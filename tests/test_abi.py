@@ -30,7 +30,7 @@ def lib():
 
 def test_header_declares_the_entry_points():
     names = declared_functions()
-    for n in ("spade_verify_attention", "spade_verify_accept", "spade_kv_commit",
+    for n in ("spade_verify_attention", "spade_verify_accept", "spade_kv_commit", "spade_verify_accept_commit",
               "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_last_error",
               "spade_status_string"):
         assert n in names
@@ -67,6 +67,8 @@ def test_null_arguments_rejected_before_any_device_work(lib):
     assert rc == 1
     rc = lib.spade_kv_commit(*([None] * 5), 1, 8, 128, 300, None, None)
     assert rc == 1
+    rc = lib.spade_verify_accept_commit(*([None] * 13), 1, 5, 512, 1024, 8, 128, 300, None, 0, None, None)
+    assert rc == 1
 
 
 def test_bad_shapes_rejected(lib):
@@ -80,3 +82,4 @@ def test_bad_shapes_rejected(lib):
     assert lib.spade_verify_accept(*([p] * 10), 1, 5, 500, 1024, p, 1 << 20, p, None) == 2
     # head dim not a multiple of 8 for commit
     assert lib.spade_kv_commit(*([p] * 5), 1, 8, 12, 300, p, None) == 2
+    assert lib.spade_verify_accept_commit(*([p] * 13), 1, 5, 512, 1024, 8, 12, 300, p, 1 << 20, p, None) == 2

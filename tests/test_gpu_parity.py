@@ -88,6 +88,29 @@ def test_kv_commit_small(dev, name):
     assert np.array_equal(parity.to_np(vc), rv)
 
 
+@pytest.mark.parametrize("name", sorted(SMALL))
+def test_accept_commit_fused_small(dev, name):
+    """The fused accept + commit launch equals the two separate calls bit for bit."""
+    wl = W.make_workload(SMALL[name], device=dev, cache_pad=5)
+    acc, tok, st = parity.gpu_accept(wl)
+    kc, vc, ctx = wl["k_cache"].clone(), wl["v_cache"].clone(), wl["ctx_lens"].clone()
+    spade.spade_kv_commit(kc, vc, ctx, acc, wl["n_draft"], status=st)
+    B = wl["B"]
+    acc2 = torch.full((B,), -7, dtype=torch.int32, device=dev)
+    tok2 = torch.full((B,), -7, dtype=torch.int32, device=dev)
+    kc2, vc2, ctx2 = wl["k_cache"].clone(), wl["v_cache"].clone(), wl["ctx_lens"].clone()
+    st2 = spade.status_tensor(dev)
+    ws = spade.accept_workspace(B, wl["R"], wl["H"], wl["V"], device=dev)
+    spade.spade_verify_accept_commit(wl["hidden"], wl["w_lm"], wl["draft_tokens"], wl["draft_probs"],
+                                     wl["uniforms"], wl["mode"], wl["cu_q"], wl["n_draft"], acc2, tok2,
+                                     kc2, vc2, ctx2, workspace=ws, status=st2)
+    torch.cuda.synchronize()
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0 and int(st2.item()) & ~spade.DEV_FALLBACK == 0
+    assert torch.equal(acc2, acc) and torch.equal(tok2, tok)
+    assert torch.equal(ctx2, ctx)
+    assert torch.equal(kc2, kc) and torch.equal(vc2, vc)
+
+
 def test_repeat_calls_reuse_workspace(dev):
     """Workspaces stay valid across calls (self-resetting counters / barriers)."""
     spec = SMALL["many_rows"]
