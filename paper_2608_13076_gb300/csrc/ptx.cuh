@@ -101,6 +101,16 @@ SPADE_DEVICE uint64_t l2_policy_evict_last() {
   asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
   return pol;
 }
+// Plain bulk copy of `bytes` from global to shared memory, completing on
+// `bar`.  Both addresses 16-byte aligned; `bytes` a multiple of 16.
+SPADE_DEVICE void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(static_cast<uint64_t>(__cvta_generic_to_global(src))), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
 // 2-D tiled load of box {x: inner, y: rows} at coordinates (x, y) into smem,
 // completing `bytes` on `bar`.  x * elemsize must be a multiple of 16 bytes.
 SPADE_DEVICE void tma_load_2d(void *dst, const CUtensorMap *map, int32_t x, int32_t y,

@@ -53,6 +53,17 @@ constexpr int kMaxRounds = 32;
 constexpr int kResident = 0, kStatsOnly = 1, kPresampled = 2;
 constexpr int kMaxTilesPerCta = 32;
 constexpr int kMaxNC = 256;  // CTAs (vocabulary slices) per launch
+// Residual masses through shared memory (phase C): groups of kFG sampled rows
+// are staged as p and q slices, then every thread sums 32-entry segments
+// serially; slices of at most kFastSlice vocab rows, at most kFastSeqs sampled
+// rows (else the register path below).
+constexpr int kFG = 8;
+static_assert(kFG <= 32, "one lane prepares each staged row");
+constexpr int kFastSlice = 1024;
+constexpr int kFastSegs = kFastSlice / 32;
+constexpr int kFastSeqs = 64;
+constexpr int kQStride = kFastSlice + 4;  // floats per staged q row (16-byte multiple)
+constexpr int kSegPad = 33;               // floats per staged 32-entry segment (bank skew)
 constexpr int kTmemCols = 512;
 constexpr int kSmemBudget = 220 * 1024;
 constexpr int kSmemMax = 225 * 1024;  // opt-in limit (227 KB) minus static shared memory
@@ -69,11 +80,11 @@ struct Params {
   int32_t *accepted_len;
   int32_t *next_token;
   int32_t *status;
-  unsigned *bar;     // [0]: arrival count, [kGenWord]: generation
+  unsigned *bar;     // [0]: arrival count, [kGenWord * (1 + r)]: generation copy r
   float4 *pstat;     // [NC][R]: slice max, slice sum-exp, slice argmax (bits), -
   float *ldraft;     // [R]: logit of the row's draft token
-  float4 *gstat;     // [R]: merged row max, sum-exp, argmax (bits)
-  float4 *zpart;     // [NC][B]: slice mass of the sampled distribution and of p (float-float)
+  float4 *gstat;     // [kReplicas][R]: merged row max, sum-exp, argmax (bits)
+  float2 *zpart;     // [kReplicas][NC][B]: slice mass of the sampled distribution (float-float)
   int4 *samp;        // [B]: sample specs written by kStatsOnly, read by kPresampled:
                      //      draft_probs row (-1: sample p), uniform bits, output index, row
   int *samp_count;   // number of specs
@@ -98,6 +109,8 @@ struct Params {
   int round_tiles[kMaxRounds];
   int HS, WS;        // hidden / W ring slots
   int BRS;           // box rows of the map used for a slice's last, partial tile
+  int fastc;         // phase C through shared memory (slices <= kFastSlice, room in the rings)
+  int qbulk;         // q rows may be bulk-copied (16-byte aligned rows)
   uint32_t idesc;
   uint32_t tmem_cols;
 };
@@ -144,19 +157,28 @@ __device__ __forceinline__ unsigned ld_relaxed(const unsigned *p) {
 // Word offset of the grid barrier's generation counter: its own 128-byte line,
 // apart from the arrival count, so the waiting CTAs' polls do not queue behind
 // the arrival atomics on one L2 line.
-constexpr int kGenWord = 32;
-static_assert(kGenWord * 4 + 4 <= 256, "barrier words live in the workspace's first 256 bytes");
+// Data that every CTA reads right after a grid barrier (the merged row
+// statistics, the slice masses) is written in kReplicas copies, and CTA c reads
+// copy c % kReplicas: 152 CTAs loading the same L2 lines at once queue on them
+// for several microseconds, a handful per line do not.  The barrier's
+// generation word is replicated the same way, one 128-byte line per copy.
+constexpr int kReplicas = 8;
+constexpr int kGenWord = 32;      // words between the arrival count and each generation copy
+constexpr int kBarBytes = 2048;  // barrier words at the workspace's start
+static_assert(kGenWord * (kReplicas + 1) * 4 <= kBarBytes, "barrier words fit their region");
 
 // Device-wide barrier among the NC co-resident CTAs (cooperative launch).  The
 // last CTA to arrive resets the count and bumps the generation; the others
 // poll the generation (relaxed loads with a short back-off, then an acquire
 // fence) with a time limit.  Returns false if the wait expired.
-__device__ bool grid_barrier(unsigned *bar, int nctas) {
+// Not inlined: the kernel passes it four times after the vocabulary sweep,
+// and one copy of its code stays in the instruction cache.
+__device__ __noinline__ bool grid_barrier(unsigned *bar, int nctas) {
   __shared__ int s_ok;
   block_sync();
   if (threadIdx.x == 0) {
     s_ok = 1;
-    unsigned *gen_p = bar + kGenWord;
+    unsigned *gen_p = bar + kGenWord * (1 + blockIdx.x % kReplicas);
     // Read before arriving (the arrival's release orders this load first).
     const unsigned gen = ld_relaxed(gen_p);
     unsigned arrived;
@@ -164,7 +186,10 @@ __device__ bool grid_barrier(unsigned *bar, int nctas) {
     asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(arrived) : "l"(bar) : "memory");
     if (arrived == static_cast<unsigned>(nctas) - 1) {
       asm volatile("st.relaxed.gpu.global.u32 [%0], 0;" ::"l"(bar) : "memory");
-      asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(gen_p) : "memory");
+      // One release fence orders everything above before all the copies.
+      asm volatile("fence.acq_rel.gpu;" ::: "memory");
+      for (int r = 0; r < kReplicas; ++r)
+        asm volatile("red.relaxed.gpu.global.add.u32 [%0], 1;" ::"l"(bar + kGenWord * (1 + r)) : "memory");
     } else {
       const uint64_t t0 = globaltimer();
       while (ld_relaxed(gen_p) == gen) {
@@ -251,8 +276,9 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     const __grid_constant__ CUtensorMap tm_w2, const __grid_constant__ CUtensorMap tm_w2s,
     const __grid_constant__ CUtensorMap tm_h3, const __grid_constant__ CUtensorMap tm_h2) {
   extern __shared__ uint8_t smem_raw[];
-  uint8_t *smem = reinterpret_cast<uint8_t *>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // 1024-byte aligned base, derived by pointer arithmetic so that the compiler
+  // keeps the shared state space (plain ld/st.shared, not generic accesses).
+  uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const Smem L = smem_layout(p);
   uint8_t *w_ring = smem;
   uint8_t *h_ring = smem + L.off_h;
@@ -265,6 +291,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L.off_misc);
   uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + L.off_misc + 8);
   int *s_any_stoch = reinterpret_cast<int *>(smem + L.off_misc + 16);
+  uint64_t *q_bar = reinterpret_cast<uint64_t *>(smem + L.off_misc + 24);  // q slice bulk copies
   int32_t *s_draft = reinterpret_cast<int32_t *>(smem + L.off_rows);
   int32_t *s_seq = s_draft + kMaxR;
   int32_t *s_pos = s_seq + kMaxR;
@@ -295,6 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     for (int s = 0; s < p.HS; ++s) { mbar_init(&h_full[s], 1); mbar_init(&h_empty[s], 1); }
     mbar_init(acc_full, 1);
     mbar_init(acc_empty, kEpiWarps);
+    mbar_init(q_bar, 33);  // thread 0 (with the copies' bytes) and the 32 lanes of warp 1
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -611,7 +639,11 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
         stat_merge(m, sm, idx, om, os, oi);
       }
-      if (lane == 0) __stcg(&p.gstat[n], make_float4(m, sm, __int_as_float(idx), 0.f));
+      // Every copy holds lane 0's values.
+      m = __shfl_sync(0xffffffffu, m, 0);
+      sm = __shfl_sync(0xffffffffu, sm, 0);
+      idx = __shfl_sync(0xffffffffu, idx, 0);
+      if (lane < kReplicas) __stcg(&p.gstat[static_cast<size_t>(lane) * p.R + n], make_float4(m, sm, __int_as_float(idx), 0.f));
     }
   }
   if (!grid_barrier(p.bar, p.NC)) {
@@ -631,13 +663,19 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   int *s_qidx = s_stoch + kMaxB;                            // [B] draft_probs row, -1: p
   float *s_usmp = reinterpret_cast<float *>(s_qidx + kMaxB); // [B] sampling uniform
   int *s_outb = reinterpret_cast<int *>(s_usmp + kMaxB);    // [B] next_token index
-  int *s_seg = s_outb + kMaxB;                              // [2]: tile, quarter; [4]: count
+  int *s_seg = s_outb + kMaxB;  // [0..1] tile, quarter; [4], [5] row counts; [6..7] retry flags
   float2 *s_T = reinterpret_cast<float2 *>(s_seg + 16);     // [B] float-float
   float4 *s_zw = reinterpret_cast<float4 *>(s_T + kMaxB);   // [B][kEpiWarps]
   float2 *s_tw = reinterpret_cast<float2 *>(s_zw + kMaxB * kEpiWarps);  // [tiles][kEpiWarps]
+  int *s_slist = reinterpret_cast<int *>(s_tw + kMaxTilesPerCta * kEpiWarps);  // [B] sampled sequences
+  int *s_slpos = s_slist + kMaxB;                           // [B] position in s_slist, -1: none
+  float *f_R = reinterpret_cast<float *>(s_slpos + kMaxB);  // [kFG][kFastSegs][kSegPad] residual terms
+  float *f_Q = f_R + kFG * kFastSegs * kSegPad;             // [kFG][kQStride] q of staged rows
+  float2 *f_seg = reinterpret_cast<float2 *>(f_Q + kFG * kQStride);  // [kFastSeqs][kFastSegs]
+  uint32_t q_phase = 0;
   // (2) Every CTA reads the merged statistics of all rows.
   for (int n = tid; n < p.R; n += kThreads) {
-    const float4 g = __ldcg(&p.gstat[n]);
+    const float4 g = __ldcg(&p.gstat[static_cast<size_t>(c % kReplicas) * p.R + n]);
     g_m[n] = g.x;
     g_s[n] = g.y;
     g_arg[n] = __float_as_int(g.z);
@@ -767,147 +805,335 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     // Terms are fp32 (p = 2^((l - m) log2 e) / Z on the SFU, the same formula
     // here and in phase D, so the slice and segment masses agree); every sum is
     // float-float, so the cumulative masses that place u*Z are as exact as the
-    // terms allow.
-    if (warp >= 2) {
-      const int ew = warp - 2, q4 = warp & 3;
-      const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
-      // Stochastic sequences in groups of kG: the TMEM reads and q loads of a
-      // whole group are in flight together.
-      constexpr int kG = 4;
-      for (int b0 = 0; b0 < p.B;) {
-        int bl[kG], nb = 0;
-        while (b0 < p.B && nb < kG) {
-          if (s_stoch[b0]) bl[nb++] = b0;
-          ++b0;
+    // terms allow.  Attempt 0 sums the residual max(0, p - q) (p for a bonus
+    // row).  A sequence whose residual has no mass at all falls back to p: a
+    // second attempt sums p for those sequences only.  Every CTA reads the
+    // same slice masses, so all take the same number of attempts.
+    // The sampled sequences, in order (warp 0 compacts them).
+    if (warp == 0) {
+      int base = 0;
+      for (int b0 = 0; b0 < p.B; b0 += 32) {
+        const int b = b0 + lane;
+        const bool st = b < p.B && s_stoch[b];
+        const unsigned m = __ballot_sync(0xffffffffu, st);
+        if (st) s_slist[base + __popc(m & ((1u << lane) - 1u))] = b;
+        if (b < p.B) {
+          s_slpos[b] = st ? base + __popc(m & ((1u << lane) - 1u)) : -1;
+          s_usep[b] = 0;
         }
-        if (nb == 0) break;
-        const float *qrow[kG];
-        int nrow[kG];
-        float M[kG], invS[kG];
-        ff2 z[kG], zp[kG];
-#pragma unroll
-        for (int g = 0; g < kG; ++g) {
-          const int b = g < nb ? bl[g] : bl[0];
-          nrow[g] = s_rstar[b];
-          qrow[g] = s_qidx[b] >= 0 ? p.draft_probs + static_cast<size_t>(s_qidx[b]) * p.V : nullptr;
-          M[g] = g_m[nrow[g]];
-          invS[g] = 1.f / g_s[nrow[g]];
-          z[g] = ff2{0.f, 0.f};
-          zp[g] = ff2{0.f, 0.f};
-        }
-        for (int j0 = 0; j0 < ntiles; j0 += 8) {
-          const int nj = min(8, ntiles - j0);
-          uint32_t raw[kG][8];
-          float qv[kG][8];
-#pragma unroll
-          for (int g = 0; g < kG; ++g) {
-#pragma unroll
-            for (int j = 0; j < 8; ++j)
-              if (g < nb && j < nj)
-                tmem_ld1(tmem + lane_base + static_cast<uint32_t>((j0 + j) * p.Rs + nrow[g]), raw[g][j]);
-          }
-#pragma unroll
-          for (int g = 0; g < kG; ++g) {
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-              const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
-              qv[g][j] = (g < nb && j < nj && qrow[g] && v < v_hi) ? qrow[g][v] : 0.f;
-            }
-          }
-          tmem_wait_ld();
-#pragma unroll
-          for (int g = 0; g < kG; ++g) {
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-              const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
-              if (g < nb && j < nj && v < v_hi) {
-                const float pv = ex2((__uint_as_float(raw[g][j]) - M[g]) * kLog2e) * invS[g];
-                zp[g] = ff_add_f(zp[g], pv);
-                z[g] = ff_add_f(z[g], qrow[g] ? fmaxf(0.f, pv - qv[g][j]) : pv);
-              }
-            }
-          }
-        }
-#pragma unroll
-        for (int g = 0; g < kG; ++g) {
-          z[g] = warp_sum_ff(z[g]);
-          zp[g] = warp_sum_ff(zp[g]);
-          if (lane == 0 && g < nb) s_zw[bl[g] * kEpiWarps + ew] = make_float4(z[g].hi, z[g].lo, zp[g].hi, zp[g].lo);
-        }
+        base += __popc(m);
+      }
+      if (lane == 0) {
+        s_seg[5] = base;
+        s_seg[6] = s_seg[7] = 0;  // per attempt: some residual had no mass
       }
     }
     block_sync();
-    for (int b = tid; b < p.B; b += kThreads) {
-      if (!s_stoch[b]) continue;
-      ff2 zs{0.f, 0.f}, zps{0.f, 0.f};
-      for (int w = 0; w < kEpiWarps; ++w) {
-        const float4 t = s_zw[b * kEpiWarps + w];
-        zs = ff_add(zs, ff2{t.x, t.y});
-        zps = ff_add(zps, ff2{t.z, t.w});
-      }
-      __stcg(&p.zpart[static_cast<size_t>(c) * p.B + b], make_float4(zs.hi, zs.lo, zps.hi, zps.lo));
-    }
-    if (!grid_barrier(p.bar, p.NC)) {
-      atomicOr(p.status, SPADE_DEV_TIMEOUT);
-      *s_abort = 1;
-    }
-    // =================== phase D: owner slice of u*Z, in-slice scan =========
-    // One warp per sequence: all NC slice masses in registers (one round of
-    // loads), their total, then a chunked prefix scan for the first slice whose
-    // cumulative mass passes u*Z.
-    constexpr int kZC = kMaxNC / 32;
-    for (int b = warp; b < p.B; b += kThreads / 32) {
-      if (!s_stoch[b]) { if (lane == 0) s_owner[b] = -1; continue; }
-      float4 zz[kZC];
+    const int ns = s_seg[5];
+    const int slen = v_hi - v_lo;
+    const int nseg = (slen + 31) / 32;
+    const bool fastc = p.fastc && ns <= kFastSeqs;  // the same on every CTA
+#pragma unroll 1  // one copy of the code: the second attempt is rare
+    for (int attempt = 0; attempt < 2; ++attempt) {
+      if (fastc) {
+        // Per group of kFG rows:
+        // (a) thread 0 starts bulk copies of the rows' q slices (their 16-byte
+        //     aligned interior) and warp 1 loads the ragged ends; both arrive
+        //     on q_bar.  Meanwhile the epilogue warps read the rows' logits
+        //     from TMEM (lane = vocabulary entry) and form p, then, with q in
+        //     shared memory, the residual r = max(0, p - q) (p for a bonus row
+        //     or in the fallback attempt), stored per 32-entry segment with a
+        //     one-float pad (f_R[row][segment][33]);
+        // (b) every thread sums one segment of one row: four chains of
+        //     compensated sums (the terms are >= 0, so ordering the two addends
+        //     by size makes the error term exact);
+        // (c) one warp per row adds its segment masses into the slice mass.
+        //     Segment masses stay in shared memory for the in-slice search.
+        // q of slice entry e sits at f_Q[row * kQStride + e + qoff], so that
+        // the interior's first element lands on a 16-byte boundary.
+        const int qoff = v_lo & 3;
+        const int va = (v_lo + 3) & ~3, vb = v_hi & ~3;  // bulk-copied interior [va, vb)
+        const bool bulk = attempt == 0 && p.qbulk && va < vb;
+        const int e_tail = (va > vb ? va : vb) - v_lo;   // first entry after the interior
+        for (int g0 = 0; g0 < ns; g0 += kFG) {
+          const int ng = min(kFG, ns - g0);
+          if (warp == 0) {
+            if (lane == 0) {
+              int nq = 0;
+              for (int gi = 0; bulk && gi < ng; ++gi) nq += s_qidx[s_slist[g0 + gi]] >= 0;
+              if (nq > 0) {
+                fence_proxy_async_smem();  // earlier generic reads of f_Q come first
+                mbar_arrive_expect_tx(q_bar, static_cast<uint32_t>(nq * (vb - va) * 4));
+                for (int gi = 0; gi < ng; ++gi) {
+                  const int qi = s_qidx[s_slist[g0 + gi]];
+                  if (qi < 0) continue;
+                  bulk_load(f_Q + gi * kQStride + (va - v_lo + qoff),
+                            p.draft_probs + static_cast<size_t>(qi) * p.V + va,
+                            static_cast<uint32_t>((vb - va) * 4), q_bar);
+                }
+              } else {
+                mbar_arrive(q_bar);
+              }
+            }
+          } else if (warp == 1) {
+            if (attempt == 0) {
+              // With bulk copies: at most three entries before va and three
+              // after vb; else the whole slice.
+              const int gi = lane >> 2, k = lane & 3;
+              for (int row = bulk ? gi : 0; row < (bulk ? min(ng, gi + 1) : ng); ++row) {
+                const int qi = s_qidx[s_slist[g0 + row]];
+                if (qi < 0) continue;
+                const float *q = p.draft_probs + static_cast<size_t>(qi) * p.V + v_lo;
+                if (bulk) {
+                  if (k < va - v_lo && k < slen) f_Q[row * kQStride + k + qoff] = __ldg(q + k);
+                  if (e_tail + k < slen) f_Q[row * kQStride + e_tail + k + qoff] = __ldg(q + e_tail + k);
+                } else {
+                  for (int e = lane; e < slen; e += 32) f_Q[row * kQStride + e + qoff] = __ldg(q + e);
+                }
+              }
+            }
+            mbar_arrive(q_bar);  // each lane after its own stores
+          } else {
+            const int q4 = warp & 3;
+            const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
+            constexpr int kTiles = kFastSlice / kTileV;
+            // Lane gi prepares row gi's parameters (kFG <= 32); each row then
+            // broadcasts them.  The loop body has no divergent branch: tiles
+            // past the slice re-read its last tile and store zeros.
+            int n_l = -1, hq_l = 0;
+            float m_l = 0.f, is_l = 0.f;
+            if (lane < ng) {
+              const int b = s_slist[g0 + lane];
+              n_l = (attempt == 0 || s_usep[b]) ? s_rstar[b] : -1;
+              hq_l = attempt == 0 && s_qidx[b] >= 0;
+              if (n_l >= 0) {
+                m_l = g_m[n_l];
+                is_l = 1.f / g_s[n_l];
+              }
+            }
+#pragma unroll 1
+            for (int gi = 0; gi < ng; ++gi) {
+              const int n = __shfl_sync(0xffffffffu, n_l, gi);
+              const bool hasq = __shfl_sync(0xffffffffu, hq_l, gi) != 0;
+              const float M = __shfl_sync(0xffffffffu, m_l, gi), invS = __shfl_sync(0xffffffffu, is_l, gi);
+              uint32_t raw[kTiles];
+              if (n >= 0) {
 #pragma unroll
-      for (int i = 0; i < kZC; ++i) {
-        const int cc = i * 32 + lane;
-        zz[i] = (i * 32 < p.NC && cc < p.NC) ? __ldcg(&p.zpart[static_cast<size_t>(cc) * p.B + b])
-                                            : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-      ff2 tot{0.f, 0.f}, totp{0.f, 0.f};
+                for (int t = 0; t < kTiles; ++t)
+                  tmem_ld1(tmem + lane_base + static_cast<uint32_t>(min(t, ntiles - 1) * p.Rs + n), raw[t]);
+                tmem_wait_ld();
+              }
+              if (gi == 0 && !mbar_wait_unabortable(q_bar, q_phase)) {
+                // The copies read valid memory, so this wait does not give up
+                // on an earlier expired wait: no copy is left in flight at exit.
+                atomicOr(p.status, SPADE_DEV_TIMEOUT);
+                *s_abort = 1;
+              }
+              if (n < 0) continue;
+              const float *qs = f_Q + gi * kQStride + qoff;
+              float *rrow = f_R + gi * kFastSegs * kSegPad;
 #pragma unroll
-      for (int i = 0; i < kZC; ++i) {
-        tot = ff_add(tot, ff2{zz[i].x, zz[i].y});
-        totp = ff_add(totp, ff2{zz[i].z, zz[i].w});
-      }
-      tot = warp_sum_ff(tot);
-      totp = warp_sum_ff(totp);
-      const bool usep = !(tot.hi > 0.f && isfinite(tot.hi));
-      const ff2 Z = usep ? totp : tot;
-      const ff2 Tgt = ff_mul_f(Z, s_usmp[b]);
-      // First slice whose cumulative mass exceeds Tgt; else the last slice with mass.
-      ff2 base{0.f, 0.f}, base_owner{0.f, 0.f}, base_last{0.f, 0.f};
-      int owner = -1, last_pos = -1;
-#pragma unroll
-      for (int i = 0; i < kZC; ++i) {
-        if (i * 32 >= p.NC || owner >= 0) break;
-        const int cc = i * 32 + lane;
-        const ff2 z = usep ? ff2{zz[i].z, zz[i].w} : ff2{zz[i].x, zz[i].y};
-        const ff2 incl = warp_scan_ff(z, lane);
-        const ff2 reach = ff_add(base, incl);
-        const ff2 before = ff_add(base, ff_sub(incl, z));  // mass of the slices before cc
-        const unsigned hit = __ballot_sync(0xffffffffu, cc < p.NC && ff_gt(reach, Tgt));
-        const unsigned pos = __ballot_sync(0xffffffffu, cc < p.NC && z.hi > 0.f);
-        if (hit) {
-          const int l = __ffs(hit) - 1;
-          owner = i * 32 + l;
-          base_owner = ff_shfl(before, l);
+              for (int t = 0; t < kTiles; ++t) {
+                const int e = t * kTileV + q4 * 32 + lane;  // < kFastSlice: inside the row's buffers
+                const float pv = ex2((__uint_as_float(raw[t]) - M) * kLog2e) * invS;
+                const float rv = hasq ? fmaxf(0.f, pv - qs[e]) : pv;
+                rrow[(e >> 5) * kSegPad + (e & 31)] = e < slen ? rv : 0.f;
+              }
+            }
+          }
+          q_phase ^= 1u;
+          block_sync();
+          for (int task = tid; task < ng * nseg; task += kThreads) {
+            const int gi = task / nseg, sg = task - gi * nseg;
+            if (attempt == 1 && !s_usep[s_slist[g0 + gi]]) continue;
+            const float *rr = f_R + (gi * kFastSegs + sg) * kSegPad;
+            float hi[4] = {0.f, 0.f, 0.f, 0.f}, lo[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 8
+            for (int i = 0; i < 32; ++i) {
+              const float x = rr[i];
+              const int k = i & 3;
+              const float sm = hi[k] + x;
+              lo[k] += (fmaxf(hi[k], x) - sm) + fminf(hi[k], x);
+              hi[k] = sm;
+            }
+            const ff2 zs = ff_add(ff_add(ff_norm(hi[0], lo[0]), ff_norm(hi[1], lo[1])),
+                                  ff_add(ff_norm(hi[2], lo[2]), ff_norm(hi[3], lo[3])));
+            f_seg[(g0 + gi) * kFastSegs + sg] = make_float2(zs.hi, zs.lo);
+          }
+          block_sync();
         }
-        if (pos) {
-          const int l = 31 - __clz(pos);
-          last_pos = i * 32 + l;
-          base_last = ff_shfl(before, l);
+        for (int sl = warp; sl < ns; sl += kThreads / 32) {
+          const int b = s_slist[sl];
+          if (attempt == 1 && !s_usep[b]) continue;
+          const float2 t = lane < nseg ? f_seg[sl * kFastSegs + lane] : make_float2(0.f, 0.f);
+          const ff2 z = ff_shfl(warp_sum_ff(ff2{t.x, t.y}), 0);  // every copy holds lane 0's sum
+          if (lane < kReplicas)
+            __stcg(&p.zpart[(static_cast<size_t>(lane) * p.NC + c) * p.B + b], make_float2(z.hi, z.lo));
         }
-        base = ff_shfl(reach, 31);
+      } else {
+      if (warp >= 2) {
+        const int ew = warp - 2, q4 = warp & 3;
+        const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
+        // Stochastic sequences in groups of kG: the TMEM reads and q loads of a
+        // whole group are in flight together.
+        constexpr int kG = 4;
+        for (int b0 = 0; b0 < p.B;) {
+          int bl[kG], nb = 0;
+          while (b0 < p.B && nb < kG) {
+            if (s_stoch[b0] && (attempt == 0 || s_usep[b0])) bl[nb++] = b0;
+            ++b0;
+          }
+          if (nb == 0) break;
+          const float *qrow[kG];
+          int nrow[kG];
+          float M[kG], invS[kG];
+          ff2 z[kG], zp[kG];
+  #pragma unroll
+          for (int g = 0; g < kG; ++g) {
+            const int b = g < nb ? bl[g] : bl[0];
+            nrow[g] = s_rstar[b];
+            qrow[g] = (attempt == 0 && s_qidx[b] >= 0) ? p.draft_probs + static_cast<size_t>(s_qidx[b]) * p.V : nullptr;
+            M[g] = g_m[nrow[g]];
+            invS[g] = 1.f / g_s[nrow[g]];
+            z[g] = ff2{0.f, 0.f};
+            zp[g] = ff2{0.f, 0.f};
+          }
+          for (int j0 = 0; j0 < ntiles; j0 += 8) {
+            const int nj = min(8, ntiles - j0);
+            uint32_t raw[kG][8];
+            float qv[kG][8];
+  #pragma unroll
+            for (int g = 0; g < kG; ++g) {
+  #pragma unroll
+              for (int j = 0; j < 8; ++j)
+                if (g < nb && j < nj)
+                  tmem_ld1(tmem + lane_base + static_cast<uint32_t>((j0 + j) * p.Rs + nrow[g]), raw[g][j]);
+            }
+  #pragma unroll
+            for (int g = 0; g < kG; ++g) {
+  #pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
+                qv[g][j] = (g < nb && j < nj && qrow[g] && v < v_hi) ? qrow[g][v] : 0.f;
+              }
+            }
+            tmem_wait_ld();
+  #pragma unroll
+            for (int g = 0; g < kG; ++g) {
+  #pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
+                if (g < nb && j < nj && v < v_hi) {
+                  const float pv = ex2((__uint_as_float(raw[g][j]) - M[g]) * kLog2e) * invS[g];
+                  zp[g] = ff_add_f(zp[g], pv);
+                  z[g] = ff_add_f(z[g], qrow[g] ? fmaxf(0.f, pv - qv[g][j]) : pv);
+                }
+              }
+            }
+          }
+  #pragma unroll
+          for (int g = 0; g < kG; ++g) {
+            z[g] = warp_sum_ff(z[g]);
+            zp[g] = warp_sum_ff(zp[g]);
+            if (lane == 0 && g < nb) s_zw[bl[g] * kEpiWarps + ew] = make_float4(z[g].hi, z[g].lo, zp[g].hi, zp[g].lo);
+          }
+        }
       }
-      if (lane == 0) {
-        if (usep && c == 0) atomicOr(p.status, SPADE_DEV_FALLBACK);
-        s_owner[b] = owner >= 0 ? owner : last_pos;
-        const ff2 t = ff_sub(Tgt, owner >= 0 ? base_owner : base_last);  // past the total: clamp
-        s_T[b] = make_float2(t.hi, t.lo);
-        s_usep[b] = usep;
+      block_sync();
+      for (int b = tid; b < p.B; b += kThreads) {
+        if (!s_stoch[b] || (attempt == 1 && !s_usep[b])) continue;
+        ff2 zs{0.f, 0.f}, zps{0.f, 0.f};
+        for (int w = 0; w < kEpiWarps; ++w) {
+          const float4 t = s_zw[b * kEpiWarps + w];
+          zs = ff_add(zs, ff2{t.x, t.y});
+          zps = ff_add(zps, ff2{t.z, t.w});
+        }
+        const ff2 v = attempt == 0 ? zs : zps;
+        for (int r = 0; r < kReplicas; ++r)
+          __stcg(&p.zpart[(static_cast<size_t>(r) * p.NC + c) * p.B + b], make_float2(v.hi, v.lo));
       }
+      }  // register path
+      if (!grid_barrier(p.bar, p.NC)) {
+        atomicOr(p.status, SPADE_DEV_TIMEOUT);
+        *s_abort = 1;
+      }
+      // =================== phase D: owner slice of u*Z ======================
+      // One warp per sampled sequence.  Lane l holds the masses of the K
+      // consecutive slices [l*K, l*K + K) (all loads in flight at once); a warp
+      // scan of the lane sums gives the total and the lane whose cumulative
+      // mass passes u*Z, and that lane walks its K slices to the owner (else,
+      // rounding past the total, the last slice with mass).  Every CTA reaches
+      // the same owner from the same masses.
+      constexpr int kZC = kMaxNC / 32;
+      const int K = (p.NC + 31) / 32;
+      const float2 *zrep = p.zpart + static_cast<size_t>(c % kReplicas) * p.NC * p.B;
+#pragma unroll 1
+      for (int sl = warp; sl < ns; sl += kThreads / 32) {
+        const int b = s_slist[sl];
+        if (attempt == 1 && !s_usep[b]) continue;
+        float2 zz[kZC];
+#pragma unroll
+        for (int k = 0; k < kZC; ++k) {
+          const int cc = lane * K + k;
+          zz[k] = (k < K && cc < p.NC) ? __ldcg(&zrep[static_cast<size_t>(cc) * p.B + b])
+                                       : make_float2(0.f, 0.f);
+        }
+        float shi = 0.f, slo = 0.f;
+#pragma unroll
+        for (int k = 0; k < kZC; ++k) {
+          const float sm = shi + zz[k].x;
+          slo += ((fmaxf(shi, zz[k].x) - sm) + fminf(shi, zz[k].x)) + zz[k].y;
+          shi = sm;
+        }
+        const ff2 mine = ff_norm(shi, slo);
+        const ff2 incl = warp_scan_ff(mine, lane);
+        const ff2 tot = ff_shfl(incl, 31);
+        const bool bad = !(tot.hi > 0.f && isfinite(tot.hi));
+        if (bad) {
+          if (lane == 0) {
+            s_owner[b] = -1;
+            if (attempt == 0) {
+              s_usep[b] = 1;  // retry on p
+              s_seg[6] = 1;
+            } else if (c == 0) {
+              p.next_token[s_outb[b]] = -1;  // p has no mass either
+            }
+          }
+          continue;
+        }
+        const ff2 Tgt = ff_mul_f(tot, s_usmp[b]);
+        ff2 before = ff_shfl(incl, lane > 0 ? lane - 1 : 0);
+        if (lane == 0) before = ff2{0.f, 0.f};
+        const unsigned hit = __ballot_sync(0xffffffffu, mine.hi > 0.f && ff_gt(incl, Tgt));
+        const unsigned pos = __ballot_sync(0xffffffffu, mine.hi > 0.f);
+        const int l = hit ? __ffs(hit) - 1 : 31 - __clz(pos);  // pos != 0 as the total is > 0
+        if (l < 0 && lane == 0) s_owner[b] = -1;
+        if (lane == l) {
+          // d: target left before slice k; the owner is the first slice with
+          // mass above it (else the last slice with mass).
+          ff2 d = ff_sub(Tgt, before), d_last = d;
+          int own = -1, lastk = -1;
+#pragma unroll
+          for (int k = 0; k < kZC; ++k) {
+            const ff2 z{zz[k].x, zz[k].y};
+            if (own < 0 && z.hi > 0.f) {
+              if (hit && ff_gt(z, d)) {
+                own = k;
+              } else {
+                lastk = k;
+                d_last = d;
+                d = ff_sub(d, z);
+              }
+            }
+          }
+          if (attempt == 1 && c == 0) atomicOr(p.status, SPADE_DEV_FALLBACK);
+          s_owner[b] = l * K + (own >= 0 ? own : lastk);
+          const ff2 t = own >= 0 ? d : d_last;
+          s_T[b] = make_float2(t.hi, t.lo);
+        }
+      }
+      block_sync();
+      if (s_seg[6 + attempt] == 0) break;  // a flag per attempt: no reset races the reads
     }
     block_sync();
     if (warp >= 2) {
@@ -919,7 +1145,16 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         const bool usep = s_usep[b] != 0;
         const float *qrow = (s_qidx[b] >= 0 && !usep) ? p.draft_probs + static_cast<size_t>(s_qidx[b]) * p.V : nullptr;
         const float M = g_m[n], invS = 1.f / g_s[n];
-        // (1) mass of every 32-entry segment (tile j, lane quarter q4) of the slice.
+        // (1) mass of every 32-entry segment (tile j, lane quarter q4) of the slice:
+        //     from phase C's shared-memory sums, else recomputed.
+        if (fastc) {
+          if (ew == 0) {
+            const int sl = s_slpos[b];
+            for (int sg = lane; sg < ntiles * kEpiWarps; sg += 32) {
+              s_tw[sg] = sg < nseg ? f_seg[sl * kFastSegs + sg] : make_float2(0.f, 0.f);
+            }
+          }
+        } else
         for (int j0 = 0; j0 < ntiles; j0 += 8) {
           const int nj = min(8, ntiles - j0);
           uint32_t raw[8];
@@ -1065,9 +1300,9 @@ static WsRegion ws_region(size_t off, int B, int R, int NC) {
   w.ldraft = off;
   off += round_up(static_cast<size_t>(R) * 4, 256);
   w.gstat = off;
-  off += round_up(static_cast<size_t>(R) * 16, 256);
+  off += round_up(static_cast<size_t>(kReplicas) * R * 16, 256);
   w.zpart = off;
-  off += round_up(static_cast<size_t>(NC) * B * 16, 256);
+  off += round_up(static_cast<size_t>(kReplicas) * NC * B * 8, 256);
   w.end = off;
   return w;
 }
@@ -1092,7 +1327,7 @@ static WsLayout ws_layout(int B, int R, int H, int V, int sms) {
   WsLayout L{};
   const int NC = make_plan(R, V, sms).NC;
   L.two_pass = !resident_fits(R, V, NC);
-  L.r1 = ws_region(256, B, R, NC);
+  L.r1 = ws_region(kBarBytes, B, R, NC);
   if (!L.two_pass) {
     L.end = L.r1.end;
     return L;
@@ -1205,6 +1440,17 @@ static spade_status prepare(Params &p, int kind, const void *hidden, const void 
     p.KG = 1;
   }
   if (p.WS < 2) return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
+  // Bytes of the W ring that phases B-D use (the per-row / per-sequence
+  // arrays, then the staging buffers and segment masses of phase C).
+  constexpr size_t kPhaseBBytes = 4 * kMaxR * 4 + 8 * kMaxB * 4 + 16 * 4 + kMaxB * 8 +
+                                  kMaxB * kEpiWarps * 16 + kMaxTilesPerCta * kEpiWarps * 8;
+  constexpr size_t kFastBytes = kPhaseBBytes + 2 * kMaxB * 4 + kFG * (kFastSegs * kSegPad + kQStride) * 4 +
+                                kFastSeqs * kFastSegs * 8;
+  const size_t ring = static_cast<size_t>(p.WS) * p.KG * kWChunkBytes;
+  if (ring < kPhaseBBytes) return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
+  // After phase A the W and hidden rings (contiguous) are free.
+  p.fastc = static_cast<size_t>(smem_layout(p).off_bar) >= kFastBytes &&
+            (p.V + p.NC - 1) / p.NC <= kFastSlice;
   p.NS = (p.KC + p.KG - 1) / p.KG;
   if (smem_layout(p).total > kSmemMax) return fail(SPADE_ERR_SHAPE, "shared memory plan too large");
 
@@ -1253,7 +1499,7 @@ static void set_region(Params &p, uint8_t *ws, const WsRegion &r) {
   p.pstat = reinterpret_cast<float4 *>(ws + r.pstat);
   p.ldraft = reinterpret_cast<float *>(ws + r.ldraft);
   p.gstat = reinterpret_cast<float4 *>(ws + r.gstat);
-  p.zpart = reinterpret_cast<float4 *>(ws + r.zpart);
+  p.zpart = reinterpret_cast<float2 *>(ws + r.zpart);
 }
 
 }  // namespace accept
@@ -1308,6 +1554,7 @@ static spade_status verify_accept_impl(const void *hidden, const void *w_lm,
   Params p{};
   p.draft_tokens = draft_tokens;
   p.draft_probs = draft_probs;
+  p.qbulk = draft_probs != nullptr && aligned(draft_probs, 16) && V % 4 == 0;
   p.uniforms = uniforms;
   p.mode = mode;
   p.cu_q = cu_q;

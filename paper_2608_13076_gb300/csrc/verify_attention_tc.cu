@@ -178,8 +178,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                                const __grid_constant__ CUtensorMap tm_v1) {
   static_assert(NR % 16 == 0 && NR >= 16 && NR <= kRowBlock, "MMA N must be 16..64, step 16");
   extern __shared__ uint8_t smem_raw[];
-  uint8_t *smem = reinterpret_cast<uint8_t *>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // 1024-byte aligned base, derived by pointer arithmetic so that the compiler
+  // keeps the shared state space (plain ld/st.shared, not generic accesses).
+  uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   int64_t *s_pref = reinterpret_cast<int64_t *>(smem + Smem::PREF);
   int32_t *s_ctx = reinterpret_cast<int32_t *>(smem + Smem::CTX);
   int32_t *s_kd = reinterpret_cast<int32_t *>(smem + Smem::KD);

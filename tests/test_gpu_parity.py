@@ -73,6 +73,42 @@ def test_accept_small(dev, name):
     assert cmp["mismatch_unflagged"] == 0, cmp
 
 
+# Phase C has two forms: shared-memory segment sums (slices of at most 1024
+# vocabulary rows and at most 64 sampled rows) and the register form beyond.
+SAMPLER_PATHS = {
+    "smem_sums": W.WorkloadSpec("smem_sums", B=6, Hq=4, Hkv=4, D=64, H=256, V=3000,
+                                ctx=(1, 64), k=(1, 4), mode="stochastic", seed=21),
+    "register_sums_wide_slices": W.WorkloadSpec("register_sums_wide_slices", B=3, Hq=4, Hkv=4, D=64,
+                                                H=256, V=160000, ctx=(1, 64), k=(1, 3),
+                                                mode="stochastic", seed=22),
+    "register_sums_many_rows": W.WorkloadSpec("register_sums_many_rows", B=72, Hq=4, Hkv=4, D=64,
+                                              H=128, V=4000, ctx=(1, 64), k=(0, 1),
+                                              mode="stochastic", seed=23),
+}
+
+
+@pytest.mark.parametrize("name", sorted(SAMPLER_PATHS))
+@pytest.mark.parametrize("no_mass", [False, True])
+def test_accept_sampler_paths(dev, name, no_mass):
+    """Both phase-C forms, and the fallback to p when a residual has no mass:
+    q = 1 on every draft row of every other sequence makes max(0, p - q) zero."""
+    wl = W.make_workload(SAMPLER_PATHS[name], device=dev)
+    if no_mass and wl["draft_probs"] is not None:
+        cu = wl["cu_q"].cpu().numpy()
+        for b in range(0, wl["B"], 2):
+            d0, d1 = int(cu[b]) - b, int(cu[b + 1]) - b - 1
+            wl["draft_probs"][d0:d1] = 1.0
+    acc, tok, st = parity.gpu_accept(wl)
+    torch.cuda.synchronize()
+    ref = parity.oracle_accept(wl)
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0
+    assert bool(int(st.item()) & spade.DEV_FALLBACK) == bool(ref["fallback"].any())
+    if no_mass:
+        assert ref["fallback"].any()
+    cmp = parity.compare_accept(acc, tok, ref)
+    assert cmp["mismatch_unflagged"] == 0, cmp
+
+
 @pytest.mark.parametrize("name", sorted(SMALL))
 def test_kv_commit_small(dev, name):
     wl = W.make_workload(SMALL[name], device=dev, cache_pad=5)
