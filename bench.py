@@ -50,14 +50,17 @@ def _peaks():
 
 
 def _traffic(kernel, workload):
-    """ncu DRAM bytes per launch for this kernel and workload, if the kernel source is unchanged."""
+    """ncu DRAM bytes per launch for this kernel and workload, if its sources are unchanged."""
     import hashlib
     try:
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
             rec = json.load(f)[kernel][workload]
-        with open(os.path.join(ROOT, rec["source"]), "rb") as f:
-            if hashlib.sha256(f.read()).hexdigest()[:16] != rec["sha256_16"]:
-                return None
+        h = hashlib.sha256()
+        for src in rec["sources"]:  # every file the kernel is built from, in this order
+            with open(os.path.join(ROOT, src), "rb") as f:
+                h.update(f.read())
+        if h.hexdigest()[:16] != rec["sha256_16"]:
+            return None
         return rec["bytes"]
     except Exception:
         return None

@@ -18,7 +18,7 @@ namespace attn {
 constexpr int kChunk = 64;     // keys per schedule slice (and per warp-MMA stage)
 constexpr int kRowBlock = 64;  // query rows per work unit
 constexpr int kMaxB = 512;     // sequences per call (per-CTA schedule lives in smem)
-constexpr int kUnitCostTc = 5; // virtual slices per unit in the tensor-memory kernel's schedule
+constexpr int kUnitCostTc = 11; // virtual slices per unit in the tensor-memory kernel's schedule
 
 struct Params {
   const __nv_bfloat16 *q;

@@ -356,6 +356,10 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   tc_fence_after();
   const uint32_t tmem = *s_tmem;
   int rounds_issued = 0;  // MMA thread: accumulator rounds committed
+  // Every CTA reads the same hidden rows: CTA c walks the K stages starting at
+  // stage c mod NS, so at any moment about NC / NS CTAs (not all of them) load
+  // the same hidden lines from L2.  Each logit's sum over K changes order only.
+  const int k_rot = c % p.NS;
 
   // ======================= phase A: logits + slice statistics =============
   if (warp == 0) {
@@ -368,7 +372,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       int tdone = 0;
       for (int r = 0; r < p.nrounds && tdone < ntiles; ++r) {
         const int nt = min(p.round_tiles[r], ntiles - tdone);
-        for (int ks = 0; ks < p.NS; ++ks) {
+        for (int it = 0; it < p.NS; ++it) {
+          const int ks = it + k_rot < p.NS ? it + k_rot : it + k_rot - p.NS;
           const int c0 = ks * p.KG;
           const int nch = min(p.KG, p.KC - c0);
           const bool box3 = (nch == p.KG) && (c0 + p.KG <= p.KCF);
@@ -434,7 +439,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         const int nt = min(p.round_tiles[r], ntiles - tdone);
         if (r > 0) mbar_wait(acc_empty, (r - 1) & 1, s_abort);
         tc_fence_after();
-        for (int ks = 0; ks < p.NS; ++ks) {
+        for (int it = 0; it < p.NS; ++it) {
+          const int ks = it + k_rot < p.NS ? it + k_rot : it + k_rot - p.NS;
           const int nch = min(p.KG, p.KC - ks * p.KG);
           const int hs = hi % p.HS;
           mbar_wait(&h_full[hs], (hi / p.HS) & 1, s_abort);
@@ -455,7 +461,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
                 for (int k16 = 0; k16 < kKChunk / 16; ++k16) {
                   tc_mma_f16(d_tmem + noff, smem_desc_sw128(w_addr + jj * kWChunkBytes + 32 * k16),
                              smem_desc_sw128(h_addr + jj * hk + noff * 128 + 32 * k16),
-                             ci ? p.idesc1 : p.idesc, (ks | jj | k16) != 0);
+                             ci ? p.idesc1 : p.idesc, (it | jj | k16) != 0);
                 }
               }
             }
