@@ -54,7 +54,7 @@ constexpr float kRescaleLog2 = 8.f;
 // still-running PV could alias.
 constexpr int kBarKFull = 0, kBarVFull = 2, kBarKEmpty = 4, kBarVEmpty = 6, kBarSFull = 8,
               kBarSFree = 10, kBarPFull = 12, kBarPFree = 14, kBarODone = 16, kBarSeg = 17,
-              kBarOFinal = 18, kNumBars = 19;
+              kBarOFinal = 18, kBarQ = 19, kNumBars = 20;
 
 struct Smem {
   static constexpr int K = 0;                               // [stage][2 slabs][128 keys][128 B]
@@ -218,6 +218,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(&bars[kBarODone], 1);
     mbar_init(&bars[kBarSeg], kSoftWarps);
+    mbar_init(&bars[kBarQ], kSoftWarps);
     mbar_init(&bars[kBarOFinal], 1);
     fence_mbar_init();
   }
@@ -308,6 +309,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t ph = (j / kStages) & 1;
         if (!mbar_wait(&bars[kBarVFull + st], ph, s_abort)) expired = true;
         if (!mbar_wait(&bars[kBarPFull + st], ph, s_abort)) expired = true;
+        // The segment's first PV overwrites O^T: the previous epilogue has read it.
+        if (first && !mbar_wait(&bars[kBarSeg], seg & 1, s_abort)) expired = true;
         tc_fence_after();
         if (!*s_abort) {
           const uint32_t v_addr = smem_base + Smem::V + st * kTile;
@@ -326,7 +329,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t x = x_begin; x < x_end;) {
         const SegInfo si = next_seg(sc, x, x_end);
         if (si.n_here == 0) break;
-        if (!mbar_wait(&bars[kBarSeg], seg & 1, s_abort)) expired = true;  // Q staged, O^T free
+        // Q staged: the segment's S products may start while the previous
+        // segment's epilogue still reads O^T.
+        if (!mbar_wait(&bars[kBarQ], seg & 1, s_abort)) expired = true;
         tc_fence_after();
         const uint32_t q_addr = smem_base + Smem::Q + (seg & 1) * 2 * kQSlab;
         for (int c = 0; c < si.nchunk; ++c, ++it) {
@@ -406,7 +411,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_proxy_async_smem();
       named_bar(1, kSoftThreads);
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bars[kBarSeg]);
+      // Segment 0's Q is ready now; a later segment's was signalled before the
+      // previous epilogue.  O^T is free (the previous epilogue is done).
+      if (lane == 0) {
+        if (seg == 0) mbar_arrive(&bars[kBarQ]);
+        mbar_arrive(&bars[kBarSeg]);
+      }
 
       // Running row maxima live in s_rmax (one writer per row); the row sums of
       // this key lane in l.
@@ -449,7 +459,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             exceed |= x_[r] > kRescaleLog2;
           }
         }
-        if (bar_any(2, kSoftThreads, exceed)) {
+        // The two halves own disjoint rows: each votes and rescales on its own
+        // barriers (ids 2-3 and 4-5), so neither waits for the other.
+        if (bar_any(2 + half, kSoftThreads / 2, exceed)) {
           // Some score is more than 2^8 above its row's running maximum (always
           // so in a unit's first chunk): take this chunk's exact row maxima.
           // The S^T buffer is still intact (it is reused only after this
@@ -464,15 +476,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float wm = warp_reduce_scatter<NP, true>(x_, lane);
             if (lane < NH) s_wred[q4 * kRowBlock + c0 + lane] = wm;
           }
-          named_bar(1, kSoftThreads);
-          if (stid < NR) {
-            const float mo = s_rmax[stid];
-            const float mn = fmaxf(fmaxf(mo, fmaxf(s_wred[stid], s_wred[kRowBlock + stid])),
-                                   fmaxf(s_wred[2 * kRowBlock + stid], s_wred[3 * kRowBlock + stid]));
-            s_alpha[stid] = mn > mo ? ex2(mo - mn) : 1.f;  // mo = -inf gives 0: nothing to keep
-            s_rmax[stid] = mn;
+          named_bar(4 + half, kSoftThreads / 2);
+          const int hs = stid - half * (kSoftThreads / 2);  // thread of this half
+          if (hs < NH) {
+            const int row = c0 + hs;
+            const float mo = s_rmax[row];
+            const float mn = fmaxf(fmaxf(mo, fmaxf(s_wred[row], s_wred[kRowBlock + row])),
+                                   fmaxf(s_wred[2 * kRowBlock + row], s_wred[3 * kRowBlock + row]));
+            s_alpha[row] = mn > mo ? ex2(mo - mn) : 1.f;  // mo = -inf gives 0: nothing to keep
+            s_rmax[row] = mn;
           }
-          named_bar(1, kSoftThreads);
+          named_bar(4 + half, kSoftThreads / 2);
 #pragma unroll
           for (int r = 0; r < NH; ++r) l[r] *= s_alpha[c0 + r];
           if (c > 0) {
@@ -539,6 +553,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars[kBarPFull + st]);
+      }
+      // The next segment's Q (prefetched at this segment's start) lets the MMA
+      // warp start its S products during this epilogue.
+      if (si_next.n_here > 0) {
+        cp_async_wait<0>();
+        fence_proxy_async_smem();
+        named_bar(1, kSoftThreads);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars[kBarQ]);
       }
 
       // ---- epilogue: row sums, O^T from tensor memory, output or partial ----
