@@ -262,6 +262,15 @@ __device__ __forceinline__ ff2 warp_sum_ff(ff2 v) {
   return ff_shfl(v, 0);  // one value for every lane
 }
 // Inclusive prefix sum over the warp's lanes.
+// Inclusive float-float scan over the 16 lanes of each half warp (j = lane & 15).
+__device__ __forceinline__ ff2 half_scan_ff(ff2 v, int j) {
+#pragma unroll
+  for (int o = 1; o < 16; o <<= 1) {
+    const ff2 t{__shfl_up_sync(0xffffffffu, v.hi, o, 16), __shfl_up_sync(0xffffffffu, v.lo, o, 16)};
+    if (j >= o) v = ff_add(t, v);
+  }
+  return v;
+}
 __device__ __forceinline__ ff2 warp_scan_ff(ff2 v, int lane) {
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -1064,25 +1073,29 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         *s_abort = 1;
       }
       // =================== phase D: owner slice of u*Z ======================
-      // One warp per sampled sequence.  Lane l holds the masses of the K
-      // consecutive slices [l*K, l*K + K) (all loads in flight at once); a warp
-      // scan of the lane sums gives the total and the lane whose cumulative
-      // mass passes u*Z, and that lane walks its K slices to the owner (else,
-      // rounding past the total, the last slice with mass).  Every CTA reaches
-      // the same owner from the same masses.
-      constexpr int kZC = kMaxNC / 32;
-      const int K = (p.NC + 31) / 32;
+      // A half warp per sampled sequence (so one pass covers 12 sequences).
+      // Lane j of the half holds the masses of the K = ceil(NC/16) slices
+      // [j*K, j*K + K) (all loads in flight at once).  A scan of the lane sums
+      // gives the total and the lane whose cumulative mass passes u*Z; that
+      // lane's K masses are then spread over the half and scanned again, which
+      // gives the owner slice (else, rounding past the total, the last slice
+      // with mass).  Every CTA reaches the same owner from the same masses.
+      constexpr int kZC = kMaxNC / 16;
+      const int K = (p.NC + 15) / 16;
+      const int half = lane >> 4, j = lane & 15;
+      const unsigned hmask = 0xffffu << (16 * half);
       const float2 *zrep = p.zpart + static_cast<size_t>(c % kReplicas) * p.NC * p.B;
 #pragma unroll 1
-      for (int sl = warp; sl < ns; sl += kThreads / 32) {
-        const int b = s_slist[sl];
-        if (attempt == 1 && !s_usep[b]) continue;
+      for (int sl0 = 2 * warp; sl0 < ns; sl0 += 2 * (kThreads / 32)) {
+        const int sl = sl0 + half;
+        const int b = sl < ns ? s_slist[sl] : -1;
+        const bool act = b >= 0 && (attempt == 0 || s_usep[b]);
         float2 zz[kZC];
 #pragma unroll
         for (int k = 0; k < kZC; ++k) {
-          const int cc = lane * K + k;
-          zz[k] = (k < K && cc < p.NC) ? __ldcg(&zrep[static_cast<size_t>(cc) * p.B + b])
-                                       : make_float2(0.f, 0.f);
+          const int cc = j * K + k;
+          zz[k] = (act && k < K && cc < p.NC) ? __ldcg(&zrep[static_cast<size_t>(cc) * p.B + b])
+                                              : make_float2(0.f, 0.f);
         }
         float shi = 0.f, slo = 0.f;
 #pragma unroll
@@ -1092,49 +1105,46 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           shi = sm;
         }
         const ff2 mine = ff_norm(shi, slo);
-        const ff2 incl = warp_scan_ff(mine, lane);
-        const ff2 tot = ff_shfl(incl, 31);
-        const bool bad = !(tot.hi > 0.f && isfinite(tot.hi));
-        if (bad) {
-          if (lane == 0) {
-            s_owner[b] = -1;
-            if (attempt == 0) {
-              s_usep[b] = 1;  // retry on p
-              s_seg[6] = 1;
-            } else if (c == 0) {
-              p.next_token[s_outb[b]] = -1;  // p has no mass either
-            }
+        const ff2 incl = half_scan_ff(mine, j);
+        const ff2 tot{__shfl_sync(0xffffffffu, incl.hi, 15, 16), __shfl_sync(0xffffffffu, incl.lo, 15, 16)};
+        const bool ok = act && tot.hi > 0.f && isfinite(tot.hi);
+        if (act && !ok && j == 0) {
+          s_owner[b] = -1;
+          if (attempt == 0) {
+            s_usep[b] = 1;  // retry on p
+            s_seg[6] = 1;
+          } else if (c == 0) {
+            p.next_token[s_outb[b]] = -1;  // p has no mass either
           }
-          continue;
         }
-        const ff2 Tgt = ff_mul_f(tot, s_usmp[b]);
-        ff2 before = ff_shfl(incl, lane > 0 ? lane - 1 : 0);
-        if (lane == 0) before = ff2{0.f, 0.f};
-        const unsigned hit = __ballot_sync(0xffffffffu, mine.hi > 0.f && ff_gt(incl, Tgt));
-        const unsigned pos = __ballot_sync(0xffffffffu, mine.hi > 0.f);
-        const int l = hit ? __ffs(hit) - 1 : 31 - __clz(pos);  // pos != 0 as the total is > 0
-        if (l < 0 && lane == 0) s_owner[b] = -1;
-        if (lane == l) {
-          // d: target left before slice k; the owner is the first slice with
-          // mass above it (else the last slice with mass).
-          ff2 d = ff_sub(Tgt, before), d_last = d;
-          int own = -1, lastk = -1;
+        const ff2 Tgt = ff_mul_f(tot, ok ? s_usmp[b] : 0.f);
+        ff2 before{__shfl_up_sync(0xffffffffu, incl.hi, 1, 16), __shfl_up_sync(0xffffffffu, incl.lo, 1, 16)};
+        if (j == 0) before = ff2{0.f, 0.f};
+        const unsigned hit = __ballot_sync(0xffffffffu, ok && mine.hi > 0.f && ff_gt(incl, Tgt)) & hmask;
+        const unsigned pos = __ballot_sync(0xffffffffu, ok && mine.hi > 0.f) & hmask;
+        const int l = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : -1);  // absolute lane
+        // Second level: lane l's K slice masses, one per lane of the half.
+        const int lsrc = l >= 0 ? (l & 15) : 0;
+        float2 zk = make_float2(0.f, 0.f);
 #pragma unroll
-          for (int k = 0; k < kZC; ++k) {
-            const ff2 z{zz[k].x, zz[k].y};
-            if (own < 0 && z.hi > 0.f) {
-              if (hit && ff_gt(z, d)) {
-                own = k;
-              } else {
-                lastk = k;
-                d_last = d;
-                d = ff_sub(d, z);
-              }
-            }
-          }
+        for (int k = 0; k < kZC; ++k) {
+          const float vx = __shfl_sync(0xffffffffu, zz[k].x, lsrc, 16);
+          const float vy = __shfl_sync(0xffffffffu, zz[k].y, lsrc, 16);
+          if (j == k) zk = make_float2(vx, vy);
+        }
+        const ff2 base{__shfl_sync(0xffffffffu, before.hi, lsrc, 16), __shfl_sync(0xffffffffu, before.lo, lsrc, 16)};
+        const ff2 z{zk.x, zk.y};
+        const ff2 inc2 = half_scan_ff(z, j);
+        const ff2 reach = ff_add(base, inc2);
+        const bool live = ok && l >= 0 && j < K && z.hi > 0.f;
+        const unsigned hit2 = __ballot_sync(0xffffffffu, live && ff_gt(reach, Tgt)) & hmask;
+        const unsigned pos2 = __ballot_sync(0xffffffffu, live) & hmask;
+        const int l2 = hit2 ? __ffs(hit2) - 1 : (pos2 ? 31 - __clz(pos2) : -1);
+        if (ok && l2 < 0 && j == 0) s_owner[b] = -1;  // no slice with mass (not reached: tot > 0)
+        if (lane == l2) {
           if (attempt == 1 && c == 0) atomicOr(p.status, SPADE_DEV_FALLBACK);
-          s_owner[b] = l * K + (own >= 0 ? own : lastk);
-          const ff2 t = own >= 0 ? d : d_last;
+          s_owner[b] = (l & 15) * K + j;
+          const ff2 t = ff_sub(Tgt, ff_add(base, ff_sub(inc2, z)));  // target left inside the slice
           s_T[b] = make_float2(t.hi, t.lo);
         }
       }
