@@ -947,11 +947,16 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               if (n < 0) continue;
               const float *qs = f_Q + gi * kQStride + qoff;
               float *rrow = f_R + gi * kFastSegs * kSegPad;
+              // All q loads before the first store: the compiler cannot tell
+              // f_Q and f_R apart, and would otherwise wait on each load in turn.
+              float qv[kTiles];
+#pragma unroll
+              for (int t = 0; t < kTiles; ++t) qv[t] = hasq ? qs[t * kTileV + q4 * 32 + lane] : 0.f;
 #pragma unroll
               for (int t = 0; t < kTiles; ++t) {
                 const int e = t * kTileV + q4 * 32 + lane;  // < kFastSlice: inside the row's buffers
                 const float pv = ex2((__uint_as_float(raw[t]) - M) * kLog2e) * invS;
-                const float rv = hasq ? fmaxf(0.f, pv - qs[e]) : pv;
+                const float rv = hasq ? fmaxf(0.f, pv - qv[t]) : pv;
                 rrow[(e >> 5) * kSegPad + (e & 31)] = e < slen ? rv : 0.f;
               }
             }
