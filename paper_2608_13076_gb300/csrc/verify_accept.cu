@@ -658,7 +658,28 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       m = __shfl_sync(0xffffffffu, m, 0);
       sm = __shfl_sync(0xffffffffu, sm, 0);
       idx = __shfl_sync(0xffffffffu, idx, 0);
-      if (lane < kReplicas) __stcg(&p.gstat[static_cast<size_t>(lane) * p.R + n], make_float4(m, sm, __int_as_float(idx), 0.f));
+      // (2) The accept test of this row, from the merged statistics (every CTA
+      //     then reads it with them instead of re-loading l[d] after the next
+      //     barrier).  Rows past a sequence's drafts, and invalid sequences,
+      //     give 0; the leading-accept count is formed after the barrier.
+      int ok = 0;
+      if (p.kind != kPresampled) {
+        const int b = s_seq[n];
+        if (b >= 0 && s_pos[n] < s_nd[b]) {
+          const int d = s_draft[n];
+          if (d < 0 || d >= p.V) {
+            if (lane == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
+          } else if (!(s_md[b] == 1 && p.draft_probs != nullptr)) {
+            ok = (d == idx);
+          } else {
+            const float pd = expf(__ldcg(&p.ldraft[n]) - m) / sm;
+            const float qd = s_qd[n];
+            ok = (qd > 0.f) ? (s_u[n] < pd / qd) : (pd > 0.f);
+          }
+        }
+      }
+      if (lane < kReplicas)
+        __stcg(&p.gstat[static_cast<size_t>(lane) * p.R + n], make_float4(m, sm, __int_as_float(idx), __int_as_float(ok)));
     }
   }
   if (!grid_barrier(p.bar, p.NC)) {
@@ -688,12 +709,13 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   float *f_Q = f_R + kFG * kFastSegs * kSegPad;             // [kFG][kQStride] q of staged rows
   float2 *f_seg = reinterpret_cast<float2 *>(f_Q + kFG * kQStride);  // [kFastSeqs][kFastSegs]
   uint32_t q_phase = 0;
-  // (2) Every CTA reads the merged statistics of all rows.
+  // (3) Every CTA reads the merged statistics and accept bits of all rows.
   for (int n = tid; n < p.R; n += kThreads) {
     const float4 g = __ldcg(&p.gstat[static_cast<size_t>(c % kReplicas) * p.R + n]);
     g_m[n] = g.x;
     g_s[n] = g.y;
     g_arg[n] = __float_as_int(g.z);
+    s_ok[n] = __float_as_int(g.w);
   }
   for (int b = tid; p.kind != kPresampled && b < p.B; b += kThreads) {
     const int md = s_md[b];
@@ -702,26 +724,6 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   }
   block_sync();
   if (p.kind != kPresampled) {
-  // (3) Accept test of every draft row, all rows at once (the tests are
-  //     independent; only the count of leading accepts depends on their order).
-  for (int n = tid; n < p.R; n += kThreads) {
-    const int b = s_seq[n];
-    int ok = 0;
-    if (b >= 0 && s_pos[n] < s_nd[b]) {
-      const int d = s_draft[n];
-      if (d < 0 || d >= p.V) {
-        if (c == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
-      } else if (!s_stoch[b]) {
-        ok = (d == g_arg[n]);
-      } else {
-        const float pd = expf(__ldcg(&p.ldraft[n]) - g_m[n]) / g_s[n];
-        const float qd = s_qd[n];
-        ok = (qd > 0.f) ? (s_u[n] < pd / qd) : (pd > 0.f);
-      }
-    }
-    s_ok[n] = ok;
-  }
-  block_sync();
   // (4) Accepted length = leading accepts; the row that emits the next token.
   for (int b = tid; b < p.B; b += kThreads) {
     const int r0 = s_cuq[b], k = s_nd[b];
