@@ -244,13 +244,20 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ============================ producer: TMA ============================
-    if (lane == 0) {
-      tma_prefetch_desc(&tm_k2);
-      tma_prefetch_desc(&tm_v2);
-      tma_prefetch_desc(&tm_k1);
-      tma_prefetch_desc(&tm_v1);
+    // Lane 0 loads the K tiles, lane 1 the V tiles: a K stage is refilled as
+    // soon as its S product is done, without waiting behind the V stage that
+    // only frees after the softmax and the PV product.
+    if (lane < 2) {
+      const bool is_v = lane == 1;
+      const CUtensorMap *tm2 = is_v ? &tm_v2 : &tm_k2;
+      const CUtensorMap *tm1 = is_v ? &tm_v1 : &tm_k1;
+      tma_prefetch_desc(tm2);
+      tma_prefetch_desc(tm1);
+      const int bar_empty = is_v ? kBarVEmpty : kBarKEmpty;
+      const int bar_full = is_v ? kBarVFull : kBarKFull;
+      uint8_t *const ring = smem + (is_v ? Smem::V : Smem::K);
       const uint64_t pol = l2_policy_evict_first();
-      uint32_t it = 0, k_issued = 0, v_issued = 0;
+      uint32_t it = 0, issued = 0;
       bool expired = false;
       for (int64_t x = x_begin; x < x_end;) {
         const SegInfo si = next_seg(sc, x, x_end);
@@ -261,38 +268,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t ph = (it / kStages) & 1;
           const int nsl = min(2, si.n_here - 2 * c);
           const int key_row = row0 + (si.g.ci + 2 * c) * kChunk;
-          uint8_t *kt = smem + Smem::K + st * kTile;
-          uint8_t *vt = smem + Smem::V + st * kTile;
-          if (!mbar_wait(&bars[kBarKEmpty + st], ph ^ 1, s_abort)) expired = true;
+          uint8_t *tile = ring + st * kTile;
+          if (!mbar_wait(&bars[bar_empty + st], ph ^ 1, s_abort)) expired = true;
           if (*s_abort) continue;
-          mbar_arrive_expect_tx(&bars[kBarKFull + st], nsl * kSlab);
+          mbar_arrive_expect_tx(&bars[bar_full + st], nsl * kSlab);
           if (nsl == 2) {
-            tma_load_3d(kt, &tm_k2, 0, key_row, 0, &bars[kBarKFull + st], pol);
+            tma_load_3d(tile, tm2, 0, key_row, 0, &bars[bar_full + st], pol);
           } else {
-            tma_load_3d(kt, &tm_k1, 0, key_row, 0, &bars[kBarKFull + st], pol);
-            tma_load_3d(kt + kSlab, &tm_k1, 0, key_row, 1, &bars[kBarKFull + st], pol);
+            tma_load_3d(tile, tm1, 0, key_row, 0, &bars[bar_full + st], pol);
+            tma_load_3d(tile + kSlab, tm1, 0, key_row, 1, &bars[bar_full + st], pol);
           }
-          k_issued = it + 1;
-          if (!mbar_wait(&bars[kBarVEmpty + st], ph ^ 1, s_abort)) expired = true;
-          if (*s_abort) continue;
-          mbar_arrive_expect_tx(&bars[kBarVFull + st], nsl * kSlab);
-          if (nsl == 2) {
-            tma_load_3d(vt, &tm_v2, 0, key_row, 0, &bars[kBarVFull + st], pol);
-          } else {
-            tma_load_3d(vt, &tm_v1, 0, key_row, 0, &bars[kBarVFull + st], pol);
-            tma_load_3d(vt + kSlab, &tm_v1, 0, key_row, 1, &bars[kBarVFull + st], pol);
-          }
-          v_issued = it + 1;
+          issued = it + 1;
         }
         x = si.seg_end;
       }
       if (expired || *s_abort) {
         atomicOr(p.status, SPADE_DEV_TIMEOUT);
         // Drain: every copy issued must land before the CTA's smem goes away.
-        for (uint32_t j = (k_issued > kStages ? k_issued - kStages : 0); j < k_issued; ++j)
-          mbar_wait_unabortable(&bars[kBarKFull + j % kStages], (j / kStages) & 1);
-        for (uint32_t j = (v_issued > kStages ? v_issued - kStages : 0); j < v_issued; ++j)
-          mbar_wait_unabortable(&bars[kBarVFull + j % kStages], (j / kStages) & 1);
+        for (uint32_t j = (issued > kStages ? issued - kStages : 0); j < issued; ++j)
+          mbar_wait_unabortable(&bars[bar_full + j % kStages], (j / kStages) & 1);
       }
     }
   } else if (warp == 1) {
