@@ -283,7 +283,8 @@ __device__ __forceinline__ ff2 warp_scan_ff(ff2 v, int lane) {
 __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tm_w3,
     const __grid_constant__ CUtensorMap tm_w2, const __grid_constant__ CUtensorMap tm_w2s,
-    const __grid_constant__ CUtensorMap tm_h3, const __grid_constant__ CUtensorMap tm_h2) {
+    const __grid_constant__ CUtensorMap tm_w3s, const __grid_constant__ CUtensorMap tm_h3,
+    const __grid_constant__ CUtensorMap tm_h2) {
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte aligned base, derived by pointer arithmetic so that the compiler
   // keeps the shared state space (plain ld/st.shared, not generic accesses).
@@ -374,6 +375,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   if (warp == 0) {
     if (lane == 0 && ntiles > 0) {
       tma_prefetch_desc(&tm_w3);
+      tma_prefetch_desc(&tm_w3s);
       tma_prefetch_desc(&tm_h3);
       const uint64_t pol_w = l2_policy_evict_first();
       const uint64_t pol_h = l2_policy_evict_last();
@@ -412,11 +414,17 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               uint8_t *dst = w_ring + s * L.w_slot;
               const int row0 = v_lo + (tdone + j) * kTileV;
               if (short_last && tdone + j == ntiles - 1) {
-                // Partial last tile: BRS-row boxes, one per k-chunk; the slot's
-                // remaining rows feed accumulator lanes that are never read.
+                // Partial last tile: BRS-row boxes (BRS a multiple of 8), the k-chunks
+                // packed at BRS * 128-byte strides: one 3-D box per stage when it
+                // holds KG full chunks (small 2-D boxes stream far slower).  The
+                // slot's remaining rows feed accumulator lanes that are never read.
                 mbar_arrive_expect_tx(&w_full[s], nch * p.BRS * 128);
-                for (int jj = 0; jj < nch; ++jj)
-                  tma_load_2d(dst + jj * kWChunkBytes, &tm_w2s, (c0 + jj) * kKChunk, row0, &w_full[s], pol_w);
+                if (box3) {
+                  tma_load_3d(dst, &tm_w3s, 0, row0, c0, &w_full[s], pol_w);
+                } else {
+                  for (int jj = 0; jj < nch; ++jj)
+                    tma_load_2d(dst + jj * p.BRS * 128, &tm_w2s, (c0 + jj) * kKChunk, row0, &w_full[s], pol_w);
+                }
               } else if (box3) {
                 mbar_arrive_expect_tx(&w_full[s], nch * kWChunkBytes);
                 tma_load_3d(dst, &tm_w3, 0, row0, c0, &w_full[s], pol_w);
@@ -460,6 +468,10 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             mbar_wait(&w_full[ws], (wi / p.WS) & 1, s_abort);
             tc_fence_after();
             const uint32_t w_addr = smem_u32(w_ring + ws * L.w_slot);
+            // k-chunk stride in the slot: a full tile's chunks are 16 KB apart,
+            // the short last tile's are packed (BRS rows each).
+            const uint32_t w_chunk = (short_last && tdone + j == ntiles - 1) ? static_cast<uint32_t>(p.BRS * 128)
+                                                                            : static_cast<uint32_t>(kWChunkBytes);
             const uint32_t d_tmem = tmem + static_cast<uint32_t>(used + j * p.Ncols);
             const int hk = p.h_boxes * p.h_box_rows * 128;
             for (int jj = 0; jj < nch; ++jj) {
@@ -468,7 +480,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
                 const uint32_t noff = ci ? static_cast<uint32_t>(p.n0w) : 0u;
 #pragma unroll
                 for (int k16 = 0; k16 < kKChunk / 16; ++k16) {
-                  tc_mma_f16(d_tmem + noff, smem_desc_sw128(w_addr + jj * kWChunkBytes + 32 * k16),
+                  tc_mma_f16(d_tmem + noff, smem_desc_sw128(w_addr + jj * w_chunk + 32 * k16),
                              smem_desc_sw128(h_addr + jj * hk + noff * 128 + 32 * k16),
                              ci ? p.idesc1 : p.idesc, (it | jj | k16) != 0);
                 }
@@ -1403,7 +1415,7 @@ static bool encode_kslab_view(CUtensorMap *map, const void *base, int rows, int 
 }
 
 struct Maps {
-  CUtensorMap w3, w2, w2s, h3, h2;
+  CUtensorMap w3, w2, w2s, w3s, h3, h2;
 };
 
 // Fills the plan-dependent fields of `p` for a launch of kind `kind` over the
@@ -1486,10 +1498,12 @@ static spade_status prepare(Params &p, int kind, const void *hidden, const void 
     return SPADE_ERR_CUDA;
   if (p.KCF >= 1) {
     if (!encode_kslab_view(&m.w3, w_lm, p.V, p.H, kTileV, p.KG) ||
+        !encode_kslab_view(&m.w3s, w_lm, p.V, p.H, p.BRS, p.KG) ||
         !encode_kslab_view(&m.h3, hidden, R, p.H, pl.Ncols < 256 ? pl.Ncols : 256, p.KG))
       return SPADE_ERR_CUDA;
   } else {
     m.w3 = m.w2;  // never used: every stage takes the 2-D path
+    m.w3s = m.w2s;
     m.h3 = m.h2;
   }
   return SPADE_OK;
@@ -1513,7 +1527,7 @@ static spade_status launch(const Params &p, const Maps &m, cudaStream_t stream) 
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, verify_accept_kernel, p, m.w3, m.w2, m.w2s, m.h3, m.h2);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, verify_accept_kernel, p, m.w3, m.w2, m.w2s, m.w3s, m.h3, m.h2);
   if (e != cudaSuccess) return cuda_fail(e, "verify_accept cooperative launch");
   return SPADE_OK;
 }
