@@ -370,6 +370,12 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   // stage c mod NS, so at any moment about NC / NS CTAs (not all of them) load
   // the same hidden lines from L2.  Each logit's sum over K changes order only.
   const int k_rot = c % p.NS;
+  // A round that holds only the short last tile streams one k-chunk per stage
+  // with its W rows and hidden rows together in one slot of either ring, so all
+  // 4 + 3 slots are in flight (a two-ring stage keeps at most HS = 3 in flight,
+  // and its W slots would be 60 % empty).  Needs both boxes to fit an H slot.
+  const bool comb_ok = p.kind != kStatsOnly && short_last && p.nchunks == 1 && p.h_boxes == 1 &&
+                       (p.BRS + p.h_box_rows) * 128 <= L.h_slot;
 
   // ======================= phase A: logits + slice statistics =============
   if (warp == 0) {
@@ -383,6 +389,28 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       int tdone = 0;
       for (int r = 0; r < p.nrounds && tdone < ntiles; ++r) {
         const int nt = min(p.round_tiles[r], ntiles - tdone);
+        if (comb_ok && nt == 1 && tdone == ntiles - 1) {
+          const int row0 = v_lo + tdone * kTileV;
+          const int kr = c % p.KC;
+          for (int it = 0; it < p.KC; ++it) {
+            const int kc = it + kr < p.KC ? it + kr : it + kr - p.KC;
+            const bool use_w = it % 7 < 4;  // four W slots, then three H slots
+            const int s = use_w ? wi % p.WS : hi % p.HS;
+            uint64_t *full = use_w ? &w_full[s] : &h_full[s];
+            mbar_wait(use_w ? &w_empty[s] : &h_empty[s],
+                      ((use_w ? wi / p.WS : hi / p.HS) & 1) ^ 1, s_abort);
+            if (!*s_abort) {
+              uint8_t *dst = use_w ? w_ring + s * L.w_slot : h_ring + s * L.h_slot;
+              mbar_arrive_expect_tx(full, (p.BRS + p.h_box_rows) * 128);
+              tma_load_2d(dst, &tm_w2s, kc * kKChunk, row0, full, pol_w);
+              tma_load_2d(dst + p.BRS * 128, &tm_h2, kc * kKChunk, 0, full, pol_h);
+              if (use_w) w_issued = wi + 1; else h_issued = hi + 1;
+            }
+            if (use_w) ++wi; else ++hi;
+          }
+          tdone += nt;
+          continue;
+        }
         for (int it = 0; it < p.NS; ++it) {
           const int ks = it + k_rot < p.NS ? it + k_rot : it + k_rot - p.NS;
           const int c0 = ks * p.KG;
@@ -456,6 +484,27 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         const int nt = min(p.round_tiles[r], ntiles - tdone);
         if (r > 0) mbar_wait(acc_empty, (r - 1) & 1, s_abort);
         tc_fence_after();
+        if (comb_ok && nt == 1 && tdone == ntiles - 1) {
+          const uint32_t d_tmem = tmem + static_cast<uint32_t>(used);
+          for (int it = 0; it < p.KC; ++it) {
+            const bool use_w = it % 7 < 4;
+            const int s = use_w ? wi % p.WS : hi % p.HS;
+            mbar_wait(use_w ? &w_full[s] : &h_full[s], (use_w ? wi / p.WS : hi / p.HS) & 1, s_abort);
+            tc_fence_after();
+            const uint32_t base = smem_u32(use_w ? w_ring + s * L.w_slot : h_ring + s * L.h_slot);
+#pragma unroll
+            for (int k16 = 0; k16 < kKChunk / 16; ++k16)
+              tc_mma_f16(d_tmem, smem_desc_sw128(base + 32 * k16), smem_desc_sw128(base + p.BRS * 128 + 32 * k16),
+                         p.idesc, (it | k16) != 0);
+            tc_commit(use_w ? &w_empty[s] : &h_empty[s]);
+            if (use_w) ++wi; else ++hi;
+          }
+          tc_commit(acc_full);
+          ++rounds_issued;
+          used += nt * p.Rs;
+          tdone += nt;
+          continue;
+        }
         for (int it = 0; it < p.NS; ++it) {
           const int ks = it + k_rot < p.NS ? it + k_rot : it + k_rot - p.NS;
           const int nch = min(p.KG, p.KC - ks * p.KG);
