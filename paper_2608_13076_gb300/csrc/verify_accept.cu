@@ -53,6 +53,7 @@ constexpr int kMaxRounds = 32;
 constexpr int kResident = 0, kStatsOnly = 1, kPresampled = 2;
 constexpr int kMaxTilesPerCta = 32;
 constexpr int kMaxNC = 256;  // CTAs (vocabulary slices) per launch
+
 // Residual masses through shared memory (phase C): groups of kFG sampled rows
 // are staged as p and q slices, then every thread sums 32-entry segments
 // serially; slices of at most kFastSlice vocab rows, at most kFastSeqs sampled
@@ -96,6 +97,7 @@ struct Params {
   int32_t *ctx_lens;
   int Hkv, Dk, cap;
   int kind;
+  int pair;          // statistics pass on CTA pairs (cta_group::2), see phase A
   int nchunks;       // MMA N-chunks per tile (2 when Ncols > 256)
   int n0w;           // width of the first N-chunk
   uint32_t idesc1;   // instruction descriptor of the second N-chunk
@@ -126,7 +128,9 @@ __host__ __device__ inline Smem smem_layout(const Params &p) {
   s.h_slot = p.KG * p.h_boxes * p.h_box_rows * 128;
   s.off_h = p.WS * s.w_slot;
   s.off_bar = s.off_h + p.HS * s.h_slot;
-  s.off_misc = s.off_bar + (2 * p.WS + 2 * p.HS + 2) * 8;
+  // 128-byte aligned: the float4 statistics in the transpose region below
+  // inherit this alignment.
+  s.off_misc = (s.off_bar + (2 * p.WS + 2 * p.HS + 3) * 8 + 127) & ~127;
   s.off_rows = s.off_misc + 64;  // int/float [5][kMaxR] + int [3][kMaxB + 1]
   // Per epilogue warp a 32 x 33 float transpose buffer; after the last round
   // the same bytes hold the warps' per-row statistics (float4 [kEpiWarps][R]).
@@ -280,6 +284,9 @@ __device__ __forceinline__ ff2 warp_scan_ff(ff2 v, int lane) {
   return v;
 }
 
+// PAIR: the statistics pass on CTA pairs (tcgen05 cta_group::2); a kernel uses
+// one CTA granularity throughout, so pair mode is its own instance.
+template <bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tm_w3,
     const __grid_constant__ CUtensorMap tm_w2, const __grid_constant__ CUtensorMap tm_w2s,
@@ -298,6 +305,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   uint64_t *h_empty = h_full + p.HS;
   uint64_t *acc_full = h_empty + p.HS;
   uint64_t *acc_empty = acc_full + 1;
+  uint64_t *fin = acc_empty + 1;  // pair mode: teardown handshake
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L.off_misc);
   uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + L.off_misc + 8);
   int *s_any_stoch = reinterpret_cast<int *>(smem + L.off_misc + 16);
@@ -316,11 +324,18 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c = blockIdx.x;
   // This CTA's vocabulary slice [v_lo, v_hi): equal row counts (within one),
-  // cut into 128-row tiles; the last tile may be partial.
-  const int v_lo = static_cast<int>(static_cast<int64_t>(c) * p.V / p.NC);
-  const int v_hi = static_cast<int>(static_cast<int64_t>(c + 1) * p.V / p.NC);
-  const int ntiles = (v_hi - v_lo + kTileV - 1) / kTileV;
-  const bool short_last = (v_hi - v_lo) - (ntiles - 1) * kTileV <= p.BRS && p.BRS < kTileV;
+  // cut into 128-row tiles; the last tile may be partial.  Pair mode: the
+  // pair's slice, cut into 256-row pair tiles whose rows 0-127 belong to the
+  // even CTA and 128-255 to the odd one; tile t of this CTA starts at
+  // v_lo + t * tstride + toff.
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+  const int nsl = PAIR ? p.NC / 2 : p.NC, sl = PAIR ? c >> 1 : c;
+  const int v_lo = static_cast<int>(static_cast<int64_t>(sl) * p.V / nsl);
+  const int v_hi = static_cast<int>(static_cast<int64_t>(sl + 1) * p.V / nsl);
+  const int tstride = PAIR ? 2 * kTileV : kTileV;
+  const int toff = static_cast<int>(rank) * kTileV;
+  const int ntiles = (v_hi - v_lo + tstride - 1) / tstride;
+  const bool short_last = !PAIR && (v_hi - v_lo) - (ntiles - 1) * kTileV <= p.BRS && p.BRS < kTileV;
   // Second pass with nothing to sample: the whole grid leaves before any set-up.
   if (p.kind == kPresampled && *p.samp_count == 0) return;
 
@@ -331,13 +346,24 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     for (int s = 0; s < p.WS; ++s) { mbar_init(&w_full[s], 1); mbar_init(&w_empty[s], 1); }
     for (int s = 0; s < p.HS; ++s) { mbar_init(&h_full[s], 1); mbar_init(&h_empty[s], 1); }
     mbar_init(acc_full, 1);
-    mbar_init(acc_empty, kEpiWarps);
+    mbar_init(acc_empty, PAIR ? 2 * kEpiWarps : kEpiWarps);  // pair: both CTAs' epilogues
+    mbar_init(fin, 1);
+    if (PAIR && rank == 0) {
+      // Pair mode: arm every slot's first use with both CTAs' bytes.
+      for (int s = 0; s < p.WS; ++s) mbar_arrive_expect_tx(&w_full[s], 2 * kWChunkBytes);
+      for (int s = 0; s < p.HS; ++s) mbar_arrive_expect_tx(&h_full[s], 2 * p.h_boxes * p.h_box_rows * 128);
+    }
     mbar_init(q_bar, 33);  // thread 0 (with the copies' bytes) and the 32 lanes of warp 1
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(s_tmem, p.tmem_cols);
-    tmem_relinquish();
+    if constexpr (PAIR) {
+      tmem_alloc_pair(s_tmem, p.tmem_cols);  // collective: the same columns in both SMs
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(s_tmem, p.tmem_cols);
+      tmem_relinquish();
+    }
   }
   for (int n = tid; n < kMaxR; n += kThreads) { s_draft[n] = -1; s_seq[n] = -1; s_pos[n] = 0; }
   block_sync();
@@ -363,13 +389,15 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   }
   tc_fence_before();
   block_sync();
+  // Pair mode: both CTAs' barriers exist before either signals the other.
+  if constexpr (PAIR) cluster_sync();
   tc_fence_after();
   const uint32_t tmem = *s_tmem;
   int rounds_issued = 0;  // MMA thread: accumulator rounds committed
   // Every CTA reads the same hidden rows: CTA c walks the K stages starting at
   // stage c mod NS, so at any moment about NC / NS CTAs (not all of them) load
   // the same hidden lines from L2.  Each logit's sum over K changes order only.
-  const int k_rot = c % p.NS;
+  const int k_rot = sl % p.NS;  // a pair walks its stages in one order
   // A round that holds only the short last tile streams one k-chunk per stage
   // with its W rows and hidden rows together in one slot of either ring, so all
   // 4 + 3 slots are in flight (a two-ring stage keeps at most HS = 3 in flight,
@@ -379,7 +407,62 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
 
   // ======================= phase A: logits + slice statistics =============
   if (warp == 0) {
-    if (lane == 0 && ntiles > 0) {
+    if constexpr (PAIR) {
+     if (lane == 0 && ntiles > 0) {
+      // Pair mode (statistics pass, one k-chunk per stage): this CTA's 128 W
+      // rows of the pair tile, and its half of every MMA N-chunk of the hidden
+      // rows: N-chunk 0 covers rows [0, n0w), N-chunk 1 rows [n0w, Ncols); the
+      // even CTA holds the first half of each, the odd CTA the second.
+      tma_prefetch_desc(&tm_w2);
+      tma_prefetch_desc(&tm_h2);
+      const uint64_t pol_w = l2_policy_evict_first();
+      const uint64_t pol_h = l2_policy_evict_last();
+      const int hb = p.h_box_rows;  // n0w / 2
+      const int hrow0 = static_cast<int>(rank) * hb;
+      const int hrow1 = p.n0w + static_cast<int>(rank) * ((p.Ncols - p.n0w) / 2);
+      // Both CTAs' copies of a stage complete on the even CTA's full barrier,
+      // armed with the bytes of both before either CTA may issue them (at
+      // set-up, then by the MMA thread as it takes the previous use).
+      const uint32_t h_full0 = cluster_map(h_full, 0), w_full0 = cluster_map(w_full, 0);
+      uint32_t wi = 0, hi = 0, w_issued = 0, h_issued = 0;
+      for (int t = 0; t < ntiles; ++t) {
+        const int row0 = v_lo + t * tstride + toff;
+        for (int it = 0; it < p.NS; ++it) {
+          const int kc = it + k_rot < p.NS ? it + k_rot : it + k_rot - p.NS;
+          {
+            const int s = hi % p.HS;
+            mbar_wait(&h_empty[s], ((hi / p.HS) & 1) ^ 1, s_abort);
+            if (!*s_abort) {
+              uint8_t *dst = h_ring + s * L.h_slot;
+              for (int bi = 0; bi < p.h_boxes; ++bi)
+                tma_load_2d_pair(dst + bi * hb * 128, &tm_h2, kc * kKChunk, bi ? hrow1 : hrow0,
+                                 h_full0 + 8u * s, pol_h);
+              h_issued = hi + 1;
+            }
+            ++hi;
+          }
+          {
+            const int s = wi % p.WS;
+            mbar_wait(&w_empty[s], ((wi / p.WS) & 1) ^ 1, s_abort);
+            if (!*s_abort) {
+              tma_load_2d_pair(w_ring + s * L.w_slot, &tm_w2, kc * kKChunk, row0, w_full0 + 8u * s, pol_w);
+              w_issued = wi + 1;
+            }
+            ++wi;
+          }
+        }
+      }
+      // After an expired wait the even CTA drains the copies of both (its full
+      // barriers count them); the odd CTA's shared memory stays alive until
+      // the teardown handshake with the even CTA.
+      if (*s_abort && rank == 0) {
+        for (uint32_t j = (w_issued > (uint32_t)p.WS ? w_issued - p.WS : 0); j < w_issued; ++j)
+          mbar_wait_unabortable(&w_full[j % p.WS], (j / p.WS) & 1);
+        for (uint32_t j = (h_issued > (uint32_t)p.HS ? h_issued - p.HS : 0); j < h_issued; ++j)
+          mbar_wait_unabortable(&h_full[j % p.HS], (j / p.HS) & 1);
+      }
+     }
+    } else if (lane == 0 && ntiles > 0) {
       tma_prefetch_desc(&tm_w3);
       tma_prefetch_desc(&tm_w3s);
       tma_prefetch_desc(&tm_h3);
@@ -477,7 +560,48 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       }
     }
   } else if (warp == 1) {
-    if (lane == 0 && ntiles > 0) {
+    if constexpr (PAIR) {
+     if (lane == 0 && ntiles > 0 && rank == 0) {
+      // Pair mode, even CTA: M = 256 MMAs over both CTAs' stages (its full
+      // barriers complete when both CTAs' copies have landed); the slots are
+      // freed in both CTAs by one multicast commit.
+      uint32_t wi = 0, hi = 0;
+      const uint32_t hb_bytes = static_cast<uint32_t>(p.h_box_rows) * 128u;
+      const uint32_t h_pair_bytes = 2u * p.h_boxes * hb_bytes;
+      for (int t = 0; t < ntiles; ++t) {
+        if (t > 0) mbar_wait_cluster(acc_empty, (t - 1) & 1, s_abort);
+        tc_fence_after();
+        for (int it = 0; it < p.NS; ++it) {
+          const int hs = hi % p.HS, ws = wi % p.WS;
+          mbar_wait_cluster(&h_full[hs], (hi / p.HS) & 1, s_abort);
+          mbar_wait_cluster(&w_full[ws], (wi / p.WS) & 1, s_abort);
+          // Arm the slots' next use now: its copies are issued only after this
+          // stage's commit frees the slots.
+          mbar_arrive_expect_tx(&h_full[hs], h_pair_bytes);
+          mbar_arrive_expect_tx(&w_full[ws], 2 * kWChunkBytes);
+          tc_fence_after();
+          const uint32_t w_addr = smem_u32(w_ring + ws * L.w_slot);
+          const uint32_t h_addr = smem_u32(h_ring + hs * L.h_slot);
+          for (int ci = 0; ci < p.nchunks; ++ci) {
+#pragma unroll
+            for (int k16 = 0; k16 < kKChunk / 16; ++k16)
+              tc_mma_f16_pair(tmem + (ci ? static_cast<uint32_t>(p.n0w) : 0u),
+                              smem_desc_sw128(w_addr + 32 * k16),
+                              smem_desc_sw128(h_addr + ci * hb_bytes + 32 * k16), ci ? p.idesc1 : p.idesc,
+                              (it | k16) != 0);
+          }
+          tc_commit_pair(&w_empty[ws]);
+          tc_commit_pair(&h_empty[hs]);
+          ++wi;
+          ++hi;
+        }
+        tc_commit_pair(acc_full);
+        ++rounds_issued;
+      }
+     } else if (lane == 0 && ntiles > 0) {
+      rounds_issued = ntiles;  // odd CTA: the even CTA's commits reach its acc_full too
+     }
+    } else if (lane == 0 && ntiles > 0) {
       uint32_t wi = 0, hi = 0;
       int tdone = 0, used = 0;
       for (int r = 0; r < p.nrounds && tdone < ntiles; ++r) {
@@ -613,7 +737,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       // serially -- no shuffles.
       for (int j = 0; j < nt; ++j) {
         const int t = tdone + j;
-        const int vlane0 = v_lo + t * kTileV + q4 * 32;  // vocab id of lane 0's row
+        const int vlane0 = v_lo + t * tstride + toff + q4 * 32;  // vocab id of lane 0's row
         const bool my_valid = vlane0 + lane < v_hi;       // lanes past the slice are masked
         const uint32_t col = tmem + lane_base + static_cast<uint32_t>(p.kind == kStatsOnly ? 0 : t * p.Rs);
 #pragma unroll
@@ -655,10 +779,14 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         }
       }
       if (p.kind == kStatsOnly) {
-        // The accumulator slot is read: the next tile may overwrite it.
+        // The accumulator slot is read: the next tile may overwrite it (pair
+        // mode: the even CTA's MMA thread counts both CTAs' epilogue warps).
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(acc_empty);
+        if (lane == 0) {
+          if (rank == 0) mbar_arrive(acc_empty);
+          else mbar_arrive_cluster(cluster_map(acc_empty, 0));
+        }
       } else {
         used += nt * p.Rs;
       }
@@ -1322,9 +1450,35 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     // No MMA may still write TMEM when it is released (matters only after an
     // expired wait; otherwise the epilogue already consumed the last round).
     if (lane == 0 && rounds_issued > 0) mbar_wait_unabortable(acc_full, (rounds_issued - 1) & 1);
-    __syncwarp();
-    tc_fence_after();
-    tmem_dealloc(tmem, p.tmem_cols);
+    if constexpr (PAIR) {
+      // Pair mode: the allocation is released by both CTAs together, once
+      // both are done with it (bounded handshake on each other's `fin`).
+      if (lane == 0) {
+        mbar_arrive_cluster(cluster_map(fin, rank ^ 1u));
+        const uint64_t t0 = globaltimer();
+        uint32_t ok = 0;
+        while (!ok) {
+          asm volatile(
+              "{\n\t.reg .pred p;\n\t"
+              "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], 0;\n\t"
+              "selp.b32 %0, 1, 0, p;\n\t}"
+              : "=r"(ok)
+              : "r"(smem_u32(fin))
+              : "memory");
+          if (!ok && globaltimer() - t0 > kWaitLimitNs) {
+            atomicOr(p.status, SPADE_DEV_TIMEOUT);
+            break;
+          }
+        }
+      }
+      __syncwarp();
+      tc_fence_after();
+      tmem_dealloc_pair(tmem, p.tmem_cols);
+    } else {
+      __syncwarp();
+      tc_fence_after();
+      tmem_dealloc(tmem, p.tmem_cols);
+    }
   }
 }
 
@@ -1486,20 +1640,37 @@ static spade_status prepare(Params &p, int kind, const void *hidden, const void 
     return fail(SPADE_ERR_SHAPE, "vocabulary %d needs %d tiles per SM (max %d)", p.V, tiles_max,
                 kMaxTilesPerCta);
   p.tmem_cols = kTmemCols;
+  p.pair = 0;
   if (kind == kStatsOnly) {
     // One tile per round in one accumulator slot; rows beyond 256 take a
     // second MMA N-chunk.  Hidden rows arrive in <= 256-row boxes.
     if (pl.Ncols > kTmemCols) return fail(SPADE_ERR_SHAPE, "R = %d rows exceed %d", R, kTmemCols);
-    p.nrounds = tiles_max;
-    for (int r = 0; r < tiles_max; ++r) p.round_tiles[r] = 1;
     p.nchunks = pl.Ncols > 256 ? 2 : 1;
     p.n0w = p.nchunks == 2 ? ((pl.Ncols / 2 + 15) / 16 * 16) : pl.Ncols;
-    p.idesc = idesc_bf16_f32(kTileV, p.n0w);
-    p.idesc1 = idesc_bf16_f32(kTileV, p.nchunks == 2 ? pl.Ncols - p.n0w : 16);
-    p.h_boxes = p.nchunks;
-    p.h_box_rows = p.nchunks == 2 ? 256 : pl.Ncols;
-    p.HS = 2;
     p.KG = 1;
+    if (pl.NC % 2 == 0) {
+      // CTA pairs: M = 256 MMAs (cta_group::2) over 256-row pair tiles, each
+      // CTA holding half of every N-chunk's hidden rows, so an SM receives
+      // 128 W rows + Ncols / 2 hidden rows per k-chunk instead of
+      // 128 + Ncols: the statistics pass is bound by those bytes in flight.
+      p.pair = 1;
+      const int NP = pl.NC / 2;
+      const int lmax = (p.V + NP - 1) / NP;
+      tiles_max = (lmax + 2 * kTileV - 1) / (2 * kTileV);
+      p.idesc = idesc_bf16_f32(2 * kTileV, p.n0w);
+      p.idesc1 = idesc_bf16_f32(2 * kTileV, p.nchunks == 2 ? pl.Ncols - p.n0w : 16);
+      p.h_boxes = p.nchunks;
+      p.h_box_rows = p.n0w / 2;
+      p.HS = 4;
+    } else {
+      p.idesc = idesc_bf16_f32(kTileV, p.n0w);
+      p.idesc1 = idesc_bf16_f32(kTileV, p.nchunks == 2 ? pl.Ncols - p.n0w : 16);
+      p.h_boxes = p.nchunks;
+      p.h_box_rows = p.nchunks == 2 ? 256 : pl.Ncols;
+      p.HS = 2;
+    }
+    p.nrounds = tiles_max;
+    for (int r = 0; r < tiles_max; ++r) p.round_tiles[r] = 1;
   } else {
     if (!plan_rounds(tiles_max, pl.Ncols, pl.Rs, p.round_tiles, &p.nrounds))
       return fail(SPADE_ERR_SHAPE,
@@ -1561,9 +1732,10 @@ static spade_status prepare(Params &p, int kind, const void *hidden, const void 
 static spade_status launch(const Params &p, const Maps &m, cudaStream_t stream) {
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(verify_accept_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(verify_accept)");
+    for (auto kern : {verify_accept_kernel<false>, verify_accept_kernel<true>}) {
+      cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(verify_accept)");
+    }
     configured = true;
   }
   cudaLaunchConfig_t cfg = {};
@@ -1571,12 +1743,17 @@ static spade_status launch(const Params &p, const Maps &m, cudaStream_t stream) 
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem_layout(p).total;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeCooperative;
   attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;  // pair mode: CTAs 2j, 2j+1 share a cluster
+  attr[1].val.clusterDim.x = 2;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, verify_accept_kernel, p, m.w3, m.w2, m.w2s, m.w3s, m.h3, m.h2);
+  cfg.numAttrs = p.pair ? 2 : 1;
+  const cudaError_t e = p.pair ? cudaLaunchKernelEx(&cfg, verify_accept_kernel<true>, p, m.w3, m.w2, m.w2s, m.w3s, m.h3, m.h2)
+                               : cudaLaunchKernelEx(&cfg, verify_accept_kernel<false>, p, m.w3, m.w2, m.w2s, m.w3s, m.h3, m.h2);
   if (e != cudaSuccess) return cuda_fail(e, "verify_accept cooperative launch");
   return SPADE_OK;
 }
