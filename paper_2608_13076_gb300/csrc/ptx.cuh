@@ -244,19 +244,23 @@ SPADE_DEVICE void mbar_arrive_cluster(uint32_t cluster_addr) {
 }
 // Bounded wait (as mbar_wait) with cluster-scope acquire: for barriers that
 // the other CTA of the pair arrives on.
+SPADE_DEVICE bool mbar_try_wait_cluster(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.b32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 SPADE_DEVICE bool mbar_wait_cluster(uint64_t *bar, uint32_t parity, volatile int *abort) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;  // no timer read on the fast path
   const uint64_t t0 = globaltimer();
   while (true) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.b32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
-        : "memory");
-    if (ok) return true;
     if (*abort) return true;
+    if (mbar_try_wait_cluster(bar, parity)) return true;
     if (globaltimer() - t0 > kWaitLimitNs) {
       *abort = 1;
       return false;

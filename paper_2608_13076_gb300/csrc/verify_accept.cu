@@ -69,6 +69,7 @@ constexpr int kTmemCols = 512;
 constexpr int kSmemBudget = 220 * 1024;
 constexpr int kSmemMax = 225 * 1024;  // opt-in limit (227 KB) minus static shared memory
 constexpr int kWChunkBytes = kTileV * kKChunk * 2;  // 16 KB: one tile x one k-chunk
+static_assert(kEpiWarps * kMaxR * 16 <= 2 * kWChunkBytes, "per-warp row statistics fit two W slots");
 constexpr float kLog2e = 1.4426950408889634f;
 
 struct Params {
@@ -132,11 +133,11 @@ __host__ __device__ inline Smem smem_layout(const Params &p) {
   // inherit this alignment.
   s.off_misc = (s.off_bar + (2 * p.WS + 2 * p.HS + 3) * 8 + 127) & ~127;
   s.off_rows = s.off_misc + 64;  // int/float [5][kMaxR] + int [3][kMaxB + 1]
-  // Per epilogue warp a 32 x 33 float transpose buffer; after the last round
-  // the same bytes hold the warps' per-row statistics (float4 [kEpiWarps][R]).
+  // Per epilogue warp a 32 x 33 float transpose buffer.  After the last round
+  // the warps' per-row statistics (float4 [kEpiWarps][R], at most 32 KB) go to
+  // the start of the W ring (at least two 16 KB slots), idle by then.
   s.off_tbuf = s.off_rows + 5 * kMaxR * 4 + 3 * (kMaxB + 1) * 4 + 4;
-  const int tbuf = kEpiWarps * 32 * 33 * 4, wst = kEpiWarps * p.R * 16;
-  s.total = s.off_tbuf + (tbuf > wst ? tbuf : wst) + 1024;
+  s.total = s.off_tbuf + kEpiWarps * 32 * 33 * 4 + 1024;
   return s;
 }
 
@@ -319,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   int32_t *s_nd = s_cuq + kMaxB + 1;
   int32_t *s_md = s_nd + kMaxB;
   float *s_tbuf = reinterpret_cast<float *>(smem + L.off_tbuf);
-  float4 *s_wst = reinterpret_cast<float4 *>(smem + L.off_tbuf);  // after the last round
+  float4 *s_wst = reinterpret_cast<float4 *>(smem);  // after the last round (W ring)
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c = blockIdx.x;
@@ -408,58 +409,52 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   // ======================= phase A: logits + slice statistics =============
   if (warp == 0) {
     if constexpr (PAIR) {
-     if (lane == 0 && ntiles > 0) {
+     if (lane < 2 && ntiles > 0) {
       // Pair mode (statistics pass, one k-chunk per stage): this CTA's 128 W
-      // rows of the pair tile, and its half of every MMA N-chunk of the hidden
-      // rows: N-chunk 0 covers rows [0, n0w), N-chunk 1 rows [n0w, Ncols); the
-      // even CTA holds the first half of each, the odd CTA the second.
-      tma_prefetch_desc(&tm_w2);
-      tma_prefetch_desc(&tm_h2);
-      const uint64_t pol_w = l2_policy_evict_first();
-      const uint64_t pol_h = l2_policy_evict_last();
-      const int hb = p.h_box_rows;  // n0w / 2
-      const int hrow0 = static_cast<int>(rank) * hb;
-      const int hrow1 = p.n0w + static_cast<int>(rank) * ((p.Ncols - p.n0w) / 2);
+      // rows of the pair tile (lane 1), and its half of every MMA N-chunk of
+      // the hidden rows (lane 0): N-chunk 0 covers rows [0, n0w), N-chunk 1
+      // rows [n0w, Ncols); the even CTA holds the first half of each, the odd
+      // CTA the second.  The two rings run independently, so W (from HBM)
+      // keeps its slots in flight while the hidden ring waits for the MMAs.
       // Both CTAs' copies of a stage complete on the even CTA's full barrier,
       // armed with the bytes of both before either CTA may issue them (at
       // set-up, then by the MMA thread as it takes the previous use).
-      const uint32_t h_full0 = cluster_map(h_full, 0), w_full0 = cluster_map(w_full, 0);
-      uint32_t wi = 0, hi = 0, w_issued = 0, h_issued = 0;
+      const bool is_w = lane == 1;
+      tma_prefetch_desc(is_w ? &tm_w2 : &tm_h2);
+      const uint64_t pol = is_w ? l2_policy_evict_first() : l2_policy_evict_last();
+      const int hb = p.h_box_rows;  // n0w / 2
+      const int hrow0 = static_cast<int>(rank) * hb;
+      const int hrow1 = p.n0w + static_cast<int>(rank) * ((p.Ncols - p.n0w) / 2);
+      uint64_t *const full = is_w ? w_full : h_full;
+      uint64_t *const empty = is_w ? w_empty : h_empty;
+      const uint32_t full0 = cluster_map(full, 0);
+      const int slots = is_w ? p.WS : p.HS;
+      uint8_t *const ring = is_w ? w_ring : h_ring;
+      const int slot_bytes = is_w ? L.w_slot : L.h_slot;
+      uint32_t i = 0, issued = 0;
       for (int t = 0; t < ntiles; ++t) {
         const int row0 = v_lo + t * tstride + toff;
-        for (int it = 0; it < p.NS; ++it) {
+        for (int it = 0; it < p.NS; ++it, ++i) {
           const int kc = it + k_rot < p.NS ? it + k_rot : it + k_rot - p.NS;
-          {
-            const int s = hi % p.HS;
-            mbar_wait(&h_empty[s], ((hi / p.HS) & 1) ^ 1, s_abort);
-            if (!*s_abort) {
-              uint8_t *dst = h_ring + s * L.h_slot;
-              for (int bi = 0; bi < p.h_boxes; ++bi)
-                tma_load_2d_pair(dst + bi * hb * 128, &tm_h2, kc * kKChunk, bi ? hrow1 : hrow0,
-                                 h_full0 + 8u * s, pol_h);
-              h_issued = hi + 1;
-            }
-            ++hi;
+          const int s = i % slots;
+          mbar_wait(&empty[s], ((i / slots) & 1) ^ 1, s_abort);
+          if (*s_abort) continue;
+          uint8_t *dst = ring + s * slot_bytes;
+          if (is_w) {
+            tma_load_2d_pair(dst, &tm_w2, kc * kKChunk, row0, full0 + 8u * s, pol);
+          } else {
+            for (int bi = 0; bi < p.h_boxes; ++bi)
+              tma_load_2d_pair(dst + bi * hb * 128, &tm_h2, kc * kKChunk, bi ? hrow1 : hrow0, full0 + 8u * s, pol);
           }
-          {
-            const int s = wi % p.WS;
-            mbar_wait(&w_empty[s], ((wi / p.WS) & 1) ^ 1, s_abort);
-            if (!*s_abort) {
-              tma_load_2d_pair(w_ring + s * L.w_slot, &tm_w2, kc * kKChunk, row0, w_full0 + 8u * s, pol_w);
-              w_issued = wi + 1;
-            }
-            ++wi;
-          }
+          issued = i + 1;
         }
       }
       // After an expired wait the even CTA drains the copies of both (its full
       // barriers count them); the odd CTA's shared memory stays alive until
       // the teardown handshake with the even CTA.
       if (*s_abort && rank == 0) {
-        for (uint32_t j = (w_issued > (uint32_t)p.WS ? w_issued - p.WS : 0); j < w_issued; ++j)
-          mbar_wait_unabortable(&w_full[j % p.WS], (j / p.WS) & 1);
-        for (uint32_t j = (h_issued > (uint32_t)p.HS ? h_issued - p.HS : 0); j < h_issued; ++j)
-          mbar_wait_unabortable(&h_full[j % p.HS], (j / p.HS) & 1);
+        for (uint32_t j = (issued > (uint32_t)slots ? issued - slots : 0); j < issued; ++j)
+          mbar_wait_unabortable(&full[j % slots], (j / slots) & 1);
       }
      }
     } else if (lane == 0 && ntiles > 0) {
@@ -573,8 +568,10 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         tc_fence_after();
         for (int it = 0; it < p.NS; ++it) {
           const int hs = hi % p.HS, ws = wi % p.WS;
-          mbar_wait_cluster(&h_full[hs], (hi / p.HS) & 1, s_abort);
-          mbar_wait_cluster(&w_full[ws], (wi / p.WS) & 1, s_abort);
+          // (cta-scope waits: the copies' completion on this barrier orders them
+          // for the MMAs issued after it, the odd CTA's included)
+          mbar_wait(&h_full[hs], (hi / p.HS) & 1, s_abort);
+          mbar_wait(&w_full[ws], (wi / p.WS) & 1, s_abort);
           // Arm the slots' next use now: its copies are issued only after this
           // stage's commit frees the slots.
           mbar_arrive_expect_tx(&h_full[hs], h_pair_bytes);
