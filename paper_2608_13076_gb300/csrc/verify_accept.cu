@@ -431,22 +431,24 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       const int slots = is_w ? p.WS : p.HS;
       uint8_t *const ring = is_w ? w_ring : h_ring;
       const int slot_bytes = is_w ? L.w_slot : L.h_slot;
-      uint32_t i = 0, issued = 0;
+      uint32_t i = 0, issued = 0, eph = 1;  // empty-barrier parity (the first pass: the preceding phase)
+      int s = 0;                           // slot and parity advance by counters
       for (int t = 0; t < ntiles; ++t) {
         const int row0 = v_lo + t * tstride + toff;
         for (int it = 0; it < p.NS; ++it, ++i) {
           const int kc = it + k_rot < p.NS ? it + k_rot : it + k_rot - p.NS;
-          const int s = i % slots;
-          mbar_wait(&empty[s], ((i / slots) & 1) ^ 1, s_abort);
-          if (*s_abort) continue;
-          uint8_t *dst = ring + s * slot_bytes;
-          if (is_w) {
-            tma_load_2d_pair(dst, &tm_w2, kc * kKChunk, row0, full0 + 8u * s, pol);
-          } else {
-            for (int bi = 0; bi < p.h_boxes; ++bi)
-              tma_load_2d_pair(dst + bi * hb * 128, &tm_h2, kc * kKChunk, bi ? hrow1 : hrow0, full0 + 8u * s, pol);
+          mbar_wait(&empty[s], eph, s_abort);
+          if (!*s_abort) {
+            uint8_t *dst = ring + s * slot_bytes;
+            if (is_w) {
+              tma_load_2d_pair(dst, &tm_w2, kc * kKChunk, row0, full0 + 8u * s, pol);
+            } else {
+              for (int bi = 0; bi < p.h_boxes; ++bi)
+                tma_load_2d_pair(dst + bi * hb * 128, &tm_h2, kc * kKChunk, bi ? hrow1 : hrow0, full0 + 8u * s, pol);
+            }
+            issued = i + 1;
           }
-          issued = i + 1;
+          if (++s == slots) { s = 0; eph ^= 1u; }
         }
       }
       // After an expired wait the even CTA drains the copies of both (its full
@@ -560,18 +562,19 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       // Pair mode, even CTA: M = 256 MMAs over both CTAs' stages (its full
       // barriers complete when both CTAs' copies have landed); the slots are
       // freed in both CTAs by one multicast commit.
-      uint32_t wi = 0, hi = 0;
+      // Slot indices and phases advance by counters (no divisions per stage).
+      int hs = 0, ws = 0;
+      uint32_t hph = 0, wph = 0;
       const uint32_t hb_bytes = static_cast<uint32_t>(p.h_box_rows) * 128u;
       const uint32_t h_pair_bytes = 2u * p.h_boxes * hb_bytes;
       for (int t = 0; t < ntiles; ++t) {
         if (t > 0) mbar_wait_cluster(acc_empty, (t - 1) & 1, s_abort);
         tc_fence_after();
         for (int it = 0; it < p.NS; ++it) {
-          const int hs = hi % p.HS, ws = wi % p.WS;
           // (cta-scope waits: the copies' completion on this barrier orders them
           // for the MMAs issued after it, the odd CTA's included)
-          mbar_wait(&h_full[hs], (hi / p.HS) & 1, s_abort);
-          mbar_wait(&w_full[ws], (wi / p.WS) & 1, s_abort);
+          mbar_wait(&h_full[hs], hph, s_abort);
+          mbar_wait(&w_full[ws], wph, s_abort);
           // Arm the slots' next use now: its copies are issued only after this
           // stage's commit frees the slots.
           mbar_arrive_expect_tx(&h_full[hs], h_pair_bytes);
@@ -589,8 +592,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           }
           tc_commit_pair(&w_empty[ws]);
           tc_commit_pair(&h_empty[hs]);
-          ++wi;
-          ++hi;
+          if (++hs == p.HS) { hs = 0; hph ^= 1u; }
+          if (++ws == p.WS) { ws = 0; wph ^= 1u; }
         }
         tc_commit_pair(acc_full);
         ++rounds_issued;
