@@ -466,6 +466,9 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       const uint64_t pol_w = l2_policy_evict_first();
       const uint64_t pol_h = l2_policy_evict_last();
       uint32_t wi = 0, hi = 0, w_issued = 0, h_issued = 0;
+      // Ring slots and parities advance by counters (no per-stage divisions).
+      int ws_ = 0, hs_ = 0;
+      uint32_t wph_ = 0, hph_ = 0;
       int tdone = 0;
       for (int r = 0; r < p.nrounds && tdone < ntiles; ++r) {
         const int nt = min(p.round_tiles[r], ntiles - tdone);
@@ -475,10 +478,9 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           for (int it = 0; it < p.KC; ++it) {
             const int kc = it + kr < p.KC ? it + kr : it + kr - p.KC;
             const bool use_w = it % 7 < 4;  // four W slots, then three H slots
-            const int s = use_w ? wi % p.WS : hi % p.HS;
+            const int s = use_w ? ws_ : hs_;
             uint64_t *full = use_w ? &w_full[s] : &h_full[s];
-            mbar_wait(use_w ? &w_empty[s] : &h_empty[s],
-                      ((use_w ? wi / p.WS : hi / p.HS) & 1) ^ 1, s_abort);
+            mbar_wait(use_w ? &w_empty[s] : &h_empty[s], (use_w ? wph_ : hph_) ^ 1, s_abort);
             if (!*s_abort) {
               uint8_t *dst = use_w ? w_ring + s * L.w_slot : h_ring + s * L.h_slot;
               mbar_arrive_expect_tx(full, (p.BRS + p.h_box_rows) * 128);
@@ -486,7 +488,13 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               tma_load_2d(dst + p.BRS * 128, &tm_h2, kc * kKChunk, 0, full, pol_h);
               if (use_w) w_issued = wi + 1; else h_issued = hi + 1;
             }
-            if (use_w) ++wi; else ++hi;
+            if (use_w) {
+              ++wi;
+              if (++ws_ == p.WS) { ws_ = 0; wph_ ^= 1u; }
+            } else {
+              ++hi;
+              if (++hs_ == p.HS) { hs_ = 0; hph_ ^= 1u; }
+            }
           }
           tdone += nt;
           continue;
@@ -497,8 +505,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           const int nch = min(p.KG, p.KC - c0);
           const bool box3 = (nch == p.KG) && (c0 + p.KG <= p.KCF);
           {
-            const int s = hi % p.HS;
-            mbar_wait(&h_empty[s], ((hi / p.HS) & 1) ^ 1, s_abort);
+            const int s = hs_;
+            mbar_wait(&h_empty[s], hph_ ^ 1, s_abort);
             if (!*s_abort) {
               uint8_t *dst = h_ring + s * L.h_slot;
               const int hk = p.h_boxes * p.h_box_rows * 128;  // bytes per k-chunk
@@ -514,10 +522,11 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               h_issued = hi + 1;
             }
             ++hi;
+            if (++hs_ == p.HS) { hs_ = 0; hph_ ^= 1u; }
           }
           for (int j = 0; j < nt; ++j) {
-            const int s = wi % p.WS;
-            mbar_wait(&w_empty[s], ((wi / p.WS) & 1) ^ 1, s_abort);
+            const int s = ws_;
+            mbar_wait(&w_empty[s], wph_ ^ 1, s_abort);
             if (!*s_abort) {
               uint8_t *dst = w_ring + s * L.w_slot;
               const int row0 = v_lo + (tdone + j) * kTileV;
@@ -544,6 +553,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               w_issued = wi + 1;
             }
             ++wi;
+            if (++ws_ == p.WS) { ws_ = 0; wph_ ^= 1u; }
           }
         }
         tdone += nt;
@@ -602,7 +612,9 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       rounds_issued = ntiles;  // odd CTA: the even CTA's commits reach its acc_full too
      }
     } else if (lane == 0 && ntiles > 0) {
-      uint32_t wi = 0, hi = 0;
+      // Ring slots and parities advance by counters (no per-stage divisions).
+      int ws_ = 0, hs_ = 0;
+      uint32_t wph_ = 0, hph_ = 0;
       int tdone = 0, used = 0;
       for (int r = 0; r < p.nrounds && tdone < ntiles; ++r) {
         const int nt = min(p.round_tiles[r], ntiles - tdone);
@@ -612,8 +624,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           const uint32_t d_tmem = tmem + static_cast<uint32_t>(used);
           for (int it = 0; it < p.KC; ++it) {
             const bool use_w = it % 7 < 4;
-            const int s = use_w ? wi % p.WS : hi % p.HS;
-            mbar_wait(use_w ? &w_full[s] : &h_full[s], (use_w ? wi / p.WS : hi / p.HS) & 1, s_abort);
+            const int s = use_w ? ws_ : hs_;
+            mbar_wait(use_w ? &w_full[s] : &h_full[s], use_w ? wph_ : hph_, s_abort);
             tc_fence_after();
             const uint32_t base = smem_u32(use_w ? w_ring + s * L.w_slot : h_ring + s * L.h_slot);
 #pragma unroll
@@ -621,7 +633,11 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               tc_mma_f16(d_tmem, smem_desc_sw128(base + 32 * k16), smem_desc_sw128(base + p.BRS * 128 + 32 * k16),
                          p.idesc, (it | k16) != 0);
             tc_commit(use_w ? &w_empty[s] : &h_empty[s]);
-            if (use_w) ++wi; else ++hi;
+            if (use_w) {
+              if (++ws_ == p.WS) { ws_ = 0; wph_ ^= 1u; }
+            } else {
+              if (++hs_ == p.HS) { hs_ = 0; hph_ ^= 1u; }
+            }
           }
           tc_commit(acc_full);
           ++rounds_issued;
@@ -632,13 +648,13 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         for (int it = 0; it < p.NS; ++it) {
           const int ks = it + k_rot < p.NS ? it + k_rot : it + k_rot - p.NS;
           const int nch = min(p.KG, p.KC - ks * p.KG);
-          const int hs = hi % p.HS;
-          mbar_wait(&h_full[hs], (hi / p.HS) & 1, s_abort);
+          const int hs = hs_;
+          mbar_wait(&h_full[hs], hph_, s_abort);
           tc_fence_after();
           const uint32_t h_addr = smem_u32(h_ring + hs * L.h_slot);
           for (int j = 0; j < nt; ++j) {
-            const int ws = wi % p.WS;
-            mbar_wait(&w_full[ws], (wi / p.WS) & 1, s_abort);
+            const int ws = ws_;
+            mbar_wait(&w_full[ws], wph_, s_abort);
             tc_fence_after();
             const uint32_t w_addr = smem_u32(w_ring + ws * L.w_slot);
             // k-chunk stride in the slot: a full tile's chunks are 16 KB apart,
@@ -660,10 +676,10 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               }
             }
             tc_commit(&w_empty[ws]);
-            ++wi;
+            if (++ws_ == p.WS) { ws_ = 0; wph_ ^= 1u; }
           }
           tc_commit(&h_empty[hs]);
-          ++hi;
+          if (++hs_ == p.HS) { hs_ = 0; hph_ ^= 1u; }
         }
         tc_commit(acc_full);
         ++rounds_issued;
