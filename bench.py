@@ -296,6 +296,33 @@ def run_spade(args, ws, rank, local):
                "overlap": "inputs of step i+1 copied on a second stream while step i runs",
                "state_resident": "KV cache and W_lm stay in HBM (model state)"}
 
+    # Kernel launches per step: attention, the accept call's one or two passes
+    # (asked from the library), the separate commit if requested.
+    n_acc_launches = spade.spade_accept_launches(B, R, wl["H"], wl["V"])
+
+    # ---- the LM head's statistics pass alone (two-pass shapes) ----------------
+    # It runs every LM-head flop; the sampling pass recomputes only the rows to
+    # sample, and exits at once when no sequence samples.  So the accept call
+    # with every sequence greedy times the statistics pass (plus that empty
+    # second launch), after the timed region, L2 flushed between calls.
+    pass1 = None
+    if n_acc_launches == 2:
+        greedy = torch.zeros_like(wl["mode"])
+        acc_g = torch.zeros_like(acc)
+        tok_g = torch.zeros_like(tok)
+        ev1 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
+        for i in range(13):
+            if flush:
+                flush_buf.zero_()
+            if i >= 3:
+                ev1[i - 3][0].record(stream)
+            spade.spade_verify_accept(wl["hidden"], wl["w_lm"], wl["draft_tokens"], wl["draft_probs"],
+                                      wl["uniforms"], greedy, wl["cu_q"], wl["n_draft"], acc_g, tok_g,
+                                      workspace=ws_acc, status=status)
+            if i >= 3:
+                ev1[i - 3][1].record(stream)
+        torch.cuda.synchronize()
+        pass1 = statistics.median(a.elapsed_time(b) * 1e-3 for a, b in ev1)
     hbm, bf16, bf16_sus, peak_src = _peaks()
     m_acc = statistics.mean(t_acc)
     m_attn = statistics.mean(t_attn)
@@ -325,9 +352,14 @@ def run_spade(args, ws, rank, local):
                         "kv_commit": statistics.mean(t_com) * 1e6} if args.separate_commit else
                        {"verify_attention": m_attn * 1e6, "verify_accept_commit": m_acc * 1e6}),
         "roofline": dominant, "roofline_attention": roof_attn, "roofline_lm_head": roof_lm,
-        "e2e": e2e, "gpu_launches": (3 if args.separate_commit else 2) * args.steps, "wall_s_timed_loop": t_wall,
+        "e2e": e2e, "gpu_launches": (1 + n_acc_launches + (1 if args.separate_commit else 0)) * args.steps,
+        "wall_s_timed_loop": t_wall,
         "clocks": clk.summary(),
     }
+    if pass1 is not None:
+        line["lm_head_pass1"] = {"us": pass1 * 1e6, "tensor_tflops": lm_flop / pass1 / 1e12,
+                                 "tensor_frac_of_bf16_peak": lm_flop / pass1 / 1e12 / bf16, "peak_source": peak_src,
+                                 "how": "accept call with every sequence greedy (the sampling pass exits at once)"}
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl)
     return line

@@ -182,6 +182,16 @@ spade_status spade_verify_accept(const void *hidden, const void *w_lm,
 size_t spade_accept_workspace_size(int32_t B, int32_t R, int32_t H, int32_t V);
 
 /*
+ * Kernel launches one spade_verify_accept (or spade_verify_accept_commit) call
+ * makes for these sizes on the current device: 1 when the logits of all R
+ * rows stay on chip, 2 when they do not (a statistics pass over all rows --
+ * on pairs of SMs sharing each MMA when the grid is even -- then a pass that
+ * recomputes only the rows to sample); 0 on invalid sizes.  For launch
+ * accounting and graph capture; no device work.
+ */
+int32_t spade_accept_launches(int32_t B, int32_t R, int32_t H, int32_t V);
+
+/*
  * spade_verify_accept followed by spade_kv_commit, in one launch: once the
  * accept decisions are taken on the device, the same kernel clears the
  * rejected draft slots [ctx_b + a_b + 1, ctx_b + n_draft[b]] of k_cache and

@@ -23,7 +23,7 @@ from . import _build
 __all__ = [
     "SpadeError", "load", "build", "library_path",
     "spade_verify_attention", "spade_verify_accept", "spade_kv_commit", "spade_verify_attention_noalloc",
-    "spade_attn_workspace_size", "spade_accept_workspace_size",
+    "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_accept_launches",
     "attn_workspace", "accept_workspace", "status_tensor", "check_status",
     "DEV_BAD_INDEX", "DEV_CAPACITY", "DEV_TIMEOUT", "DEV_FALLBACK",
 ]
@@ -81,6 +81,8 @@ def load():
     lib.spade_verify_accept_commit.argtypes = [_vp] * 13 + [_i32] * 7 + [_vp, _sz, _vp, _vp]
     lib.spade_accept_workspace_size.restype = _sz
     lib.spade_accept_workspace_size.argtypes = [_i32] * 4
+    lib.spade_accept_launches.restype = _i32
+    lib.spade_accept_launches.argtypes = [_i32] * 4
     lib.spade_kv_commit.restype = _i32
     lib.spade_kv_commit.argtypes = [_vp] * 5 + [_i32] * 4 + [_vp, _vp]
     lib.spade_status_string.restype = ctypes.c_char_p
@@ -195,6 +197,11 @@ def spade_verify_attention_noalloc(q, k_cache, v_cache, ctx_lens, n_draft, cu_q,
 # ---------------------------------------------------------------------------
 def spade_accept_workspace_size(B, R, H, V):
     return int(load().spade_accept_workspace_size(B, R, H, V))
+
+
+def spade_accept_launches(B, R, H, V):
+    """Kernel launches of one accept call: 1 (logits on chip) or 2 (statistics pass, then sampling pass)."""
+    return int(load().spade_accept_launches(B, R, H, V))
 
 
 def accept_workspace(B, R, H, V, device="cuda"):

@@ -1786,6 +1786,13 @@ static void set_region(Params &p, uint8_t *ws, const WsRegion &r) {
 
 using namespace spade;
 
+extern "C" int32_t spade_accept_launches(int32_t B, int32_t R, int32_t H, int32_t V) {
+  if (B <= 0 || R < B || H <= 0 || V <= 0) return 0;
+  int sms = 0;
+  if (device_info(&sms, nullptr) != SPADE_OK) return 0;
+  return accept::ws_layout(B, R, H, V, sms).two_pass ? 2 : 1;
+}
+
 extern "C" size_t spade_accept_workspace_size(int32_t B, int32_t R, int32_t H, int32_t V) {
   if (B <= 0 || R < B || H <= 0 || V <= 0) return 0;
   int sms = 0;

@@ -71,6 +71,13 @@ def test_null_arguments_rejected_before_any_device_work(lib):
     assert rc == 1
 
 
+def test_launch_count_rejects_invalid_sizes(lib):
+    # Validation precedes the device query, so these need no GPU.
+    assert lib.spade_accept_launches(0, 5, 512, 1024) == 0
+    assert lib.spade_accept_launches(4, 3, 512, 1024) == 0   # R < B
+    assert lib.spade_accept_launches(1, 5, 0, 1024) == 0
+
+
 def test_bad_shapes_rejected(lib):
     p = ctypes.c_void_p(16)
     args = [p] * 7 + [None]

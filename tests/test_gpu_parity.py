@@ -147,6 +147,15 @@ def test_accept_commit_fused_small(dev, name):
     assert torch.equal(kc2, kc) and torch.equal(vc2, vc)
 
 
+def test_accept_launch_count(dev):
+    """One launch while the logits stay on chip, two for the two-pass shapes."""
+    for name, want in (("gqa_mixed", 1), ("two_pass_mixed", 2), ("two_pass_stochastic", 2)):
+        wl = W.make_workload(SMALL[name], device="cpu")
+        assert spade.spade_accept_launches(wl["B"], wl["R"], wl["H"], wl["V"]) == want, name
+    wl = W.make_workload(W.SPECS["ragged"], device="cpu")
+    assert spade.spade_accept_launches(wl["B"], wl["R"], wl["H"], wl["V"]) == 2
+
+
 def test_repeat_calls_reuse_workspace(dev):
     """Workspaces stay valid across calls (self-resetting counters / barriers)."""
     spec = SMALL["many_rows"]
