@@ -586,16 +586,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int64_t c_last = sc.owner(g.ust + sc.E + g.nch - 1);
       const int nparts = static_cast<int>(c_last - c_first + 1);
       if (nparts == 1) {
+        // Output row of this warp's row c0 + r, advanced row by row (one
+        // division for the warp's first row instead of one per row).
+        const int row0 = kRowBlock * g.rb + c0;
+        int gh = row0 % p.G;
+        size_t orow = static_cast<size_t>(q_row0 + row0 / p.G) * p.Hq + g.kvh * p.G + gh;
 #pragma unroll
         for (int j = 0; j < NH / 8; ++j) {
           uint32_t o8[8];
           tmem_ld8(tlane + kColO + c0 + j * 8, o8);
           tmem_wait_ld();
 #pragma unroll
-          for (int e = 0; e < 8; ++e)
+          for (int e = 0; e < 8; ++e) {
+            // l >= 1 (the row maximum's own term), so the fast divide is exact
+            // to a few fp32 ulps, far below the bf16 rounding that follows.
             if (j * 8 + e < hi)
-              p.out[out_row(p, q_row0, g.kvh, g.rb, c0 + j * 8 + e) * kD + t] =
-                  __float2bfloat16_rn(__uint_as_float(o8[e]) / l[j * 8 + e]);
+              p.out[orow * kD + t] = __float2bfloat16_rn(__fdividef(__uint_as_float(o8[e]), l[j * 8 + e]));
+            if (++gh == p.G) {
+              gh = 0;
+              orow += p.Hq - p.G + 1;
+            } else {
+              ++orow;
+            }
+          }
         }
         tc_fence_before();
         if (p.lse && row_writer)
