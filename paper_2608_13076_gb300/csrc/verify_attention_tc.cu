@@ -70,7 +70,8 @@ struct Smem {
   static constexpr int ALPHA = RMAX + kRowBlock * 4;        // float [64 rows]: rescale factors
   static constexpr int BAR = ALPHA + kRowBlock * 4;
   static constexpr int MISC = BAR + kNumBars * 8;           // abort, last, tmem base
-  static constexpr int BYTES = MISC + 64 + 1024;            // + slack for 1024-byte alignment
+  static constexpr int SEG0 = MISC + 64;                    // SegInfo: this CTA's first segment
+  static constexpr int BYTES = SEG0 + 64 + 1024;            // + slack for 1024-byte alignment
 };
 static_assert(Smem::BAR % 8 == 0, "mbarriers need 8-byte alignment");
 static_assert(Smem::RMAX % 16 == 0, "row maxima are read as float4");
@@ -198,47 +199,69 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int lane = tid & 31;
 
   if (tid == 0) { *s_abort = 0; *s_last = 0; }
+  // The producer's tensor-map fetches overlap the schedule loads below.
+  if (warp == 0 && lane < 2) {
+    tma_prefetch_desc(lane ? &tm_v2 : &tm_k2);
+    tma_prefetch_desc(lane ? &tm_v1 : &tm_k1);
+  }
   sched_validate(p, s_ctx, s_kd, tid, kThreads);
   block_sync();
   Sched sc;
   sc.pref = s_pref; sc.ctx = s_ctx; sc.kd = s_kd;
   sc.B = p.B; sc.Hkv = p.Hkv; sc.G = p.G; sc.RB = p.RB; sc.E = p.unit_cost; sc.num_ctas = p.num_ctas;
+  // One barrier for the schedule (warp 0: the prefix scan, then this CTA's
+  // first segment, which every role starts from) and the mbarriers and the
+  // tensor-memory allocation (warp 1).
+  SegInfo *s_seg0 = reinterpret_cast<SegInfo *>(smem + Smem::SEG0);
   if (warp == 0) {
     sched_scan(p, sc, s_pref, lane);
-  } else if (warp == 1 && lane == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&bars[kBarKFull + s], 1);
-      mbar_init(&bars[kBarVFull + s], 1);
-      mbar_init(&bars[kBarKEmpty + s], 1);
-      mbar_init(&bars[kBarVEmpty + s], 1);
-      mbar_init(&bars[kBarSFull + s], 1);
-      mbar_init(&bars[kBarSFree + s], kSoftWarps);
-      mbar_init(&bars[kBarPFull + s], kSoftWarps);
-      mbar_init(&bars[kBarPFree + s], 1);
+    __syncwarp();
+    if (lane == 0) {
+      Sched s0 = sc;
+      s0.total = s_pref[p.B];
+      s0.num_ctas = static_cast<int>(s0.total < p.num_ctas ? s0.total : p.num_ctas);
+      if (s0.total > 0 && static_cast<int>(blockIdx.x) < s0.num_ctas) {
+        const int64_t xb = static_cast<int64_t>(blockIdx.x) * s0.total / s0.num_ctas;
+        const int64_t xe = static_cast<int64_t>(blockIdx.x + 1) * s0.total / s0.num_ctas;
+        *s_seg0 = next_seg(s0, xb, xe);
+      }
     }
-    mbar_init(&bars[kBarODone], 1);
-    mbar_init(&bars[kBarSeg], kSoftWarps);
-    mbar_init(&bars[kBarQ], kSoftWarps);
-    mbar_init(&bars[kBarOFinal], 1);
-    fence_mbar_init();
-  }
-  block_sync();
-  sc.total = s_pref[p.B];
-  if (sc.total == 0) return;
-  // Never more CTAs than slices: every CTA kept has a non-empty range, so the
-  // CTAs between a unit's first and last owner all contribute a partial.
-  sc.num_ctas = static_cast<int>(sc.total < p.num_ctas ? sc.total : p.num_ctas);
-  if (static_cast<int>(blockIdx.x) >= sc.num_ctas) return;
-  const int64_t x_begin = static_cast<int64_t>(blockIdx.x) * sc.total / sc.num_ctas;
-  const int64_t x_end = static_cast<int64_t>(blockIdx.x + 1) * sc.total / sc.num_ctas;
-
-  if (warp == 1) {
+  } else if (warp == 1) {
+    if (lane == 0) {
+      for (int s = 0; s < kStages; ++s) {
+        mbar_init(&bars[kBarKFull + s], 1);
+        mbar_init(&bars[kBarVFull + s], 1);
+        mbar_init(&bars[kBarKEmpty + s], 1);
+        mbar_init(&bars[kBarVEmpty + s], 1);
+        mbar_init(&bars[kBarSFull + s], 1);
+        mbar_init(&bars[kBarSFree + s], kSoftWarps);
+        mbar_init(&bars[kBarPFull + s], kSoftWarps);
+        mbar_init(&bars[kBarPFree + s], 1);
+      }
+      mbar_init(&bars[kBarODone], 1);
+      mbar_init(&bars[kBarSeg], kSoftWarps);
+      mbar_init(&bars[kBarQ], kSoftWarps);
+      mbar_init(&bars[kBarOFinal], 1);
+      fence_mbar_init();
+    }
+    __syncwarp();
     tmem_alloc(s_tmem, kTmemCols);
     tmem_relinquish();
   }
   tc_fence_before();
   block_sync();
   tc_fence_after();
+  sc.total = s_pref[p.B];
+  // Never more CTAs than slices: every CTA kept has a non-empty range, so the
+  // CTAs between a unit's first and last owner all contribute a partial.
+  sc.num_ctas = static_cast<int>(sc.total < p.num_ctas ? sc.total : p.num_ctas);
+  if (sc.total == 0 || static_cast<int>(blockIdx.x) >= sc.num_ctas) {
+    if (warp == 1) tmem_dealloc(*s_tmem, kTmemCols);
+    return;
+  }
+  const int64_t x_begin = static_cast<int64_t>(blockIdx.x) * sc.total / sc.num_ctas;
+  const int64_t x_end = static_cast<int64_t>(blockIdx.x + 1) * sc.total / sc.num_ctas;
+  const SegInfo seg0 = *s_seg0;
   const uint32_t tmem = *s_tmem;
   const uint32_t smem_base = smem_u32(smem);
 
@@ -251,8 +274,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool is_v = lane == 1;
       const CUtensorMap *tm2 = is_v ? &tm_v2 : &tm_k2;
       const CUtensorMap *tm1 = is_v ? &tm_v1 : &tm_k1;
-      tma_prefetch_desc(tm2);
-      tma_prefetch_desc(tm1);
       const int bar_empty = is_v ? kBarVEmpty : kBarKEmpty;
       const int bar_full = is_v ? kBarVFull : kBarKFull;
       uint8_t *const ring = smem + (is_v ? Smem::V : Smem::K);
@@ -260,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t it = 0, issued = 0;
       bool expired = false;
       for (int64_t x = x_begin; x < x_end;) {
-        const SegInfo si = next_seg(sc, x, x_end);
+        const SegInfo si = x == x_begin ? seg0 : next_seg(sc, x, x_end);
         if (si.n_here == 0) break;
         const int row0 = (si.g.b * p.Hkv + si.g.kvh) * p.cap;
         for (int c = 0; c < si.nchunk; ++c, ++it) {
@@ -321,7 +342,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (last) tc_commit(&bars[kBarOFinal]);
       };
       for (int64_t x = x_begin; x < x_end;) {
-        const SegInfo si = next_seg(sc, x, x_end);
+        const SegInfo si = x == x_begin ? seg0 : next_seg(sc, x, x_end);
         if (si.n_here == 0) break;
         // Q staged: the segment's S products may start while the previous
         // segment's epilogue still reads O^T.
@@ -381,7 +402,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     };
 
-    SegInfo si = next_seg(sc, x_begin, x_end);
+    SegInfo si = seg0;
     if (si.n_here > 0) prefetch_q(si, 0);
     cp_async_commit();
     for (int64_t x = x_begin; x < x_end && si.n_here > 0;) {
