@@ -33,6 +33,10 @@ SMALL = {
                                      ctx=(5, 300), k=(4, 10), mode="mixed", seed=17),
     "two_pass_stochastic": W.WorkloadSpec("two_pass_stochastic", B=48, Hq=4, Hkv=4, D=64, H=256,
                                           V=40000, ctx=(1, 64), k=(6, 9), mode="stochastic", seed=18),
+    # R = 256 rows over a vocabulary of 3 tiles per SM: two passes, the first on
+    # CTA pairs with a single MMA N-chunk (each CTA holds 128 hidden rows).
+    "two_pass_pair_one_chunk": W.WorkloadSpec("two_pass_pair_one_chunk", B=32, Hq=8, Hkv=2, D=128, H=320,
+                                              V=40000, ctx=(4, 96), k=(7, 7), mode="mixed", seed=19),
 }
 
 
@@ -149,7 +153,8 @@ def test_accept_commit_fused_small(dev, name):
 
 def test_accept_launch_count(dev):
     """One launch while the logits stay on chip, two for the two-pass shapes."""
-    for name, want in (("gqa_mixed", 1), ("two_pass_mixed", 2), ("two_pass_stochastic", 2)):
+    for name, want in (("gqa_mixed", 1), ("two_pass_mixed", 2), ("two_pass_stochastic", 2),
+                       ("two_pass_pair_one_chunk", 2)):
         wl = W.make_workload(SMALL[name], device="cpu")
         assert spade.spade_accept_launches(wl["B"], wl["R"], wl["H"], wl["V"]) == want, name
     wl = W.make_workload(W.SPECS["ragged"], device="cpu")
