@@ -27,6 +27,13 @@
 //    masses of the distribution to sample (residual or p, float-float sums)
 //    are known, and the CTA whose slice holds the point u*Z locates its
 //    32-entry segment and scans it in vocabulary order to pick the token.
+//  * More verify rows than TMEM keeps resident: two launches.  The first keeps
+//    only the row statistics and takes the decisions; with an even grid it
+//    runs on CTA pairs (clusters of two, tcgen05 cta_group::2): one MMA of
+//    M = 256 takes A rows 0-127 from the even CTA's shared memory and
+//    128-255 from the odd one's, and splits each N-chunk's hidden rows
+//    between them, so an SM receives half the hidden bytes per k-chunk.  The
+//    second launch recomputes only the rows to sample.
 #include <cuda_bf16.h>
 
 #include <cfloat>
