@@ -73,6 +73,21 @@ def _dist():
     return ws, rank, local
 
 
+def _job_rate(tokens_local, t_local, ws, device):
+    """Whole-job rate of ws replicas: every rank's tokens over the slowest rank's time.
+
+    Returns (rate, slowest time).  With ws > 1 every rank must call it (two
+    all-reduces on the default process group).
+    """
+    if ws > 1:
+        t = torch.tensor([t_local], dtype=torch.float64, device=device)
+        n = torch.tensor([float(tokens_local)], dtype=torch.float64, device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        torch.distributed.all_reduce(n, op=torch.distributed.ReduceOp.SUM)
+        return float(n.item()) / float(t.item()), float(t.item())
+    return tokens_local / t_local, t_local
+
+
 def _work_bytes(wl):
     """Algorithmic bytes of the two dominant kernels for one step."""
     ctx = wl["ctx_lens"].long().cpu()
@@ -233,12 +248,7 @@ def run_spade(args, ws, rank, local):
     t_attn = [e[0].elapsed_time(e[1]) * 1e-3 for e in evs]
     t_acc = [e[1].elapsed_time(e[2]) * 1e-3 for e in evs]
     t_com = [e[2].elapsed_time(e[3]) * 1e-3 for e in evs]
-    total = sum(t_step)
-    if ws > 1:
-        tt = torch.tensor([total], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        total = float(tt.item())
-    value = tokens_per_step * args.steps * ws / total
+    value, total = _job_rate(tokens_per_step * args.steps, sum(t_step), ws, dev)
 
     # ---- end to end through the public API with pinned host inputs -------------
     # Every step copies its inputs from pinned host memory and reads its result
@@ -310,6 +320,9 @@ def run_spade(args, ws, rank, local):
         e_end.record(stream)
         torch.cuda.synchronize()
         t_e2e = e_start.elapsed_time(e_end) * 1e-3
+        if ws > 1:
+            torch.distributed.barrier()
+        e2e_rate, t_e2e = _job_rate(tokens_per_step * n_e2e, t_e2e, ws, dev)
         # The input copy alone (what the end-to-end rate overlaps with compute).
         c0 = torch.cuda.Event(enable_timing=True)
         c1 = torch.cuda.Event(enable_timing=True)
@@ -320,7 +333,7 @@ def run_spade(args, ws, rank, local):
             c1.record(copy_stream)
         torch.cuda.synchronize()
         t_copy = c0.elapsed_time(c1) * 1e-3 / 5
-        e2e = {"value": tokens_per_step * n_e2e * ws / t_e2e, "unit": UNIT, "h2d_bytes_per_step": h2d,
+        e2e = {"value": e2e_rate, "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "steps": n_e2e, "copies_per_step": {"h2d": 1, "d2h": 1},
                "h2d_copy_us": t_copy * 1e6, "h2d_gbs": h2d / t_copy / 1e9,
                "overlap": "inputs of step i+1 copied on a second stream while step i runs",
