@@ -246,6 +246,17 @@ const char *spade_last_error(void);
 /* Library version, e.g. "spade-gb300 0.1 sm_103a". */
 const char *spade_version(void);
 
+/*
+ * Self-test of the device-side timeout path that every kernel above uses for
+ * its waits: launches one CTA on `stream` whose thread waits on an mbarrier
+ * that nothing completes.  After limit_us microseconds of %globaltimer
+ * (1 .. 1000000) the wait gives up, SPADE_DEV_TIMEOUT is OR-ed into *status
+ * (device int32) and the kernel returns normally, so the context stays
+ * usable.  No other effect; for health checks and tests of status reporting.
+ * Returns SPADE_ERR_INVALID_ARG for a null status or a limit out of range.
+ */
+spade_status spade_selftest_wait_timeout(int32_t *status, int32_t limit_us, spade_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

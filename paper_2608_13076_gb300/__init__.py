@@ -23,7 +23,7 @@ from . import _build
 __all__ = [
     "SpadeError", "load", "build", "library_path",
     "spade_verify_attention", "spade_verify_accept", "spade_kv_commit", "spade_verify_attention_noalloc",
-    "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_accept_launches",
+    "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_accept_launches", "spade_selftest_wait_timeout",
     "attn_workspace", "accept_workspace", "status_tensor", "check_status",
     "DEV_BAD_INDEX", "DEV_CAPACITY", "DEV_TIMEOUT", "DEV_FALLBACK",
 ]
@@ -83,6 +83,8 @@ def load():
     lib.spade_accept_workspace_size.argtypes = [_i32] * 4
     lib.spade_accept_launches.restype = _i32
     lib.spade_accept_launches.argtypes = [_i32] * 4
+    lib.spade_selftest_wait_timeout.restype = _i32
+    lib.spade_selftest_wait_timeout.argtypes = [_vp, _i32, _vp]
     lib.spade_kv_commit.restype = _i32
     lib.spade_kv_commit.argtypes = [_vp] * 5 + [_i32] * 4 + [_vp, _vp]
     lib.spade_status_string.restype = ctypes.c_char_p
@@ -197,6 +199,12 @@ def spade_verify_attention_noalloc(q, k_cache, v_cache, ctx_lens, n_draft, cu_q,
 # ---------------------------------------------------------------------------
 def spade_accept_workspace_size(B, R, H, V):
     return int(load().spade_accept_workspace_size(B, R, H, V))
+
+
+def spade_selftest_wait_timeout(status, limit_us, stream=None):
+    """One bounded wait that nothing completes: SPADE_DEV_TIMEOUT lands in `status` after limit_us."""
+    _need(status, "status", torch.int32, 1)
+    _check_rc(load().spade_selftest_wait_timeout(_ptr(status), int(limit_us), _stream(stream)))
 
 
 def spade_accept_launches(B, R, H, V):

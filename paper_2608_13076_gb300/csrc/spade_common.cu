@@ -5,6 +5,7 @@
 #include <mutex>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace spade {
 
@@ -127,9 +128,37 @@ bool encode_tmap_rows_by_slab(CUtensorMap *map, const void *base, uint64_t rows,
   return true;
 }
 
+// One thread waits on an mbarrier that nothing completes, bounded as every
+// kernel's waits are, and reports the expiry in the status word.
+__global__ void selftest_wait_kernel(int32_t *status, uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    const uint64_t t0 = globaltimer();
+    bool done = mbar_try_wait(&bar, 0);
+    while (!done && globaltimer() - t0 <= limit_ns) done = mbar_try_wait(&bar, 0);
+    if (!done) atomicOr(status, SPADE_DEV_TIMEOUT);
+  }
+}
+
 }  // namespace spade
 
 extern "C" {
+
+spade_status spade_selftest_wait_timeout(int32_t *status, int32_t limit_us, spade_stream_t stream) {
+  using namespace spade;
+  if (!status) return fail(SPADE_ERR_INVALID_ARG, "spade_selftest_wait_timeout: null status");
+  if (limit_us < 1 || limit_us > 1000000)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_selftest_wait_timeout: limit %d us out of [1, 1000000]", limit_us);
+  spade_status st = device_info(nullptr, nullptr);
+  if (st != SPADE_OK) return st;
+  selftest_wait_kernel<<<1, 32, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      status, static_cast<uint64_t>(limit_us) * 1000u);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "selftest launch");
+  return SPADE_OK;
+}
 
 const char *spade_status_string(spade_status s) {
   switch (s) {

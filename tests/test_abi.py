@@ -71,6 +71,13 @@ def test_null_arguments_rejected_before_any_device_work(lib):
     assert rc == 1
 
 
+def test_selftest_rejects_bad_arguments_before_device_work(lib):
+    assert lib.spade_selftest_wait_timeout(None, 1000, None) == 1
+    p = ctypes.c_void_p(16)
+    assert lib.spade_selftest_wait_timeout(p, 0, None) == 1
+    assert lib.spade_selftest_wait_timeout(p, 2000000, None) == 1
+
+
 def test_launch_count_rejects_invalid_sizes(lib):
     # Validation precedes the device query, so these need no GPU.
     assert lib.spade_accept_launches(0, 5, 512, 1024) == 0

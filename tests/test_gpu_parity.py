@@ -151,6 +151,21 @@ def test_accept_commit_fused_small(dev, name):
     assert torch.equal(kc2, kc) and torch.equal(vc2, vc)
 
 
+def test_bounded_wait_reports_timeout_and_context_survives(dev):
+    """A device wait that nothing completes gives up after its limit and sets the status bit;
+    the context stays usable (the next verify call runs and passes)."""
+    st = spade.status_tensor(dev)
+    spade.spade_selftest_wait_timeout(st, 20000)  # 20 ms
+    torch.cuda.synchronize()
+    assert int(st.item()) & spade.DEV_TIMEOUT
+    wl = W.make_workload(SMALL["gqa_mixed"], device=dev)
+    out, lse, st2 = parity.gpu_attention(wl)
+    torch.cuda.synchronize()
+    assert int(st2.item()) == 0
+    n, bad, worst = parity.compare_attention(out, parity.oracle_attention(wl)[0])
+    assert bad == 0
+
+
 def test_accept_launch_count(dev):
     """One launch while the logits stay on chip, two for the two-pass shapes."""
     for name, want in (("gqa_mixed", 1), ("two_pass_mixed", 2), ("two_pass_stochastic", 2),
