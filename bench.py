@@ -374,7 +374,7 @@ def run_spade(args, ws, rank, local):
                "traffic": _traffic("verify_accept_kernel", args.workload),
                "algorithmic_bytes": lm_bytes, "peak_source": peak_src,
                "tensor_tflops": lm_flop / m_acc / 1e12, "tensor_frac_of_bf16_peak": lm_flop / m_acc / 1e12 / bf16}
-    attn_kernel = "verify_attention_tc_kernel" if wl["D"] == 128 else "verify_attention_kernel"
+    attn_kernel = "verify_attention_tc_kernel"
     roof_attn = {"kernel": attn_kernel, "bound": "hbm", "achieved": attn_bytes / m_attn / 1e9,
                  "peak": hbm, "unit": "GB/s", "frac": attn_bytes / m_attn / 1e9 / hbm,
                  "traffic": _traffic(attn_kernel, args.workload),

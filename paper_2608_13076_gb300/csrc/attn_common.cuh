@@ -1,8 +1,8 @@
-// attn_common.cuh -- pieces shared by the two verify-attention kernels (the
-// tensor-memory kernel for head dim 128 and the warp-MMA kernel for head dim
-// 64): parameters, the stream-K schedule over key chunks, and the
-// log-sum-exp merge of split partials (Sec. III-B "Verification Stage": the
-// verifier's attention of the k+1 draft positions against the cached context).
+// attn_common.cuh -- pieces of the verify-attention kernel (tensor memory,
+// head dims 64 and 128) shared with its host entry points: parameters, the
+// stream-K schedule over key chunks, and the log-sum-exp merge of split
+// partials (Sec. III-B "Verification Stage": the verifier's attention of the
+// k+1 draft positions against the cached context).
 #pragma once
 #include <cuda_bf16.h>
 
@@ -15,7 +15,7 @@
 namespace spade {
 namespace attn {
 
-constexpr int kChunk = 64;     // keys per schedule slice (and per warp-MMA stage)
+constexpr int kChunk = 64;     // keys per schedule slice (two per MMA chunk)
 constexpr int kRowBlock = 64;  // query rows per work unit
 constexpr int kMaxB = 512;     // sequences per call (per-CTA schedule lives in smem)
 constexpr int kUnitCostTc = 11; // virtual slices per unit in the tensor-memory kernel's schedule
@@ -259,11 +259,11 @@ __device__ __forceinline__ bool arrive_part(int32_t *counter, int nparts) {
   return old == nparts - 1;
 }
 
-// Tensor-memory kernel for head dim 128 (verify_attention_tc.cu).  The four
-// tensor maps view the K and V caches as [rows][64] slabs: `k2`/`v2` fetch
-// 128 keys x both slabs per box, `k1`/`v1` 64 keys x one slab.
+// Tensor-memory kernel for head dims 64 and 128 (verify_attention_tc.cu).  The
+// four tensor maps view the K and V caches as [rows][64] slabs: `k2`/`v2`
+// fetch 128 keys x every slab per box, `k1`/`v1` 64 keys x one slab.
 cudaError_t launch_tc(const Params &p, const CUtensorMap &k2, const CUtensorMap &v2,
-                      const CUtensorMap &k1, const CUtensorMap &v1, int nr, cudaStream_t stream);
+                      const CUtensorMap &k1, const CUtensorMap &v1, int nr, int d, cudaStream_t stream);
 
 }  // namespace attn
 }  // namespace spade

@@ -1,5 +1,5 @@
-// ptx.cuh -- thin inline-PTX wrappers for sm_103a: mbarrier, TMA, ldmatrix,
-// mma.sync, tcgen05 (TMEM allocation, MMA, loads/stores, fences).
+// ptx.cuh -- thin inline-PTX wrappers for sm_103a: mbarrier, TMA, bulk copies,
+// cluster addressing, tcgen05 (TMEM allocation, MMA, loads/stores, fences).
 #pragma once
 #include <cstdint>
 #include <cuda.h>
@@ -132,27 +132,6 @@ SPADE_DEVICE void tma_load_3d(void *dst, const CUtensorMap *map, int32_t x, int3
       : "memory");
 }
 
-// ---------------------------------------------------------------- warp MMA
-SPADE_DEVICE void ldmatrix_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
-                              uint32_t &r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-SPADE_DEVICE void ldmatrix_x4_trans(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
-                                    uint32_t &r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-// D[16x8] += A[16x16] * B[16x8], bf16 inputs, fp32 accumulators.
-SPADE_DEVICE void mma_bf16_16816(float *d, const uint32_t *a, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
-      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
 SPADE_DEVICE uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t *>(&v);

@@ -1,9 +1,8 @@
-// verify_attention_tc.cu -- verify attention for head dim 128 on the
+// verify_attention_tc.cu -- verify attention for head dims 64 and 128 on the
 // fifth-generation tensor cores (tcgen05 MMAs with accumulators in tensor
-// memory).  It computes the same thing as the warp-MMA kernel: the attention
-// of the k_b+1 verify positions of every sequence against its cached keys and
-// values, causal inside the draft block (Sec. III-B "Verification Stage",
-// Algorithm 1 cloud step).
+// memory): the attention of the k_b+1 verify positions of every sequence
+// against its cached keys and values, causal inside the draft block
+// (Sec. III-B "Verification Stage", Algorithm 1 cloud step).
 //
 // Design (GB300):
 //  * Keys on the MMA M side.  A unit (sequence, KV head, <= 64 query rows) has
@@ -13,9 +12,10 @@
 //    scores for every row, and the softmax work spreads over all 128 lanes
 //    whatever the row count.  The output is accumulated transposed too:
 //    O^T[d][row] += V^T P^T with M = 128 (head dim), both operands read from
-//    shared memory in MN-major form straight from the TMA tiles.
-//  * Warp roles: warp 0 streams K and V tiles (TMA, 128 keys x 128 dims per
-//    box) into a two-stage ring; warp 1 issues the MMAs (one elected thread)
+//    shared memory in MN-major form straight from the TMA tiles.  Head dim 64
+//    keeps M = 128 with a V tile whose second 64-dim slab stays zero.
+//  * Warp roles: warp 0 streams K and V tiles (TMA, 128 keys x all head dims
+//    per box) into a two-stage ring; warp 1 issues the MMAs (one elected thread)
 //    and owns the tensor-memory allocation; warps 2-9 run the softmax and the
 //    epilogue, two per tensor-memory lane quadrant, each on half of the rows.
 //    The next unit's Q is prefetched (cp.async) into a second buffer while
@@ -25,8 +25,8 @@
 //    <= 256 and the O^T columns in tensor memory are rescaled only then.  Row
 //    maxima and per-key-lane row sums live in registers; the sums are reduced
 //    across lanes once per unit.
-//  * The same stream-K split over 64-key slices as the warp-MMA kernel, with
-//    the same partials and log-sum-exp merge.  Keys beyond the live cache (or
+//  * Stream-K split over 64-key slices (attn_common.cuh) with fp32 partials
+//    and a log-sum-exp merge of split units.  Keys beyond the live cache (or
 //    not loaded) get P = 0 and their V rows are zeroed in shared memory, so
 //    whatever the unused cache slots hold cannot reach the result.
 #include "attn_common.cuh"
@@ -35,7 +35,7 @@ namespace spade {
 namespace attn {
 namespace tc {
 
-constexpr int kD = 128;
+constexpr int kDMax = 128;                       // head dims the shared-memory tiles hold
 constexpr int kKeys = 128;                       // keys per MMA chunk (two slices)
 constexpr int kStages = 2;                       // K/V ring depth (chunks)
 constexpr int kSoftWarps = 8;                    // softmax / epilogue warps
@@ -170,7 +170,10 @@ __device__ __forceinline__ SegInfo next_seg(const Sched &sc, int64_t x, int64_t 
   return s;
 }
 
-template <int NR>
+// D: head dim, 64 or 128.  With D = 64 the K and V tiles hold one 64-dim slab
+// and the V tiles' second slab stays zero, so O^T keeps M = 128 (its rows
+// 64-127 are zero and never stored).
+template <int NR, int D>
 __global__ void __launch_bounds__(kThreads, 1)
     verify_attention_tc_kernel(const __grid_constant__ Params p,
                                const __grid_constant__ CUtensorMap tm_k2,
@@ -178,6 +181,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                                const __grid_constant__ CUtensorMap tm_k1,
                                const __grid_constant__ CUtensorMap tm_v1) {
   static_assert(NR % 16 == 0 && NR >= 16 && NR <= kRowBlock, "MMA N must be 16..64, step 16");
+  static_assert(D == 64 || D == kDMax, "head dim 64 or 128");
+  constexpr int kD = D;
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte aligned base, derived by pointer arithmetic so that the compiler
   // keeps the shared state space (plain ld/st.shared, not generic accesses).
@@ -203,6 +208,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane < 2) {
     tma_prefetch_desc(lane ? &tm_v2 : &tm_k2);
     tma_prefetch_desc(lane ? &tm_v1 : &tm_k1);
+  }
+  if constexpr (kD == 64) {
+    // The V tiles' second 64-dim slab: zeros for the whole launch (the copies
+    // fill the first slab only).
+    for (int e = tid; e < kStages * (kSlab / 16); e += kThreads) {
+      const int st = e / (kSlab / 16), o = e % (kSlab / 16);
+      *reinterpret_cast<uint4 *>(smem + Smem::V + st * kTile + kSlab + o * 16) = make_uint4(0, 0, 0, 0);
+    }
+    fence_proxy_async_smem();
   }
   sched_validate(p, s_ctx, s_kd, tid, kThreads);
   block_sync();
@@ -292,12 +306,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint8_t *tile = ring + st * kTile;
           if (!mbar_wait(&bars[bar_empty + st], ph ^ 1, s_abort)) expired = true;
           if (*s_abort) continue;
-          mbar_arrive_expect_tx(&bars[bar_full + st], nsl * kSlab);
+          mbar_arrive_expect_tx(&bars[bar_full + st], nsl * (kSlab / kDMax) * kD);
           if (nsl == 2) {
             tma_load_3d(tile, tm2, 0, key_row, 0, &bars[bar_full + st], pol);
           } else {
             tma_load_3d(tile, tm1, 0, key_row, 0, &bars[bar_full + st], pol);
-            tma_load_3d(tile + kSlab, tm1, 0, key_row, 1, &bars[bar_full + st], pol);
+            if constexpr (kD == kDMax) tma_load_3d(tile + kSlab, tm1, 0, key_row, 1, &bars[bar_full + st], pol);
           }
           issued = it + 1;
         }
@@ -621,7 +635,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int e = 0; e < 8; ++e) {
             // l >= 1 (the row maximum's own term), so the fast divide is exact
             // to a few fp32 ulps, far below the bf16 rounding that follows.
-            if (j * 8 + e < hi)
+            if (j * 8 + e < hi && t < kD)
               p.out[orow * kD + t] = __float2bfloat16_rn(__fdividef(__uint_as_float(o8[e]), l[j * 8 + e]));
             if (++gh == p.G) {
               gh = 0;
@@ -644,7 +658,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_wait_ld();
 #pragma unroll
           for (int e = 0; e < 8; ++e)
-            if (j * 8 + e < hi) __stcg(part + (c0 + j * 8 + e) * kD + t, __uint_as_float(o8[e]));
+            if (j * 8 + e < hi && t < kD) __stcg(part + (c0 + j * 8 + e) * kD + t, __uint_as_float(o8[e]));
         }
         tc_fence_before();
         if (row_writer) {
@@ -677,10 +691,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int NR>
+template <int NR, int D>
 static cudaError_t launch_nr(const Params &p, const CUtensorMap &k2, const CUtensorMap &v2,
                              const CUtensorMap &k1, const CUtensorMap &v1, cudaStream_t stream) {
-  auto kern = verify_attention_tc_kernel<NR>;
+  auto kern = verify_attention_tc_kernel<NR, D>;
   static bool configured = false;  // per template instance; the attribute is per function
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem::BYTES);
@@ -694,12 +708,20 @@ static cudaError_t launch_nr(const Params &p, const CUtensorMap &k2, const CUten
 }  // namespace tc
 
 cudaError_t launch_tc(const Params &p, const CUtensorMap &k2, const CUtensorMap &v2,
-                      const CUtensorMap &k1, const CUtensorMap &v1, int nr, cudaStream_t stream) {
+                      const CUtensorMap &k1, const CUtensorMap &v1, int nr, int d, cudaStream_t stream) {
+  if (d == 64) {
+    switch (nr) {
+      case 16: return tc::launch_nr<16, 64>(p, k2, v2, k1, v1, stream);
+      case 32: return tc::launch_nr<32, 64>(p, k2, v2, k1, v1, stream);
+      case 48: return tc::launch_nr<48, 64>(p, k2, v2, k1, v1, stream);
+      default: return tc::launch_nr<64, 64>(p, k2, v2, k1, v1, stream);
+    }
+  }
   switch (nr) {
-    case 16: return tc::launch_nr<16>(p, k2, v2, k1, v1, stream);
-    case 32: return tc::launch_nr<32>(p, k2, v2, k1, v1, stream);
-    case 48: return tc::launch_nr<48>(p, k2, v2, k1, v1, stream);
-    default: return tc::launch_nr<64>(p, k2, v2, k1, v1, stream);
+    case 16: return tc::launch_nr<16, 128>(p, k2, v2, k1, v1, stream);
+    case 32: return tc::launch_nr<32, 128>(p, k2, v2, k1, v1, stream);
+    case 48: return tc::launch_nr<48, 128>(p, k2, v2, k1, v1, stream);
+    default: return tc::launch_nr<64, 128>(p, k2, v2, k1, v1, stream);
   }
 }
 
