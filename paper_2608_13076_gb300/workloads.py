@@ -104,25 +104,29 @@ def _mean_overlap(logits, noise, sigma):
 def make_workload(spec: WorkloadSpec, device="cpu", cache_pad: int = 0):
     """Draw all inputs of one verify step.
 
+    Every tensor is drawn on the CPU from one seeded generator and only then
+    moved to ``device``, so a seed names the same inputs on every device (the
+    GPU path, the float64 oracle and the CPU baseline all see identical data).
+
     Returns a dict of tensors on ``device``:
       q [R,Hq,D] bf16, k_cache/v_cache [B,Hkv,cap,D] bf16 (slots [0, ctx+k] filled,
       the rest zero), ctx_lens/n_draft [B] i32, cu_q [B+1] i32, hidden [R,H] bf16,
       w_lm [V,H] bf16, draft_tokens [R-B] i32, draft_probs [R-B,V] f32 or None,
       uniforms [R] f32 in [0,1), mode [B] i32, plus python ints B, R, cap, ...
     """
-    gen_cpu = torch.Generator(device="cpu").manual_seed(spec.seed)
+    gen = torch.Generator(device="cpu").manual_seed(spec.seed)
     dev = torch.device(device)
-    gen = gen_cpu if dev.type == "cpu" else torch.Generator(device=dev).manual_seed(spec.seed)
+    cpu = torch.device("cpu")
 
     B = spec.B
     if spec.ctx[0] == spec.ctx[1]:
         ctx = torch.full((B,), spec.ctx[0], dtype=torch.int32)
     else:
-        ctx = torch.randint(spec.ctx[0], spec.ctx[1] + 1, (B,), generator=gen_cpu, dtype=torch.int32)
+        ctx = torch.randint(spec.ctx[0], spec.ctx[1] + 1, (B,), generator=gen, dtype=torch.int32)
     if spec.k[0] == spec.k[1]:
         kd = torch.full((B,), spec.k[0], dtype=torch.int32)
     else:
-        kd = torch.randint(spec.k[0], spec.k[1] + 1, (B,), generator=gen_cpu, dtype=torch.int32)
+        kd = torch.randint(spec.k[0], spec.k[1] + 1, (B,), generator=gen, dtype=torch.int32)
     if spec.mode == "greedy":
         mode = torch.zeros(B, dtype=torch.int32)
     elif spec.mode == "stochastic":
@@ -136,15 +140,15 @@ def make_workload(spec: WorkloadSpec, device="cpu", cache_pad: int = 0):
     n_draft_rows = R - B
     cap = int((ctx + kd + 1).max()) + cache_pad
 
-    q = _bf16_normal(gen, (R, spec.Hq, spec.D), 1.0, dev)
-    k_cache = torch.zeros((B, spec.Hkv, cap, spec.D), dtype=torch.bfloat16, device=dev)
+    q = _bf16_normal(gen, (R, spec.Hq, spec.D), 1.0, cpu)
+    k_cache = torch.zeros((B, spec.Hkv, cap, spec.D), dtype=torch.bfloat16)
     v_cache = torch.zeros_like(k_cache)
     for b in range(B):
         L = int(ctx[b] + kd[b] + 1)
-        k_cache[b, :, :L] = _bf16_normal(gen, (spec.Hkv, L, spec.D), 1.0, dev)
-        v_cache[b, :, :L] = _bf16_normal(gen, (spec.Hkv, L, spec.D), 1.0, dev)
-    hidden = _bf16_normal(gen, (R, spec.H), 1.0, dev)
-    w_lm = _bf16_normal(gen, (spec.V, spec.H), 1.0 / math.sqrt(spec.H), dev)
+        k_cache[b, :, :L] = _bf16_normal(gen, (spec.Hkv, L, spec.D), 1.0, cpu)
+        v_cache[b, :, :L] = _bf16_normal(gen, (spec.Hkv, L, spec.D), 1.0, cpu)
+    hidden = _bf16_normal(gen, (R, spec.H), 1.0, cpu)
+    w_lm = _bf16_normal(gen, (spec.V, spec.H), 1.0 / math.sqrt(spec.H), cpu)
 
     # Draft rows: row cu_q[b]+i (i < k_b) holds draft i of sequence b.
     draft_row_of = []
@@ -154,13 +158,13 @@ def make_workload(spec: WorkloadSpec, device="cpu", cache_pad: int = 0):
     draft_row_of = torch.tensor(draft_row_of, dtype=torch.long)
     seq_of_draft = torch.repeat_interleave(torch.arange(B), kd.long())
 
-    logits = _verifier_logits_f32(hidden[draft_row_of.to(dev)], w_lm) if n_draft_rows else \
-        torch.zeros((0, spec.V), device=dev)
-    noise = torch.randn(logits.shape, generator=gen, dtype=torch.float32, device=dev)
+    logits = _verifier_logits_f32(hidden[draft_row_of], w_lm) if n_draft_rows else \
+        torch.zeros((0, spec.V))
+    noise = torch.randn(logits.shape, generator=gen, dtype=torch.float32)
     sigma = spec.noise
     if spec.target_accept > 0 and (mode == STOCHASTIC).any():
         lo, hi = 0.0, 20.0
-        for _ in range(30):
+        for _ in range(24):
             mid = 0.5 * (lo + hi)
             if _mean_overlap(logits, noise, mid) > spec.target_accept:
                 lo = mid
@@ -171,28 +175,31 @@ def make_workload(spec: WorkloadSpec, device="cpu", cache_pad: int = 0):
     q_dist = torch.softmax(draft_logits, dim=-1)
 
     stoch_draft = mode[seq_of_draft] == STOCHASTIC
-    drafts = torch.empty(n_draft_rows, dtype=torch.int64, device=dev)
+    drafts = torch.empty(n_draft_rows, dtype=torch.int64)
     if stoch_draft.any():
-        idx = stoch_draft.nonzero().flatten().to(dev)
+        idx = stoch_draft.nonzero().flatten()
         drafts[idx] = torch.multinomial(q_dist[idx], 1, generator=gen).flatten()
     if (~stoch_draft).any():
-        idx = (~stoch_draft).nonzero().flatten().to(dev)
+        idx = (~stoch_draft).nonzero().flatten()
         if spec.greedy_draft == "noisy_argmax":
             drafts[idx] = draft_logits[idx].argmax(-1)
         else:
             am = logits[idx].argmax(-1)
-            rnd = torch.randint(0, spec.V, (idx.numel(),), generator=gen, device=dev)
-            hit = torch.rand(idx.numel(), generator=gen, device=dev) < spec.match_prob
+            rnd = torch.randint(0, spec.V, (idx.numel(),), generator=gen)
+            hit = torch.rand(idx.numel(), generator=gen) < spec.match_prob
             drafts[idx] = torch.where(hit, am, rnd)
 
-    uniforms = torch.rand(R, generator=gen, dtype=torch.float32, device=dev)
+    uniforms = torch.rand(R, generator=gen, dtype=torch.float32)
     draft_probs = q_dist.contiguous() if bool((mode == STOCHASTIC).any()) else None
+
+    def mv(t):
+        return None if t is None else t.to(dev)
 
     return dict(
         spec=spec, B=B, R=R, cap=cap, Hq=spec.Hq, Hkv=spec.Hkv, D=spec.D, H=spec.H, V=spec.V,
-        q=q, k_cache=k_cache, v_cache=v_cache,
-        ctx_lens=ctx.to(dev), n_draft=kd.to(dev), cu_q=cu_q.to(dev),
-        hidden=hidden, w_lm=w_lm,
-        draft_tokens=drafts.to(torch.int32), draft_probs=draft_probs,
-        uniforms=uniforms, mode=mode.to(dev), sigma=sigma,
+        q=mv(q), k_cache=mv(k_cache), v_cache=mv(v_cache),
+        ctx_lens=mv(ctx), n_draft=mv(kd), cu_q=mv(cu_q),
+        hidden=mv(hidden), w_lm=mv(w_lm),
+        draft_tokens=mv(drafts.to(torch.int32)), draft_probs=mv(draft_probs),
+        uniforms=mv(uniforms), mode=mv(mode), sigma=sigma,
     )

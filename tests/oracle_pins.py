@@ -171,6 +171,36 @@ def check_acceptance_worked_examples(o):
     assert res["accepted_len"][0] == 0 and res["next_token"][0] == ga["argmax"]
 
 
+def check_margin_worked_examples(o):
+    """Flags of the parity rule on hand-derived cases: greedy top-2 gap and stochastic
+    |u - p/q| below 1e-3 at a deciding position, the sampled token's edge margin, and
+    no flag from rows after the first rejection."""
+    g = _golden()["decision_margins"]
+    thr = g["threshold"]
+    for ex in g["greedy"]:
+        k = ex["k"]
+        res = o.verify_accept(np.asarray(ex["logits"]), ex["draft"], None, np.full(k + 1, 0.5), [0],
+                              [0, k + 1], [k], margin=thr)
+        assert res["accepted_len"][0] == ex["accepted"], ex["about"]
+        assert res["next_token"][0] == ex["next"], ex["about"]
+        assert bool(res["flag_decision"][0]) == ex["flag_decision"], ex["about"]
+        assert not res["flag_sample"][0], ex["about"]
+    for ex in g["stochastic"]:
+        k = ex["k"]
+        q = np.asarray(ex["q"]).reshape(k, -1) if k else np.zeros((0, len(ex["p"][0])))
+        res = o.verify_accept(np.log(np.asarray(ex["p"])), ex["draft"], q, ex["u"], [1], [0, k + 1], [k],
+                              margin=thr)
+        assert res["accepted_len"][0] == ex["accepted"], ex["about"]
+        assert res["next_token"][0] == ex["next"], ex["about"]
+        assert bool(res["flag_decision"][0]) == ex["flag_decision"], ex["about"]
+        assert bool(res["flag_sample"][0]) == ex["flag_sample"], ex["about"]
+    for ex in g["sampling_margin"]["cases"]:
+        r = np.asarray(ex["r"])
+        x, m = o.inverse_cdf(r, r.sum(), ex["u"])
+        assert x == ex["x"], ex["why"]
+        assert abs(m - ex["margin"]) < 1e-9, (ex["why"], m)
+
+
 def check_residual_properties(o, seed=4):
     rng = np.random.default_rng(seed)
     for _ in range(50):
@@ -346,7 +376,7 @@ def check_kv_commit(o, seed=9):
 ALL_CHECKS = [
     check_attention_worked_examples, check_attention_vs_sdpa, check_attention_special_cases,
     check_attention_gqa_mapping, check_logits_one_hot, check_acceptance_worked_examples,
-    check_residual_properties, check_q_equals_p_accepts_all, check_strict_comparison,
+    check_margin_worked_examples, check_residual_properties, check_q_equals_p_accepts_all, check_strict_comparison,
     check_stochastic_output_law, check_progress_and_bounds, check_greedy_identity,
     check_kv_commit,
 ]

@@ -31,6 +31,21 @@ MUTANTS = {
                       "e = np.exp(2.0 * (l - l.max(axis=-1, keepdims=True)))"),
     "greedy_uses_draft_row_shift": ("l = _f64(logits[r0 + i])", "l = _f64(logits[r0 + i + 1])"),
     "uniform_of_wrong_row": ("u = float(uniforms[r0 + i])", "u = float(uniforms[r0 + k])"),
+    # Mistakes in the margins and flags that decide which GPU mismatches are excused.
+    "top2_margin_always_inf": ("return float(top[1] - top[0])", "return float('inf')"),
+    "top2_margin_always_zero": ("return float(top[1] - top[0])", "return 0.0"),
+    "sample_margin_over_Z": ("margin = min(T - lo, c[x] - T) / r[x] if r[x] > 0 else 0.0",
+                             "margin = min(T - lo, c[x] - T) / Z if r[x] > 0 else 0.0"),
+    "sample_margin_always_zero": ("margin = min(T - lo, c[x] - T) / r[x] if r[x] > 0 else 0.0",
+                                  "margin = 0.0"),
+    "flag_every_sequence": ("flag_dec = np.zeros(B, dtype=bool)", "flag_dec = np.ones(B, dtype=bool)"),
+    "flag_every_sample": ("flag_smp = np.zeros(B, dtype=bool)", "flag_smp = np.ones(B, dtype=bool)"),
+    "greedy_draft_rows_never_flag": ("                if _top2_margin(l) < margin:",
+                                     "                if _top2_margin(l) < 0.0:"),
+    "stochastic_never_flags": ("if abs(u - ratio) < margin:", "if abs(u - ratio) < 0.0:"),
+    "flag_rows_after_rejection": ("            if not ok:\n                break",
+                                  "            if not ok:\n                flag_dec[b] |= any(abs(float(uniforms[r0 + j]) - 0.5) "
+                                  "< margin for j in range(i + 1, k))\n                break"),
 }
 
 
