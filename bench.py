@@ -11,8 +11,9 @@ in and the step's result read back inside the timed region.
 
 Default workload: the Llama-3-8B-shaped verifier step (batch 8, GQA 32/8,
 head_dim 128, hidden 4096, vocab 128256, ctx 4096, k = 8, stochastic), the
-paper's own verifier shape.  `--impl reference` times the float64 CPU oracle
-on the same workload instead (bounded samples: one sequence per step).
+paper's own verifier shape; the other workloads of the suite are timed on the
+device after it (`per_workload`).  `--impl reference` times the float64 CPU
+oracle on the same workload instead (bounded samples: one sequence per step).
 """
 from __future__ import annotations
 
@@ -86,6 +87,41 @@ def _job_rate(tokens_local, t_local, ws, device):
         torch.distributed.all_reduce(n, op=torch.distributed.ReduceOp.SUM)
         return float(n.item()) / float(t.item()), float(t.item())
     return tokens_local / t_local, t_local
+
+
+def _to_device(wl, dev):
+    return {k: (v.to(dev) if isinstance(v, torch.Tensor) else v) for k, v in wl.items()}
+
+
+def _config(spec, wl, ws):
+    """The workload's config block, identical for both arms of the benchmark."""
+    attn_bytes, lm_bytes, _, _, _ = _work_bytes(wl)
+    work_set = attn_bytes + lm_bytes
+    return {"workload": spec.name, "B": wl["B"], "Hq": wl["Hq"], "Hkv": wl["Hkv"], "D": wl["D"],
+            "H": wl["H"], "V": wl["V"], "ctx": list(spec.ctx), "k": list(spec.k), "mode": spec.mode,
+            "rows": wl["R"], "parallelism": "replicas" if ws > 1 else "single",
+            "l2": ("flushed between steps" if work_set < 2 * L2_BYTES
+                   else f"working set {work_set / 1e9:.2f} GB > L2")}
+
+
+def _lm_roofline(lm_bytes, lm_flop, t, hbm, bf16_sus, bf16_burst, peak_src):
+    """Roofline of the LM-head kernel timed inside a step: the bound is whichever of its
+    HBM bytes and its bf16 flops takes longer at peak (sustained bf16 for a kernel in a
+    long step); the fraction is taken against that bound's peak."""
+    t_hbm = lm_bytes / (hbm * 1e9)
+    t_tc = lm_flop / (bf16_sus * 1e12)
+    tensor = {"tflops": lm_flop / t / 1e12, "frac_of_sustained": lm_flop / t / 1e12 / bf16_sus,
+              "frac_of_burst": lm_flop / t / 1e12 / bf16_burst,
+              "ceiling_frac_of_sustained": min(1.0, t_tc / t_hbm) if t_hbm > 0 else 1.0}
+    if t_tc > t_hbm:
+        r = {"bound": "tensor", "achieved": lm_flop / t / 1e12, "peak": bf16_sus, "unit": "TFLOP/s",
+             "frac": lm_flop / t / 1e12 / bf16_sus, "peak_kind": "bf16_tflops_sustained"}
+    else:
+        r = {"bound": "hbm", "achieved": lm_bytes / t / 1e9, "peak": hbm, "unit": "GB/s",
+             "frac": lm_bytes / t / 1e9 / hbm, "peak_kind": "hbm_gbs"}
+    r.update({"algorithmic_bytes": lm_bytes, "algorithmic_flop": lm_flop, "peak_source": peak_src,
+              "tensor": tensor})
+    return r
 
 
 def _work_bytes(wl):
@@ -176,7 +212,10 @@ def run_spade(args, ws, rank, local):
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     spec = W.SPECS[args.workload]
-    wl = W.make_workload(spec, device=dev)
+    # Inputs are drawn on the CPU (a seed names the same data on every device);
+    # the CPU copy stays untouched for the oracle, the GPU copy is stepped.
+    wl_cpu = W.make_workload(spec, device="cpu")
+    wl = _to_device(wl_cpu, dev)
     B, R = wl["B"], wl["R"]
     max_k = int(wl["n_draft"].max())
     out = torch.empty_like(wl["q"])
@@ -369,11 +408,9 @@ def run_spade(args, ws, rank, local):
     hbm, bf16, bf16_sus, peak_src = _peaks()
     m_acc = statistics.mean(t_acc)
     m_attn = statistics.mean(t_attn)
-    roof_lm = {"kernel": "verify_accept_kernel", "bound": "hbm", "achieved": lm_bytes / m_acc / 1e9,
-               "peak": hbm, "unit": "GB/s", "frac": lm_bytes / m_acc / 1e9 / hbm,
-               "traffic": _traffic("verify_accept_kernel", args.workload),
-               "algorithmic_bytes": lm_bytes, "peak_source": peak_src,
-               "tensor_tflops": lm_flop / m_acc / 1e12, "tensor_frac_of_bf16_peak": lm_flop / m_acc / 1e12 / bf16}
+    roof_lm = {"kernel": "verify_accept_kernel"}
+    roof_lm.update(_lm_roofline(lm_bytes, lm_flop, m_acc, hbm, bf16_sus, bf16, peak_src))
+    roof_lm["traffic"] = _traffic("verify_accept_kernel", args.workload)
     attn_kernel = "verify_attention_tc_kernel"
     roof_attn = {"kernel": attn_kernel, "bound": "hbm", "achieved": attn_bytes / m_attn / 1e9,
                  "peak": hbm, "unit": "GB/s", "frac": attn_bytes / m_attn / 1e9 / hbm,
@@ -385,10 +422,7 @@ def run_spade(args, ws, rank, local):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total / args.steps * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": args.workload, "B": B, "Hq": wl["Hq"], "Hkv": wl["Hkv"], "D": wl["D"],
-                   "H": wl["H"], "V": wl["V"], "ctx": list(spec.ctx), "k": list(spec.k), "mode": spec.mode,
-                   "rows": R, "parallelism": "replicas" if ws > 1 else "single",
-                   "l2": "flushed between steps" if flush else f"working set {work_set / 1e9:.2f} GB > L2"},
+        "config": _config(spec, wl_cpu, ws),
         "tokens_per_step": tokens_per_step,
         "accepted_len": acc.tolist(),
         "kernels_us": ({"verify_attention": m_attn * 1e6, "verify_accept": m_acc * 1e6,
@@ -401,40 +435,113 @@ def run_spade(args, ws, rank, local):
     }
     if pass1 is not None:
         line["lm_head_pass1"] = {"us": pass1 * 1e6, "tensor_tflops": lm_flop / pass1 / 1e12,
-                                 "tensor_frac_of_bf16_peak": lm_flop / pass1 / 1e12 / bf16, "peak_source": peak_src,
+                                 "frac_of_sustained_bf16": lm_flop / pass1 / 1e12 / bf16_sus,
+                                 "frac_of_burst_bf16": lm_flop / pass1 / 1e12 / bf16, "peak_source": peak_src,
                                  "how": "accept call with every sequence greedy (the sampling pass exits at once)"}
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl)
+        base, par = cpu_baseline(wl_cpu, acc.cpu(), tok.cpu())
+        line["cpu_baseline"] = base
+        line["parity"] = par
+    if rank == 0 and ws == 1 and not args.no_per_workload:
+        line["per_workload"] = per_workload(args, dev, skip=args.workload)
     return line
 
 
 # ---------------------------------------------------------------------------
-def _oracle_one_sequence(wl_cpu, b):
-    """Runs the oracle's verify step (attention + LM head + accept + commit) on sequence b."""
-    import oracle.spade_oracle as O
+def _time_step(wl, dev, steps, warmup):
+    """Device time of the step (attention, then accept + commit) on one workload."""
+    import paper_2608_13076_gb300 as spade
 
-    def npf(t):
-        return None if t is None else (t.float().numpy() if t.dtype == torch.bfloat16 else t.numpy())
+    B, R = wl["B"], wl["R"]
+    max_k = int(wl["n_draft"].max())
+    out = torch.empty_like(wl["q"])
+    acc = torch.zeros(B, dtype=torch.int32, device=dev)
+    tok = torch.zeros(B, dtype=torch.int32, device=dev)
+    status = spade.status_tensor(dev)
+    ws_attn = spade.attn_workspace(B, wl["Hq"], wl["Hkv"], wl["D"], wl["cap"], max_k, device=dev)
+    ws_acc = spade.accept_workspace(B, R, wl["H"], wl["V"], device=dev)
+    ctx0 = wl["ctx_lens"].clone()
+    attn_bytes, lm_bytes, lm_flop, _, _ = _work_bytes(wl)
+    flush = attn_bytes + lm_bytes < 2 * L2_BYTES
+    flush_buf = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev) if flush else None
+    stream = torch.cuda.current_stream()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for s in range(warmup + steps):
+        wl["ctx_lens"].copy_(ctx0)
+        if flush:
+            flush_buf.zero_()
+        e = evs[s - warmup] if s >= warmup else None
+        if e:
+            e[0].record(stream)
+        spade.spade_verify_attention(wl["q"], wl["k_cache"], wl["v_cache"], wl["ctx_lens"], wl["n_draft"],
+                                     wl["cu_q"], out, None, max_k=max_k, workspace=ws_attn, status=status)
+        if e:
+            e[1].record(stream)
+        spade.spade_verify_accept_commit(wl["hidden"], wl["w_lm"], wl["draft_tokens"], wl["draft_probs"],
+                                         wl["uniforms"], wl["mode"], wl["cu_q"], wl["n_draft"], acc, tok,
+                                         wl["k_cache"], wl["v_cache"], wl["ctx_lens"], workspace=ws_acc,
+                                         status=status)
+        if e:
+            e[2].record(stream)
+    torch.cuda.synchronize()
+    if int(status.item()) & ~spade.DEV_FALLBACK:
+        raise RuntimeError(f"device status {int(status.item())} on {wl['spec'].name}")
+    t_attn = statistics.median(e[0].elapsed_time(e[1]) * 1e-3 for e in evs)
+    t_acc = statistics.median(e[1].elapsed_time(e[2]) * 1e-3 for e in evs)
+    return t_attn, t_acc, int((acc.long() + 1).sum().item()), acc.tolist()
+
+
+def per_workload(args, dev, skip):
+    """Device timing of every other workload of the suite (no end-to-end leg, no oracle)."""
+    hbm, bf16, bf16_sus, peak_src = _peaks()
+    res = {}
+    for name, spec in W.SPECS.items():
+        if name == skip:
+            continue
+        wl = _to_device(W.make_workload(spec, device="cpu"), dev)
+        attn_bytes, lm_bytes, lm_flop, _, _ = _work_bytes(wl)
+        t_attn, t_acc, toks, acc = _time_step(wl, dev, args.per_workload_steps, 3)
+        lm = _lm_roofline(lm_bytes, lm_flop, t_acc, hbm, bf16_sus, bf16, peak_src)
+        res[name] = {"tokens_per_s": toks / (t_attn + t_acc), "us_per_step": (t_attn + t_acc) * 1e6,
+                     "tokens_per_step": toks, "accepted_len": acc,
+                     "verify_attention_us": t_attn * 1e6, "attention_hbm_frac": attn_bytes / t_attn / 1e9 / hbm,
+                     "verify_accept_commit_us": t_acc * 1e6, "lm_head_bound": lm["bound"],
+                     "lm_head_frac": lm["frac"], "lm_head_tensor_frac_of_sustained": lm["tensor"]["frac_of_sustained"],
+                     "steps": args.per_workload_steps, "timing": "median of CUDA-event times per launch"}
+        del wl
+        torch.cuda.empty_cache()
+    return res
+
+
+def _npf(t):
+    return None if t is None else (t.float().numpy() if t.dtype == torch.bfloat16 else t.numpy())
+
+
+def _oracle_one_sequence(wl_cpu, b):
+    """Runs the oracle's verify step (attention + LM head + accept + commit) on sequence b.
+
+    Returns (committed tokens, seconds, the oracle's accept result for b)."""
+    import oracle.spade_oracle as O
 
     cu = wl_cpu["cu_q"]
     r0, r1 = int(cu[b]), int(cu[b + 1])
     k = r1 - r0 - 1
-    q = npf(wl_cpu["q"][r0:r1])
-    kc = npf(wl_cpu["k_cache"][b:b + 1])
-    vc = npf(wl_cpu["v_cache"][b:b + 1])
-    ctx = npf(wl_cpu["ctx_lens"][b:b + 1])
+    q = _npf(wl_cpu["q"][r0:r1])
+    kc = _npf(wl_cpu["k_cache"][b:b + 1])
+    vc = _npf(wl_cpu["v_cache"][b:b + 1])
+    ctx = _npf(wl_cpu["ctx_lens"][b:b + 1])
     kd = [k]
     cu1 = [0, k + 1]
     t0 = time.perf_counter()
     O.verify_attention(q, kc, vc, ctx, kd, cu1)
-    logits = O.lm_logits(npf(wl_cpu["hidden"][r0:r1]), npf(wl_cpu["w_lm"]))
+    logits = O.lm_logits(_npf(wl_cpu["hidden"][r0:r1]), _npf(wl_cpu["w_lm"]))
     d0 = r0 - b
-    dp = npf(wl_cpu["draft_probs"][d0:d0 + k]) if wl_cpu["draft_probs"] is not None else None
-    res = O.verify_accept(logits, npf(wl_cpu["draft_tokens"][d0:d0 + k]), dp,
-                          npf(wl_cpu["uniforms"][r0:r1]), npf(wl_cpu["mode"][b:b + 1]), cu1, kd)
+    dp = _npf(wl_cpu["draft_probs"][d0:d0 + k]) if wl_cpu["draft_probs"] is not None else None
+    res = O.verify_accept(logits, _npf(wl_cpu["draft_tokens"][d0:d0 + k]), dp,
+                          _npf(wl_cpu["uniforms"][r0:r1]), _npf(wl_cpu["mode"][b:b + 1]), cu1, kd)
     O.kv_commit(kc, vc, ctx, res["accepted_len"], kd)
     dt = time.perf_counter() - t0
-    return int(res["accepted_len"][0]) + 1, dt
+    return int(res["accepted_len"][0]) + 1, dt, res
 
 
 def _cores():
@@ -444,13 +551,43 @@ def _cores():
         return os.cpu_count() or 1
 
 
-def cpu_baseline(wl):
-    wl_cpu = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in wl.items()}
-    tok, dt = _oracle_one_sequence(wl_cpu, 0)
-    return {"value": tok / dt, "unit": UNIT, "cores": _cores(), "kind": "oracle",
-            "sample": f"one sequence (b=0, {tok} committed tokens) of the workload: attention of its "
-                      f"k+1 rows x all heads, float64 LM head over the full vocabulary, accept, commit; "
-                      f"{dt:.2f} s"}
+CPU_BUDGET_S = 25.0
+
+
+def cpu_baseline(wl_cpu, acc_gpu, tok_gpu):
+    """The oracle on the benched step, sequence by sequence, until all are done or about
+    25 s of CPU time is spent; also the parity of the GPU step's decisions on them."""
+    toks, secs, per = 0, 0.0, []
+    B = wl_cpu["B"]
+    for b in range(B):
+        t, dt, res = _oracle_one_sequence(wl_cpu, b)
+        toks += t
+        secs += dt
+        per.append((b, dt, res))
+        if secs > CPU_BUDGET_S:
+            break
+    n = len(per)
+    times = [dt for _, dt, _ in per]
+    base = {"value": toks / secs, "unit": UNIT, "cores": _cores(), "kind": "oracle",
+            "sample": (f"sequences 0..{n - 1} of {B} of the workload ({toks} committed tokens), one at a time: "
+                       f"attention of its k+1 rows x all heads, float64 LM head over the full vocabulary, "
+                       f"accept, commit; {secs:.2f} s in all, per sequence mean {statistics.mean(times):.2f} s "
+                       f"(min {min(times):.2f}, max {max(times):.2f})")}
+    a_g, t_g = acc_gpu.numpy(), tok_gpu.numpy()
+    flagged = mism = mism_flagged = 0
+    acc_oracle = []
+    for b, _, res in per:
+        fl = bool(res["flag_decision"][0] or res["flag_sample"][0])
+        bad = a_g[b] != res["accepted_len"][0] or t_g[b] != res["next_token"][0]
+        flagged += fl
+        mism += bad and not fl
+        mism_flagged += bad and fl
+        acc_oracle.append(int(res["accepted_len"][0]))
+    par = {"sequences_checked": n, "of": B, "flagged": flagged, "mismatch_unflagged": mism,
+           "mismatch_flagged": mism_flagged, "accepted_len_oracle": acc_oracle,
+           "rule": "accepted length and next token bit-exact except at positions whose float64 top-2 logit "
+                   "gap, |u - p/q| or sampled-edge margin is below 1e-3 (flagged, counted here)"}
+    return base, par
 
 
 def run_reference(args):
@@ -460,19 +597,22 @@ def run_reference(args):
     for s in range(args.warmup):
         _oracle_one_sequence(wl, s % B)
     toks, secs = 0, 0.0
+    acc = [None] * B
     for s in range(args.steps):
-        t, dt = _oracle_one_sequence(wl, s % B)
+        t, dt, res = _oracle_one_sequence(wl, s % B)
         toks += t
         secs += dt
+        acc[s % B] = int(res["accepted_len"][0])
     value = toks / secs
     sample = (f"each step: one sequence of the {args.workload} workload through the float64 oracle "
-              f"(attention of its k+1 rows x {spec.Hq} heads, LM head over {spec.V} vocab, accept, commit)")
+              f"(attention of its k+1 rows x {spec.Hq} heads, LM head over {spec.V} vocab, accept, commit), "
+              f"sequences in turn")
     return {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 1, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": args.workload, "B": B, "Hq": spec.Hq, "Hkv": spec.Hkv, "D": spec.D,
-                   "H": spec.H, "V": spec.V, "ctx": list(spec.ctx), "k": list(spec.k), "mode": spec.mode},
+        "config": _config(spec, wl, 1),
+        "accepted_len": acc,
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": _cores(), "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -487,6 +627,9 @@ def main():
     ap.add_argument("--workload", default="llama3_8b", choices=sorted(W.SPECS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-per-workload", action="store_true",
+                    help="skip the device timing of the suite's other workloads")
+    ap.add_argument("--per-workload-steps", type=int, default=20)
     ap.add_argument("--separate-commit", action="store_true",
                     help="run the KV commit as its own launch instead of inside the LM-head kernel")
     args = ap.parse_args()

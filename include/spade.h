@@ -192,6 +192,25 @@ size_t spade_accept_workspace_size(int32_t B, int32_t R, int32_t H, int32_t V);
 int32_t spade_accept_launches(int32_t B, int32_t R, int32_t H, int32_t V);
 
 /*
+ * Where a completed spade_verify_accept (or spade_verify_accept_commit) call
+ * leaves its merged per-row softmax statistics inside the workspace, for
+ * tests and diagnostics that check the on-chip logits without writing them
+ * out (Sec. III-A: p = softmax(o), o = g(x_L)).  For row r (0 <= r < R):
+ *   float4 at byte row_stats_offset + 16 * r: x = max_x logits[r, x],
+ *     y = sum_x exp(logits[r, x] - x-component), z = argmax_x logits[r, x]
+ *     (int32 bits, lowest index on ties), w = accept bit of the row (int32
+ *     bits; 1 iff the row's draft passed its test);
+ *   float at byte draft_logit_offset + 4 * r: logits[r, d] of the row's draft
+ *     token d (rows i < k_b only; other entries are not written).
+ * The statistics are stored in several copies `replica_stride` float4 apart;
+ * the first copy is the one described.  Valid until the next call that uses
+ * the workspace.  Returns SPADE_ERR_INVALID_ARG on null outputs or bad sizes.
+ */
+spade_status spade_accept_stats_layout(int32_t B, int32_t R, int32_t H, int32_t V,
+                                       size_t *row_stats_offset, size_t *draft_logit_offset,
+                                       int32_t *replica_stride);
+
+/*
  * spade_verify_accept followed by spade_kv_commit, in one launch: once the
  * accept decisions are taken on the device, the same kernel clears the
  * rejected draft slots [ctx_b + a_b + 1, ctx_b + n_draft[b]] of k_cache and

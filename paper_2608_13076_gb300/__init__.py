@@ -23,7 +23,8 @@ from . import _build
 __all__ = [
     "SpadeError", "load", "build", "library_path",
     "spade_verify_attention", "spade_verify_accept", "spade_kv_commit", "spade_verify_attention_noalloc",
-    "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_accept_launches", "spade_selftest_wait_timeout",
+    "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_accept_launches",
+    "spade_accept_stats_layout", "read_accept_stats", "spade_verify_accept_commit", "spade_selftest_wait_timeout",
     "attn_workspace", "accept_workspace", "status_tensor", "check_status",
     "DEV_BAD_INDEX", "DEV_CAPACITY", "DEV_TIMEOUT", "DEV_FALLBACK",
 ]
@@ -81,6 +82,8 @@ def load():
     lib.spade_verify_accept_commit.argtypes = [_vp] * 13 + [_i32] * 7 + [_vp, _sz, _vp, _vp]
     lib.spade_accept_workspace_size.restype = _sz
     lib.spade_accept_workspace_size.argtypes = [_i32] * 4
+    lib.spade_accept_stats_layout.restype = _i32
+    lib.spade_accept_stats_layout.argtypes = [_i32] * 4 + [_vp, _vp, _vp]
     lib.spade_accept_launches.restype = _i32
     lib.spade_accept_launches.argtypes = [_i32] * 4
     lib.spade_selftest_wait_timeout.restype = _i32
@@ -205,6 +208,29 @@ def spade_selftest_wait_timeout(status, limit_us, stream=None):
     """One bounded wait that nothing completes: SPADE_DEV_TIMEOUT lands in `status` after limit_us."""
     _need(status, "status", torch.int32, 1)
     _check_rc(load().spade_selftest_wait_timeout(_ptr(status), int(limit_us), _stream(stream)))
+
+
+def spade_accept_stats_layout(B, R, H, V):
+    """Byte offsets of the merged row statistics and the draft logits in an accept workspace.
+
+    Returns (row_stats_offset, draft_logit_offset, replica_stride); see include/spade.h.
+    """
+    a, b, c = ctypes.c_size_t(0), ctypes.c_size_t(0), ctypes.c_int32(0)
+    _check_rc(load().spade_accept_stats_layout(B, R, H, V, ctypes.byref(a), ctypes.byref(b), ctypes.byref(c)))
+    return int(a.value), int(b.value), int(c.value)
+
+
+def read_accept_stats(workspace, B, R, H, V):
+    """Row statistics a completed accept call left in `workspace` (reads device memory).
+
+    Returns dict of torch CPU tensors: max [R] f32, sumexp [R] f32, argmax [R] i32,
+    accept_bit [R] i32, draft_logit [R] f32 (rows with a draft only are meaningful).
+    """
+    off_s, off_d, _ = spade_accept_stats_layout(B, R, H, V)
+    st = workspace[off_s:off_s + 16 * R].view(torch.float32).view(R, 4).cpu()
+    ld = workspace[off_d:off_d + 4 * R].view(torch.float32).cpu()
+    return dict(max=st[:, 0].clone(), sumexp=st[:, 1].clone(), argmax=st[:, 2].clone().view(torch.int32),
+                accept_bit=st[:, 3].clone().view(torch.int32), draft_logit=ld.clone())
 
 
 def spade_accept_launches(B, R, H, V):

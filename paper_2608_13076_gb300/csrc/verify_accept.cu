@@ -1807,6 +1807,25 @@ extern "C" size_t spade_accept_workspace_size(int32_t B, int32_t R, int32_t H, i
   return accept::ws_layout(B, R, H, V, sms).end;
 }
 
+extern "C" spade_status spade_accept_stats_layout(int32_t B, int32_t R, int32_t H, int32_t V,
+                                                  size_t *row_stats_offset, size_t *draft_logit_offset,
+                                                  int32_t *replica_stride) {
+  if (!row_stats_offset || !draft_logit_offset || !replica_stride)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_accept_stats_layout: null output pointer");
+  if (B <= 0 || R < B || H <= 0 || V <= 0)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_accept_stats_layout: bad sizes B=%d R=%d H=%d V=%d", B, R, H, V);
+  int sms = 0;
+  const spade_status st = device_info(&sms, nullptr);
+  if (st != SPADE_OK) return st;
+  // The statistics of every row are those of the first launch (the resident
+  // pass, or the statistics pass of a two-pass shape).
+  const accept::WsLayout L = accept::ws_layout(B, R, H, V, sms);
+  *row_stats_offset = L.r1.gstat;
+  *draft_logit_offset = L.r1.ldraft;
+  *replica_stride = R;
+  return SPADE_OK;
+}
+
 namespace spade {
 namespace accept {
 struct CommitArgs {

@@ -141,9 +141,12 @@ extern "C" spade_status spade_verify_attention_noalloc(
     int32_t Hkv, int32_t D, int32_t cap, int32_t max_k, int32_t R, int32_t *status,
     spade_stream_t stream) {
   using namespace attn_noalloc;
-  if (B <= 0 || Hq <= 0 || Hkv <= 0 || cap <= 0 || max_k < 0 || R <= 0 || Hq % Hkv ||
-      (D != 64 && D != 128))
-    return fail(SPADE_ERR_INVALID_ARG, "spade_verify_attention_noalloc: bad sizes");
+  // The same size checks, in the same order and with the same codes, as
+  // spade_verify_attention.
+  if (B <= 0 || Hq <= 0 || Hkv <= 0 || cap <= 0 || max_k < 0 || R <= 0)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_verify_attention_noalloc: non-positive size");
+  if (Hq % Hkv) return fail(SPADE_ERR_SHAPE, "Hq (%d) must be a multiple of Hkv (%d)", Hq, Hkv);
+  if (D != 64 && D != 128) return fail(SPADE_ERR_SHAPE, "head dim %d not supported (64 or 128)", D);
   int dev = 0;
   spade_status st = device_info(nullptr, &dev);
   if (st != SPADE_OK) return st;

@@ -97,3 +97,14 @@ def test_bad_shapes_rejected(lib):
     # head dim not a multiple of 8 for commit
     assert lib.spade_kv_commit(*([p] * 5), 1, 8, 12, 300, p, None) == 2
     assert lib.spade_verify_accept_commit(*([p] * 13), 1, 5, 512, 1024, 8, 12, 300, p, 1 << 20, p, None) == 2
+    # The allocation-free attention gives the workspace entry point's codes.
+    assert lib.spade_verify_attention_noalloc(*args, 1, 6, 4, 128, 300, 4, 5, p, None) == 2
+    assert lib.spade_verify_attention_noalloc(*args, 1, 8, 8, 96, 300, 4, 5, p, None) == 2
+    assert lib.spade_verify_attention_noalloc(*args, 0, 8, 8, 128, 300, 4, 5, p, None) == 1
+
+
+def test_stats_layout_rejects_bad_arguments(lib):
+    out = ctypes.c_size_t(0)
+    assert lib.spade_accept_stats_layout(1, 5, 512, 1024, None, None, None) == 1
+    assert lib.spade_accept_stats_layout(4, 3, 512, 1024, ctypes.byref(out), ctypes.byref(out),
+                                         ctypes.byref(ctypes.c_int32(0))) == 1

@@ -218,20 +218,197 @@ def _sample_pairs(wl, n, seed):
     return sorted(pairs)
 
 
+def _flag_bound(B):
+    """Most sequences a workload may have flagged: positions whose oracle margin is below
+    1e-3 are rare with N(0, 1) logits (about 0.5 % of top-2 gaps over 10^5 entries, 0.2 %
+    of sampled edges), so more than this means the margins are computed wrongly."""
+    return max(2, B // 16)
+
+
 @pytest.mark.parametrize("name", FULL)
 def test_full_workload(dev, name):
+    """The step bench.py times (attention, then accept + KV commit in one launch) against the
+    oracle at full size: attention on sampled (row, head) pairs, every accept decision, the
+    on-chip logits through the merged row statistics, and the commit of every sequence."""
     wl = W.make_workload(W.SPECS[name], device=dev)
+    B, R = wl["B"], wl["R"]
+    before = {k: wl[k].clone() for k in ("k_cache", "v_cache", "ctx_lens", "n_draft")}
     out, lse, st = parity.gpu_attention(wl)
-    acc, tok, st2 = parity.gpu_accept(wl)
+    acc, tok, ws, st2 = parity.gpu_accept_commit(wl)
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     assert int(st2.item()) & ~spade.DEV_FALLBACK == 0
     pairs = _sample_pairs(wl, 256, 7)
-    ref, _ = parity.oracle_attention(wl, rows=pairs)
+    ref, _ = parity.oracle_attention(dict(wl, **before), rows=pairs)
     n, bad, worst = parity.compare_attention(out, ref, rows=pairs)
     assert bad == 0, f"attention: {bad} bad elements over {n} pairs, worst {worst:.3g}"
-    ref_acc = parity.oracle_accept(wl)
+    logits = parity.oracle_logits(wl)
+    ref_acc = parity.oracle_accept_from_logits(wl, logits)
     cmp = parity.compare_accept(acc, tok, ref_acc)
+    stats = spade.read_accept_stats(ws, B, R, wl["H"], wl["V"])
+    rs = parity.compare_row_stats(stats, logits, wl)
     print(f"{name}: accepted {parity.to_np(acc).tolist()} flagged {cmp['flagged']} "
-          f"flagged-mismatch {cmp['mismatch_flagged']}")
+          f"flagged-mismatch {cmp['mismatch_flagged']} row stats {rs}")
     assert cmp["mismatch_unflagged"] == 0, cmp
+    assert cmp["flagged"] <= _flag_bound(B), cmp
+    assert rs["max"] <= 1 and rs["lse"] <= 1 and rs["draft_logit"] <= 1, rs
+    assert rs["argmax_mismatch"] == 0, rs
+    parity.check_commit_windows(before, wl["k_cache"], wl["v_cache"], wl["ctx_lens"], acc)
+
+
+# ---------------------------------------------------------------------------
+# Edge cases of the method that random N(0, 1) inputs almost never produce.
+
+def _integer_lm(wl, seed):
+    """Replace hidden and W by values in {-1, 0, 1} and {-1, 0, 1}/16: every product and
+    partial sum is exact in fp32, so the logits are exact multiples of 1/16 in any
+    summation order and exact ties between vocabulary entries are frequent."""
+    g = torch.Generator().manual_seed(seed)
+    shape = tuple(wl["hidden"].shape)
+    # About 8 nonzero entries per row: few distinct logit values, so ties at the top are common.
+    keep = torch.rand(shape, generator=g) < 8.0 / shape[1]
+    wl["hidden"] = (torch.randint(-1, 2, shape, generator=g) * keep).to(torch.bfloat16).to(wl["hidden"].device)
+    wl["w_lm"] = (torch.randint(-1, 2, tuple(wl["w_lm"].shape), generator=g).float() / 16).to(
+        torch.bfloat16).to(wl["w_lm"].device)
+
+
+EDGE = {
+    "ties_one_pass": W.WorkloadSpec("ties_one_pass", B=6, Hq=4, Hkv=4, D=64, H=256, V=4000, ctx=(8, 64),
+                                    k=(1, 6), mode="greedy", seed=41),
+    # 72 vocabulary tiles: an even grid, so the statistics pass runs on CTA pairs.
+    "ties_two_pass": W.WorkloadSpec("ties_two_pass", B=40, Hq=4, Hkv=4, D=64, H=256, V=9100, ctx=(8, 64),
+                                    k=(6, 9), mode="greedy", seed=42),
+}
+
+
+@pytest.mark.parametrize("name", sorted(EDGE))
+def test_exact_logit_ties_lowest_index(dev, name):
+    """Exact ties between vocabulary entries (in one tile, across tiles and across SMs):
+    the argmax is the lowest tied index, bit for bit, and the greedy decisions follow."""
+    wl = W.make_workload(EDGE[name], device=dev)
+    _integer_lm(wl, 7)
+    logits = parity.oracle_logits(wl)
+    # Half the drafts are the (lowest-index) argmax so that acceptance goes deep.
+    cu = parity.to_np(wl["cu_q"])
+    kd = parity.to_np(wl["n_draft"])
+    am = logits.argmax(axis=1)
+    drafts = parity.to_np(wl["draft_tokens"]).copy()
+    rng = np.random.default_rng(3)
+    for b in range(wl["B"]):
+        for i in range(int(kd[b])):
+            if rng.random() < 0.8:
+                drafts[int(cu[b]) - b + i] = am[int(cu[b]) + i]
+    wl["draft_tokens"] = torch.from_numpy(drafts).to(dev)
+    top = np.sort(logits, axis=1)
+    assert (top[:, -1] == top[:, -2]).sum() >= wl["R"] // 8, "the case must contain many exact ties"
+    acc, tok, ws, st = parity.gpu_accept_commit(wl)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    ref = parity.oracle_accept_from_logits(wl, logits)
+    stats = spade.read_accept_stats(ws, wl["B"], wl["R"], wl["H"], wl["V"])
+    # Exact arithmetic on both sides: no margin excuses anything here.
+    assert np.array_equal(stats["argmax"].numpy(), am)
+    assert np.array_equal(stats["max"].double().numpy(), logits.max(axis=1))
+    assert np.array_equal(parity.to_np(acc), ref["accepted_len"])
+    assert np.array_equal(parity.to_np(tok), ref["next_token"])
+
+
+def test_stochastic_zero_draft_probability_accepts(dev):
+    """q(d) = 0 with p(d) > 0 accepts (alpha = min(1, p/q) = 1) whatever u is; with every
+    draft accepted the bonus is drawn from p, and u = 0 gives the first vocabulary id."""
+    spec = W.WorkloadSpec("q_zero", B=5, Hq=4, Hkv=4, D=64, H=256, V=3000, ctx=(8, 64), k=(2, 5),
+                          mode="stochastic", seed=43)
+    wl = W.make_workload(spec, device=dev)
+    cu = parity.to_np(wl["cu_q"])
+    kd = parity.to_np(wl["n_draft"])
+    dt = parity.to_np(wl["draft_tokens"])
+    u = parity.to_np(wl["uniforms"]).copy()
+    for b in range(wl["B"]):
+        for i in range(int(kd[b])):
+            d = int(dt[int(cu[b]) - b + i])
+            wl["draft_probs"][int(cu[b]) - b + i, d] = 0.0
+            u[int(cu[b]) + i] = 0.999999
+        u[int(cu[b]) + int(kd[b])] = 0.0 if b % 2 == 0 else u[int(cu[b]) + int(kd[b])]
+    wl["uniforms"] = torch.from_numpy(u).to(dev)
+    acc, tok, ws, st = parity.gpu_accept_commit(wl)
+    torch.cuda.synchronize()
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0
+    ref = parity.oracle_accept(wl)
+    assert np.array_equal(ref["accepted_len"], kd)
+    assert np.array_equal(parity.to_np(acc), kd)
+    t = parity.to_np(tok)
+    for b in range(0, wl["B"], 2):
+        assert t[b] == 0 and ref["next_token"][b] == 0
+    assert parity.compare_accept(acc, tok, ref)["mismatch_unflagged"] == 0
+
+
+@pytest.mark.parametrize("u_sample", [0.0, 1.0 - 2.0 ** -24])
+def test_sampling_uniform_extremes(dev, u_sample):
+    """u = 0 takes the first id with residual mass; u just below 1 the last (the clamp when
+    rounding leaves u*Z at or past the total).  Both sides agree, or the position is one the
+    oracle flags as within 1e-3 of an interval edge; the token always has mass."""
+    spec = W.WorkloadSpec("u_edge", B=8, Hq=4, Hkv=4, D=64, H=256, V=5000, ctx=(8, 64), k=(1, 4),
+                          mode="stochastic", seed=44)
+    wl = W.make_workload(spec, device=dev)
+    cu = parity.to_np(wl["cu_q"])
+    kd = parity.to_np(wl["n_draft"])
+    u = parity.to_np(wl["uniforms"]).copy()
+    for b in range(wl["B"]):
+        u[int(cu[b]) + int(kd[b])] = np.float32(u_sample)
+    wl["uniforms"] = torch.from_numpy(u).to(dev)
+    acc, tok, ws, st = parity.gpu_accept_commit(wl)
+    torch.cuda.synchronize()
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0
+    logits = parity.oracle_logits(wl)
+    ref = parity.oracle_accept_from_logits(wl, logits)
+    cmp = parity.compare_accept(acc, tok, ref)
+    assert cmp["mismatch_unflagged"] == 0, cmp
+    a, t = parity.to_np(acc), parity.to_np(tok)
+    q = parity.to_np(wl["draft_probs"])
+    for b in range(wl["B"]):
+        r = int(cu[b]) + int(a[b])
+        p = O.softmax(logits[r])
+        mass = p - q[int(cu[b]) - b + int(a[b])] if a[b] < kd[b] else p
+        # (fp32 may keep an entry whose float64 residual is a rounding away from zero)
+        assert 0 <= t[b] < wl["V"] and mass[t[b]] > -1e-7
+
+
+def test_draft_ids_at_tile_and_vocabulary_edges(dev):
+    """Draft ids 0, V-1 and ids on 128-row tile edges: the draft logit captured on chip
+    matches the oracle's, and so do the decisions."""
+    spec = W.WorkloadSpec("edge_ids", B=8, Hq=4, Hkv=4, D=64, H=256, V=20000, ctx=(8, 64), k=(4, 6),
+                          mode="mixed", seed=45)
+    wl = W.make_workload(spec, device=dev)
+    V = wl["V"]
+    ids = [0, V - 1, 127, 128, 255, 256, 1023, 1024, V - 128, V - 129]
+    n = wl["draft_tokens"].numel()
+    wl["draft_tokens"] = torch.tensor([ids[i % len(ids)] for i in range(n)], dtype=torch.int32, device=dev)
+    acc, tok, ws, st = parity.gpu_accept_commit(wl)
+    torch.cuda.synchronize()
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0
+    logits = parity.oracle_logits(wl)
+    ref = parity.oracle_accept_from_logits(wl, logits)
+    assert parity.compare_accept(acc, tok, ref)["mismatch_unflagged"] == 0
+    rs = parity.compare_row_stats(spade.read_accept_stats(ws, wl["B"], wl["R"], wl["H"], V), logits, wl)
+    assert rs["draft_logit"] <= 1 and rs["max"] <= 1 and rs["lse"] <= 1 and rs["argmax_mismatch"] == 0, rs
+
+
+def test_long_greedy_sequence_in_two_pass_batch(dev):
+    """A two-pass batch (R > 256 rows) whose sequences have 60 drafts each, greedy ones with
+    drafts that mostly match, so acceptance runs deep and some sequences accept all 60."""
+    spec = W.WorkloadSpec("deep_two_pass", B=5, Hq=4, Hkv=2, D=128, H=320, V=9000, ctx=(20, 200),
+                          k=(60, 60), mode="mixed", match_prob=0.995, seed=46)
+    wl = W.make_workload(spec, device=dev)
+    assert wl["R"] > 256 and spade.spade_accept_launches(wl["B"], wl["R"], wl["H"], wl["V"]) == 2
+    before = {k: wl[k].clone() for k in ("k_cache", "v_cache", "ctx_lens", "n_draft")}
+    out, lse, st0 = parity.gpu_attention(wl)
+    acc, tok, ws, st = parity.gpu_accept_commit(wl)
+    torch.cuda.synchronize()
+    assert int(st0.item()) == 0 and int(st.item()) & ~spade.DEV_FALLBACK == 0
+    n, bad, worst = parity.compare_attention(out, parity.oracle_attention(dict(wl, **before))[0])
+    assert bad == 0, worst
+    logits = parity.oracle_logits(wl)
+    ref = parity.oracle_accept_from_logits(wl, logits)
+    assert parity.compare_accept(acc, tok, ref)["mismatch_unflagged"] == 0
+    assert int(ref["accepted_len"][0]) >= 30  # the greedy sequence b = 0 accepts deep
+    parity.check_commit_windows(before, wl["k_cache"], wl["v_cache"], wl["ctx_lens"], acc)

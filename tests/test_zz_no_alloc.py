@@ -44,14 +44,13 @@ def test_noalloc_matches_workspace_entry_point(gpu_lib, spec):
         outs.append((out, lse))
     torch.cuda.synchronize()
     assert int(st.item()) == 0
-    ref_np = parity.to_np(ref).astype("float64")
     for out, lse in outs:
-        # Same kernel, same schedule: the results agree far inside the parity tolerance.
-        g = parity.to_np(out).astype("float64")
-        err = abs(g - ref_np)
-        tol = parity.ATTN_RTOL * abs(ref_np).clip(min=float(abs(ref_np).mean()))
-        assert (err <= tol).all()
-        assert torch.allclose(lse, ref_lse, rtol=0, atol=2e-3)
+        # Same kernel, same schedule, same inputs: the results are identical.
+        assert torch.equal(out, ref)
+        assert torch.equal(lse, ref_lse)
+    # The static array starts at zero and every completed call leaves its merge
+    # counters at zero again, so the clearing memset at the start of each call
+    # only matters after an interrupted call; that path is checked by reading.
 
 
 def test_noalloc_rejects_sizes_beyond_the_static_scratch(gpu_lib):
@@ -63,3 +62,8 @@ def test_noalloc_rejects_sizes_beyond_the_static_scratch(gpu_lib):
                                             None)
     assert rc == 3  # SPADE_ERR_CAPACITY, refused before any launch
     assert b"static scratch" in lib.spade_last_error()
+    # Unsupported shapes get the codes spade_verify_attention gives them.
+    rc = lib.spade_verify_attention_noalloc(p, p, p, p, p, p, p, None, 1, 8, 8, 96, 64, 1, 2, p, None)
+    assert rc == 2  # SPADE_ERR_SHAPE: head dim 96
+    rc = lib.spade_verify_attention_noalloc(p, p, p, p, p, p, p, None, 1, 8, 3, 128, 64, 1, 2, p, None)
+    assert rc == 2  # SPADE_ERR_SHAPE: Hq % Hkv != 0
