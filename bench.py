@@ -583,8 +583,8 @@ def cpu_baseline(wl_cpu, acc_gpu, tok_gpu):
         mism += bad and not fl
         mism_flagged += bad and fl
         acc_oracle.append(int(res["accepted_len"][0]))
-    par = {"sequences_checked": n, "of": B, "flagged": flagged, "mismatch_unflagged": mism,
-           "mismatch_flagged": mism_flagged, "accepted_len_oracle": acc_oracle,
+    par = {"sequences_checked": n, "of": B, "flagged": int(flagged), "mismatch_unflagged": int(mism),
+           "mismatch_flagged": int(mism_flagged), "accepted_len_oracle": acc_oracle,
            "rule": "accepted length and next token bit-exact except at positions whose float64 top-2 logit "
                    "gap, |u - p/q| or sampled-edge margin is below 1e-3 (flagged, counted here)"}
     return base, par
@@ -618,6 +618,13 @@ def run_reference(args):
     }
 
 
+def _json_default(o):
+    """numpy scalars (from the oracle's results) as plain numbers."""
+    if hasattr(o, "item"):
+        return o.item()
+    raise TypeError(f"{type(o).__name__} is not JSON serializable")
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -637,14 +644,14 @@ def main():
     ws, rank, local = _dist()
     if args.impl == "reference":
         if rank == 0:
-            print(json.dumps(run_reference(args)), flush=True)
+            print(json.dumps(run_reference(args), default=_json_default), flush=True)
         return
     if ws > 1:
         torch.cuda.set_device(local)
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local))
     line = run_spade(args, ws, rank, local)
     if rank == 0:
-        print(json.dumps(line), flush=True)
+        print(json.dumps(line, default=_json_default), flush=True)
     if ws > 1:
         torch.distributed.destroy_process_group()
 
