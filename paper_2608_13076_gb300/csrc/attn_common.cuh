@@ -37,6 +37,15 @@ struct Params {
 
 constexpr int round_up_c(int x, int a) { return (x + a - 1) / a * a; }
 
+// n / d for n >= 0, d > 0: a 32-bit division whenever both fit (every schedule
+// of practical size), else the 64-bit one.  A 64-bit division is a long
+// software sequence, and the schedule sits on the path to the first copy.
+__device__ __forceinline__ int64_t div_nn(int64_t n, int64_t d) {
+  if (((n | d) >> 31) == 0)
+    return static_cast<int64_t>(static_cast<uint32_t>(n) / static_cast<uint32_t>(d));
+  return n / d;
+}
+
 __host__ __device__ constexpr int slot_floats(int D) { return kRowBlock * D + 2 * kRowBlock; }
 
 // Per-CTA view of the schedule.  The units' key slices are laid end to end in
@@ -64,7 +73,7 @@ struct Sched {
   __device__ int cost(int b, int rb) const { return chunks(b, rb) + E; }
   // CTA whose range holds cost position x.
   __device__ int64_t owner(int64_t x) const {
-    return ((x + 1) * num_ctas + total - 1) / total - 1;
+    return div_nn((x + 1) * num_ctas + total - 1, total) - 1;
   }
 };
 
@@ -75,12 +84,9 @@ struct Seg {
   int64_t ust;   // cost position of the unit's start (its first real slice is at ust + E)
 };
 
-__device__ __forceinline__ Seg locate(const Sched &s, int64_t x) {
-  int lo = 0, hi = s.B - 1;  // largest b with pref[b] <= x
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (s.pref[mid] <= x) lo = mid; else hi = mid - 1;
-  }
+// The unit and cost offset of position x inside sequence b's cost range.
+__device__ __forceinline__ Seg locate_in(const Sched &s, int b, int64_t x) {
+  const int lo = b;
   Seg g;
   g.b = lo;
   g.nch = 0;
@@ -88,7 +94,7 @@ __device__ __forceinline__ Seg locate(const Sched &s, int64_t x) {
   int span = 0;
   for (int rb = 0; rb < nrb; ++rb) span += s.cost(lo, rb);
   int64_t o = x - s.pref[lo];
-  g.kvh = static_cast<int>(o / span);
+  g.kvh = static_cast<int>(div_nn(o, span));
   int o2 = static_cast<int>(o - static_cast<int64_t>(g.kvh) * span);
   int cum = 0;
   g.rb = 0;
@@ -101,6 +107,41 @@ __device__ __forceinline__ Seg locate(const Sched &s, int64_t x) {
   g.ust = s.pref[lo] + static_cast<int64_t>(g.kvh) * span + cum;
   return g;
 }
+
+// Position x of the cost space (one thread): the sequence by binary search.
+__device__ __forceinline__ Seg locate(const Sched &s, int64_t x) {
+  int lo = 0, hi = s.B - 1;  // largest b with pref[b] <= x
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (s.pref[mid] <= x) lo = mid; else hi = mid - 1;
+  }
+  return locate_in(s, lo, x);
+}
+
+// The same for a whole warp (all lanes get the result): lane l tests whether
+// sequence b0 + l holds x, so 32 sequences take one vote instead of a chain of
+// dependent shared-memory loads.
+__device__ __forceinline__ Seg locate_warp(const Sched &s, int64_t x, int lane) {
+  int b = 0;
+  for (int b0 = 0; b0 < s.B; b0 += 32) {
+    const int bb = b0 + lane;
+    const bool hit = bb < s.B && s.pref[bb] <= x && x < s.pref[bb + 1];
+    const unsigned m = __ballot_sync(0xffffffffu, hit);
+    if (m) {
+      b = b0 + __ffs(m) - 1;
+      break;
+    }
+  }
+  return locate_in(s, b, x);
+}
+
+// A CTA's range [x_begin, x_end) of the cost space and the schedule totals,
+// computed once by the set-up warp and read by every role.
+struct CtaRange {
+  int64_t x_begin, x_end, total;
+  int num_ctas;
+  int active;  // 0: this CTA has no work
+};
 
 // bar.sync is the aligned form: every lane of a warp must arrive together.
 // Lanes that ran ahead of a divergent lane (a lane-0-only loop) reconverge

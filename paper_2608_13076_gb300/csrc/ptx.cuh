@@ -87,6 +87,17 @@ SPADE_DEVICE bool mbar_wait_unabortable(uint64_t *bar, uint32_t parity) {
   return true;
 }
 
+// ---------------------------------------------------------------- programmatic dependent launch
+// Waits until the grids this launch depends on have completed and their
+// writes are visible; a no-op for a launch without the programmatic attribute.
+SPADE_DEVICE void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Lets the next grid in the stream be scheduled before this one ends; that
+// grid still waits (griddep_wait) for this grid's completion before it reads
+// anything this grid writes.
+SPADE_DEVICE void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---------------------------------------------------------------- TMA
 SPADE_DEVICE void tma_prefetch_desc(const CUtensorMap *map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");

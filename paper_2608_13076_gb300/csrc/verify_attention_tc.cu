@@ -71,7 +71,8 @@ struct Smem {
   static constexpr int BAR = ALPHA + kRowBlock * 4;
   static constexpr int MISC = BAR + kNumBars * 8;           // abort, last, tmem base
   static constexpr int SEG0 = MISC + 64;                    // SegInfo: this CTA's first segment
-  static constexpr int BYTES = SEG0 + 64 + 1024;            // + slack for 1024-byte alignment
+  static constexpr int RANGE = SEG0 + 64;                   // CtaRange: this CTA's cost range
+  static constexpr int BYTES = RANGE + 64 + 1024;           // + slack for 1024-byte alignment
 };
 static_assert(Smem::BAR % 8 == 0, "mbarriers need 8-byte alignment");
 static_assert(Smem::RMAX % 16 == 0, "row maxima are read as float4");
@@ -151,9 +152,9 @@ struct SegInfo {
   int n_here;   // key slices in this segment (0: only the unit's virtual start)
   int nchunk;   // MMA chunks (pairs of slices, the last one possibly single)
 };
-__device__ __forceinline__ SegInfo seg_at(const Sched &sc, int64_t x, int64_t x_end) {
+__device__ __forceinline__ SegInfo seg_of(const Sched &sc, const Seg &g, int64_t x, int64_t x_end) {
   SegInfo s;
-  s.g = locate(sc, x);
+  s.g = g;
   s.seg_end = min(x_end, s.g.ust + sc.E + s.g.nch);
   const int lo = max(0, static_cast<int>(x - s.g.ust) - sc.E);
   const int hi = max(0, static_cast<int>(s.seg_end - s.g.ust) - sc.E);
@@ -162,11 +163,20 @@ __device__ __forceinline__ SegInfo seg_at(const Sched &sc, int64_t x, int64_t x_
   s.nchunk = (s.n_here + 1) / 2;
   return s;
 }
+__device__ __forceinline__ SegInfo seg_at(const Sched &sc, int64_t x, int64_t x_end) {
+  return seg_of(sc, locate(sc, x), x, x_end);
+}
 // The first segment at or after cost position x that holds key slices (all
 // roles skip the same empty ones); n_here == 0 when the range has none left.
 __device__ __forceinline__ SegInfo next_seg(const Sched &sc, int64_t x, int64_t x_end) {
   SegInfo s = seg_at(sc, x, x_end);
   while (s.n_here == 0 && s.seg_end < x_end) s = seg_at(sc, s.seg_end, x_end);
+  return s;
+}
+// The same, computed by a whole warp (every lane gets the result).
+__device__ __forceinline__ SegInfo next_seg_warp(const Sched &sc, int64_t x, int64_t x_end, int lane) {
+  SegInfo s = seg_of(sc, locate_warp(sc, x, lane), x, x_end);
+  while (s.n_here == 0 && s.seg_end < x_end) s = seg_of(sc, locate_warp(sc, s.seg_end, lane), s.seg_end, x_end);
   return s;
 }
 
@@ -204,42 +214,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int lane = tid & 31;
 
   if (tid == 0) { *s_abort = 0; *s_last = 0; }
-  // The producer's tensor-map fetches overlap the schedule loads below.
+  // Set-up that reads no input -- tensor-map prefetch, mbarriers, tensor
+  // memory, the zero slab -- comes first: under programmatic dependent launch
+  // it overlaps the end of the previous kernel in the stream.
   if (warp == 0 && lane < 2) {
     tma_prefetch_desc(lane ? &tm_v2 : &tm_k2);
     tma_prefetch_desc(lane ? &tm_v1 : &tm_k1);
-  }
-  if constexpr (kD == 64) {
-    // The V tiles' second 64-dim slab: zeros for the whole launch (the copies
-    // fill the first slab only).
-    for (int e = tid; e < kStages * (kSlab / 16); e += kThreads) {
-      const int st = e / (kSlab / 16), o = e % (kSlab / 16);
-      *reinterpret_cast<uint4 *>(smem + Smem::V + st * kTile + kSlab + o * 16) = make_uint4(0, 0, 0, 0);
-    }
-    fence_proxy_async_smem();
-  }
-  sched_validate(p, s_ctx, s_kd, tid, kThreads);
-  block_sync();
-  Sched sc;
-  sc.pref = s_pref; sc.ctx = s_ctx; sc.kd = s_kd;
-  sc.B = p.B; sc.Hkv = p.Hkv; sc.G = p.G; sc.RB = p.RB; sc.E = p.unit_cost; sc.num_ctas = p.num_ctas;
-  // One barrier for the schedule (warp 0: the prefix scan, then this CTA's
-  // first segment, which every role starts from) and the mbarriers and the
-  // tensor-memory allocation (warp 1).
-  SegInfo *s_seg0 = reinterpret_cast<SegInfo *>(smem + Smem::SEG0);
-  if (warp == 0) {
-    sched_scan(p, sc, s_pref, lane);
-    __syncwarp();
-    if (lane == 0) {
-      Sched s0 = sc;
-      s0.total = s_pref[p.B];
-      s0.num_ctas = static_cast<int>(s0.total < p.num_ctas ? s0.total : p.num_ctas);
-      if (s0.total > 0 && static_cast<int>(blockIdx.x) < s0.num_ctas) {
-        const int64_t xb = static_cast<int64_t>(blockIdx.x) * s0.total / s0.num_ctas;
-        const int64_t xe = static_cast<int64_t>(blockIdx.x + 1) * s0.total / s0.num_ctas;
-        *s_seg0 = next_seg(s0, xb, xe);
-      }
-    }
   } else if (warp == 1) {
     if (lane == 0) {
       for (int s = 0; s < kStages; ++s) {
@@ -262,19 +242,65 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(s_tmem, kTmemCols);
     tmem_relinquish();
   }
+  if constexpr (kD == 64) {
+    // The V tiles' second 64-dim slab: zeros for the whole launch (the copies
+    // fill the first slab only).
+    for (int e = tid; e < kStages * (kSlab / 16); e += kThreads) {
+      const int st = e / (kSlab / 16), o = e % (kSlab / 16);
+      *reinterpret_cast<uint4 *>(smem + Smem::V + st * kTile + kSlab + o * 16) = make_uint4(0, 0, 0, 0);
+    }
+    fence_proxy_async_smem();
+  }
+  // Inputs written by earlier kernels in the stream are visible from here on.
+  // The next kernel may be scheduled now: it waits for this grid to complete
+  // before it reads anything this grid writes.
+  griddep_wait();
+  griddep_launch_dependents();
+  sched_validate(p, s_ctx, s_kd, tid, kThreads);
   tc_fence_before();
   block_sync();
   tc_fence_after();
-  sc.total = s_pref[p.B];
-  // Never more CTAs than slices: every CTA kept has a non-empty range, so the
-  // CTAs between a unit's first and last owner all contribute a partial.
-  sc.num_ctas = static_cast<int>(sc.total < p.num_ctas ? sc.total : p.num_ctas);
-  if (sc.total == 0 || static_cast<int>(blockIdx.x) >= sc.num_ctas) {
+  Sched sc;
+  sc.pref = s_pref; sc.ctx = s_ctx; sc.kd = s_kd;
+  sc.B = p.B; sc.Hkv = p.Hkv; sc.G = p.G; sc.RB = p.RB; sc.E = p.unit_cost; sc.num_ctas = p.num_ctas;
+  // Warp 0: the prefix of costs over sequences, then this CTA's range and
+  // first segment (every role starts from it), all lanes together.
+  SegInfo *s_seg0 = reinterpret_cast<SegInfo *>(smem + Smem::SEG0);
+  CtaRange *s_range = reinterpret_cast<CtaRange *>(smem + Smem::RANGE);
+  if (warp == 0) {
+    sched_scan(p, sc, s_pref, lane);
+    __syncwarp();
+    Sched s0 = sc;
+    s0.total = s_pref[p.B];
+    // Never more CTAs than slices: every CTA kept has a non-empty range, so
+    // the CTAs between a unit's first and last owner all contribute a partial.
+    s0.num_ctas = static_cast<int>(s0.total < p.num_ctas ? s0.total : p.num_ctas);
+    CtaRange r;
+    r.total = s0.total;
+    r.num_ctas = s0.num_ctas;
+    r.active = s0.total > 0 && static_cast<int>(blockIdx.x) < s0.num_ctas;
+    r.x_begin = r.x_end = 0;
+    SegInfo seg0{};
+    if (r.active) {
+      r.x_begin = div_nn(static_cast<int64_t>(blockIdx.x) * s0.total, s0.num_ctas);
+      r.x_end = div_nn(static_cast<int64_t>(blockIdx.x + 1) * s0.total, s0.num_ctas);
+      seg0 = next_seg_warp(s0, r.x_begin, r.x_end, lane);
+    }
+    if (lane == 0) {
+      *s_range = r;
+      *s_seg0 = seg0;
+    }
+  }
+  block_sync();
+  const CtaRange rng = *s_range;
+  sc.total = rng.total;
+  sc.num_ctas = rng.num_ctas;
+  if (!rng.active) {
     if (warp == 1) tmem_dealloc(*s_tmem, kTmemCols);
     return;
   }
-  const int64_t x_begin = static_cast<int64_t>(blockIdx.x) * sc.total / sc.num_ctas;
-  const int64_t x_end = static_cast<int64_t>(blockIdx.x + 1) * sc.total / sc.num_ctas;
+  const int64_t x_begin = rng.x_begin;
+  const int64_t x_end = rng.x_end;
   const SegInfo seg0 = *s_seg0;
   const uint32_t tmem = *s_tmem;
   const uint32_t smem_base = smem_u32(smem);
@@ -701,8 +727,20 @@ static cudaError_t launch_nr(const Params &p, const CUtensorMap &k2, const CUten
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  kern<<<p.num_ctas, kThreads, Smem::BYTES, stream>>>(p, k2, v2, k1, v1);
-  return cudaGetLastError();
+  // Programmatic dependent launch: the kernel's input-free set-up may overlap
+  // the previous kernel in the stream (the kernel waits for it before reading
+  // any input).
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.num_ctas);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = Smem::BYTES;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, p, k2, v2, k1, v1);
 }
 
 }  // namespace tc
