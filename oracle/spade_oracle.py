@@ -18,6 +18,11 @@ What it computes (the verifier side of one speculative-decoding iteration):
   the longest accepted prefix and the correction token (Algorithm 1).
 * ``kv_commit`` -- the context update m <- m + k + 1 of Algorithm 1 applied to
   a KV cache: accepted slots stay, rejected slots are cleared.
+* ``verify_qkv_rope`` / ``kv_write`` -- the projection of the verify block's
+  hidden states into queries, keys and values with rotary position embedding,
+  and the write of its keys and values into the block's cache slots: the
+  attention input side of f_l in x_{l+1} = x_l + f_l(x_l) (Sec. III-A) for the
+  d+1 positions of the single forward pass (Sec. III-B).
 
 Readings taken where the paper is silent (each also listed in the design
 notes): greedy verification accepts a draft iff it equals the verifier's
@@ -25,7 +30,11 @@ argmax (lowest index on ties); the uniform u of position i decides acceptance
 iff u < p/q (q(d) = 0 accepts iff p(d) > 0); when every draft is accepted a
 bonus token is drawn from p of the last row; sampling is the inverse CDF in
 ascending vocabulary order, the first x whose cumulative mass exceeds u*Z; a
-residual with no positive finite mass falls back to p.
+residual with no positive finite mass falls back to p.  Rotary embedding (the
+verifier family's positional encoding; the paper names the model, Sec. IV,
+not its layers) pairs dimension j with j + D/2 and rotates the pair by
+pos * theta^(-2j/D), counter-clockwise; verify position i of sequence b sits
+at position ctx_b + i.
 
 Inputs are numpy arrays.  Floating inputs are the exact values of the bf16 /
 fp32 tensors handed to the GPU, converted to float64 before any arithmetic.
@@ -256,3 +265,65 @@ def kv_commit(k_cache, v_cache, ctx_lens, accepted_len, n_draft):
         v[b, :, lo:hi] = 0
         ctx[b] = lo
     return k, v, ctx
+
+
+# ----------------------------------------------------------------------------
+# QKV projection + rotary embedding of the verify block (Sec. III-A/III-B)
+# ----------------------------------------------------------------------------
+def rope_inv_freq(D, theta):
+    """Rotary frequencies theta^(-2j/D), j = 0 .. D/2 - 1."""
+    return float(theta) ** (-2.0 * np.arange(D // 2) / D)
+
+
+def rope(x, pos, theta):
+    """Rotary position embedding of vectors x [..., D] at positions pos (broadcast to
+    x.shape[:-1]): the pair (x_j, x_{j+D/2}) is rotated counter-clockwise by the angle
+    pos * theta^(-2j/D)."""
+    x = _f64(x)
+    h = x.shape[-1] // 2
+    ang = np.asarray(pos, dtype=np.float64)[..., None] * rope_inv_freq(x.shape[-1], theta)
+    c, s = np.cos(ang), np.sin(ang)
+    a, b = x[..., :h], x[..., h:]
+    return np.concatenate([a * c - b * s, b * c + a * s], axis=-1)
+
+
+def verify_positions(ctx_lens, n_draft, cu_q):
+    """(sequence, position) of every verify row: row cu_q[b] + i is position ctx_b + i."""
+    R = int(cu_q[len(n_draft)])
+    seq = np.empty(R, dtype=np.int64)
+    pos = np.empty(R, dtype=np.int64)
+    for b in range(len(n_draft)):
+        for i in range(int(n_draft[b]) + 1):
+            seq[int(cu_q[b]) + i] = b
+            pos[int(cu_q[b]) + i] = int(ctx_lens[b]) + i
+    return seq, pos
+
+
+def verify_qkv_rope(x, w_qkv, ctx_lens, n_draft, cu_q, Hq, Hkv, theta):
+    """Queries, keys and values of the verify block.
+
+    x [R, H] hidden states of the verify rows; w_qkv [(Hq + 2 Hkv) D, H] (nn.Linear
+    layout: the query heads' rows, then the key heads', then the value heads').
+    y = x W^T; q and k are rotated at each row's position (ctx_b + i), v is not.
+    Returns (q [R, Hq, D], k [R, Hkv, D], v [R, Hkv, D]) in float64.
+    """
+    y = _f64(x) @ _f64(w_qkv).T
+    R = y.shape[0]
+    D = w_qkv.shape[0] // (Hq + 2 * Hkv)
+    q = y[:, :Hq * D].reshape(R, Hq, D)
+    k = y[:, Hq * D:(Hq + Hkv) * D].reshape(R, Hkv, D)
+    v = y[:, (Hq + Hkv) * D:].reshape(R, Hkv, D)
+    _, pos = verify_positions(ctx_lens, n_draft, cu_q)
+    return rope(q, pos[:, None], theta), rope(k, pos[:, None], theta), v
+
+
+def kv_write(k_cache, v_cache, k, v, ctx_lens, n_draft, cu_q):
+    """Writes the verify block's keys and values into cache slots ctx_b .. ctx_b + k_b
+    of their sequence (every KV head); returns new (k_cache, v_cache) copies."""
+    kc = np.array(k_cache, dtype=np.float64, copy=True)
+    vc = np.array(v_cache, dtype=np.float64, copy=True)
+    seq, pos = verify_positions(ctx_lens, n_draft, cu_q)
+    for r in range(len(seq)):
+        kc[seq[r], :, pos[r]] = k[r]
+        vc[seq[r], :, pos[r]] = v[r]
+    return kc, vc

@@ -373,10 +373,94 @@ def check_kv_commit(o, seed=9):
                 assert (k2[b, :, s] == kc[b, :, s]).all() and (v2[b, :, s] == vc[b, :, s]).all()
 
 
+# ----------------------------------------------------------------------------
+# QKV projection + rotary embedding of the verify block
+# ----------------------------------------------------------------------------
+def check_rope_worked_examples(o):
+    g = _golden()["rope"]
+    theta = 4.0 / math.pi ** 2
+    x = np.asarray(g["x"])
+    for ex in g["cases"]:
+        y = o.rope(x, ex["pos"], theta)
+        np.testing.assert_allclose(y[[1, 3]], ex["pair13"], rtol=0, atol=1e-12, err_msg=ex["why"])
+        # The first pair keeps its length and turns by pos radians.
+        assert abs(y[0] ** 2 + y[2] ** 2 - (x[0] ** 2 + x[2] ** 2)) < 1e-12
+        turn = math.atan2(y[2], y[0]) - math.atan2(x[2], x[0])
+        assert abs(math.remainder(turn - ex["pair02_angle"], 2 * math.pi)) < 1e-12, ex["why"]
+
+
+def check_rope_vs_complex_rotation(o, seed=10):
+    """The same rotation written as a complex product in torch float64: z_j = x_j + i x_{j+D/2}
+    times exp(i pos / theta^(2j/D))."""
+    rng = np.random.default_rng(seed)
+    for D, theta in ((8, 10000.0), (64, 500000.0), (128, 10000.0)):
+        x = rng.standard_normal((5, 3, D))
+        pos = rng.integers(0, 40000, size=(5, 3))
+        got = o.rope(x, pos, theta)
+        xt = torch.from_numpy(x)
+        inv = 1.0 / (theta ** (torch.arange(0, D, 2, dtype=torch.float64) / D))
+        ang = torch.from_numpy(pos).to(torch.float64)[..., None] * inv
+        z = torch.complex(xt[..., :D // 2], xt[..., D // 2:]) * torch.polar(torch.ones_like(ang), ang)
+        ref = torch.cat([z.real, z.imag], dim=-1).numpy()
+        np.testing.assert_allclose(got, ref, rtol=1e-9, atol=1e-9)
+
+
+def check_rope_relative_position(o, seed=11):
+    """<rope(q, m), rope(k, n)> depends on m - n only."""
+    rng = np.random.default_rng(seed)
+    q, k = rng.standard_normal(64), rng.standard_normal(64)
+    for m, n, t in ((5, 2, 100), (0, 9, 7), (1000, 10, 31)):
+        a = o.rope(q, m, 10000.0) @ o.rope(k, n, 10000.0)
+        b = o.rope(q, m + t, 10000.0) @ o.rope(k, n + t, 10000.0)
+        assert abs(a - b) < 1e-9 * (1 + abs(a))
+    assert abs(o.rope(q, 3, 10000.0) @ o.rope(k, 0, 10000.0) - q @ k) > 1e-6  # not trivially constant
+
+
+def check_qkv_projection_layout(o, seed=12):
+    """One-hot hidden rows pick columns of W^T; rows of W split q | k | v by head; only q and k
+    turn (v at any position equals the projection), and row i sits at position ctx + i."""
+    rng = np.random.default_rng(seed)
+    Hq, Hkv, D, H = 2, 1, 4, 6
+    W = rng.standard_normal(((Hq + 2 * Hkv) * D, H))
+    x = np.eye(H)[[0, 3, 5]]
+    ctx, kd, cu = [7], [2], [0, 3]
+    q, k, v = o.verify_qkv_rope(x, W, ctx, kd, cu, Hq, Hkv, 10000.0)
+    y = W.T[[0, 3, 5]]
+    np.testing.assert_array_equal(v.reshape(3, -1), y[:, (Hq + Hkv) * D:])
+    for i in range(3):
+        for h in range(Hq):
+            np.testing.assert_allclose(q[i, h], o.rope(y[i, h * D:(h + 1) * D], 7 + i, 10000.0), rtol=0, atol=1e-12)
+        np.testing.assert_allclose(k[i, 0], o.rope(y[i, Hq * D:(Hq + 1) * D], 7 + i, 10000.0), rtol=0, atol=1e-12)
+    # Norms of q per head are those of the projection (a rotation).
+    np.testing.assert_allclose(np.linalg.norm(q, axis=-1), np.linalg.norm(y[:, :Hq * D].reshape(3, Hq, D), axis=-1),
+                               rtol=1e-12)
+
+
+def check_kv_write_slots(o):
+    g = _golden()["qkv_write"]
+    B, Hkv, cap, D = 2, 2, 6, 3
+    kc = np.full((B, Hkv, cap, D), -1.0)
+    vc = np.full((B, Hkv, cap, D), -2.0)
+    R = g["cu_q"][-1]
+    k = np.arange(R * Hkv * D, dtype=np.float64).reshape(R, Hkv, D)
+    v = k + 1000.0
+    k2, v2 = o.kv_write(kc, vc, k, v, g["ctx"], g["k"], g["cu_q"])
+    written = set()
+    for r, (b, slot) in enumerate(g["slots"]):
+        np.testing.assert_array_equal(k2[b, :, slot], k[r])
+        np.testing.assert_array_equal(v2[b, :, slot], v[r])
+        written.add((b, slot))
+    for b in range(B):
+        for slot in range(cap):
+            if (b, slot) not in written:
+                assert (k2[b, :, slot] == -1.0).all() and (v2[b, :, slot] == -2.0).all()
+
+
 ALL_CHECKS = [
     check_attention_worked_examples, check_attention_vs_sdpa, check_attention_special_cases,
     check_attention_gqa_mapping, check_logits_one_hot, check_acceptance_worked_examples,
     check_margin_worked_examples, check_residual_properties, check_q_equals_p_accepts_all, check_strict_comparison,
     check_stochastic_output_law, check_progress_and_bounds, check_greedy_identity,
-    check_kv_commit,
+    check_kv_commit, check_rope_worked_examples, check_rope_vs_complex_rotation,
+    check_rope_relative_position, check_qkv_projection_layout, check_kv_write_slots,
 ]

@@ -46,6 +46,20 @@ MUTANTS = {
     "flag_rows_after_rejection": ("            if not ok:\n                break",
                                   "            if not ok:\n                flag_dec[b] |= any(abs(float(uniforms[r0 + j]) - 0.5) "
                                   "< margin for j in range(i + 1, k))\n                break"),
+    # Rotary embedding and the QKV projection of the verify block.
+    "rope_interleaved_pairs": ("a, b = x[..., :h], x[..., h:]", "a, b = x[..., 0::2], x[..., 1::2]"),
+    "rope_clockwise": ("return np.concatenate([a * c - b * s, b * c + a * s], axis=-1)",
+                       "return np.concatenate([a * c + b * s, b * c - a * s], axis=-1)"),
+    "rope_exponent_j_over_D": ("return float(theta) ** (-2.0 * np.arange(D // 2) / D)",
+                               "return float(theta) ** (-1.0 * np.arange(D // 2) / D)"),
+    "rope_position_off_by_one": ("pos[int(cu_q[b]) + i] = int(ctx_lens[b]) + i",
+                                 "pos[int(cu_q[b]) + i] = int(ctx_lens[b]) + i + 1"),
+    "qkv_split_k_before_q": ("q = y[:, :Hq * D].reshape(R, Hq, D)", "q = y[:, Hkv * D:(Hq + Hkv) * D].reshape(R, Hq, D)"),
+    "values_rotated": ("return rope(q, pos[:, None], theta), rope(k, pos[:, None], theta), v",
+                       "return rope(q, pos[:, None], theta), rope(k, pos[:, None], theta), rope(v, pos[:, None], theta)"),
+    "keys_not_rotated": ("return rope(q, pos[:, None], theta), rope(k, pos[:, None], theta), v",
+                         "return rope(q, pos[:, None], theta), k, v"),
+    "kv_write_wrong_slot": ("kc[seq[r], :, pos[r]] = k[r]", "kc[seq[r], :, pos[r] - 1] = k[r]"),
 }
 
 
