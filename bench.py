@@ -405,6 +405,8 @@ def run_spade(args, ws, rank, local):
                 ev1[i - 3][1].record(stream)
         torch.cuda.synchronize()
         pass1 = statistics.median(a.elapsed_time(b) * 1e-3 for a, b in ev1)
+    wl["ctx_lens"].copy_(ctx0)  # the step's commits advanced it
+    qkv = _time_qkv(spec, wl, dev, flush_buf)
     hbm, bf16, bf16_sus, peak_src = _peaks()
     m_acc = statistics.mean(t_acc)
     m_attn = statistics.mean(t_attn)
@@ -433,6 +435,8 @@ def run_spade(args, ws, rank, local):
         "wall_s_timed_loop": t_wall,
         "clocks": clk.summary(),
     }
+    if qkv is not None:
+        line["qkv_rope"] = qkv
     if pass1 is not None:
         line["lm_head_pass1"] = {"us": pass1 * 1e6, "tensor_tflops": lm_flop / pass1 / 1e12,
                                  "frac_of_sustained_bf16": lm_flop / pass1 / 1e12 / bf16_sus,
@@ -448,6 +452,43 @@ def run_spade(args, ws, rank, local):
 
 
 # ---------------------------------------------------------------------------
+def _time_qkv(spec, wl, dev, flush_buf=None, launches=20):
+    """The verify block's QKV projection + rotary embedding (writes the K/V of the verify
+    slots, as the step's attention expects them): median CUDA-event time per launch, L2
+    flushed before each launch (W of a layer fits in L2), and its HBM roofline."""
+    import paper_2608_13076_gb300 as spade
+
+    x, w = W.make_qkv_inputs(spec, wl["R"], device=dev)
+    q = torch.empty((wl["R"], wl["Hq"], wl["D"]), dtype=torch.bfloat16, device=dev)
+    status = spade.status_tensor(dev)
+    if flush_buf is None:
+        flush_buf = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+    kc, vc = wl["k_cache"].clone(), wl["v_cache"].clone()  # the step's caches stay as they were
+    stream = torch.cuda.current_stream()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(launches)]
+    for i in range(launches + 3):
+        flush_buf.zero_()
+        if i >= 3:
+            ev[i - 3][0].record(stream)
+        spade.spade_verify_qkv_rope(x, w, wl["ctx_lens"], wl["n_draft"], wl["cu_q"], q, kc, vc, Hq=wl["Hq"],
+                                    Hkv=wl["Hkv"], rope_theta=spec.rope_theta, max_k=int(wl["n_draft"].max()),
+                                    status=status)
+        if i >= 3:
+            ev[i - 3][1].record(stream)
+    torch.cuda.synchronize()
+    if int(status.item()):
+        raise RuntimeError(f"qkv_rope device status {int(status.item())}")
+    t = statistics.median(a.elapsed_time(b) * 1e-3 for a, b in ev)
+    hbm = _peaks()[0]
+    R, H, Hq, Hkv, D = wl["R"], wl["H"], wl["Hq"], wl["Hkv"], wl["D"]
+    nbytes = (Hq + 2 * Hkv) * D * H * 2 + R * H * 2 + R * (Hq + 2 * Hkv) * D * 2
+    flop = 2.0 * R * (Hq + 2 * Hkv) * D * H
+    return {"kernel": "qkv_rope_kernel", "us": t * 1e6, "bound": "hbm", "achieved": nbytes / t / 1e9, "peak": hbm,
+            "unit": "GB/s", "frac": nbytes / t / 1e9 / hbm, "algorithmic_bytes": nbytes, "tflops": flop / t / 1e12,
+            "launches": launches, "l2": "flushed before each launch",
+            "note": "not part of the timed step (the step's q and cache slots are inputs); measured after it"}
+
+
 def _time_step(wl, dev, steps, warmup):
     """Device time of the step (attention, then accept + commit) on one workload."""
     import paper_2608_13076_gb300 as spade
@@ -486,6 +527,7 @@ def _time_step(wl, dev, steps, warmup):
     torch.cuda.synchronize()
     if int(status.item()) & ~spade.DEV_FALLBACK:
         raise RuntimeError(f"device status {int(status.item())} on {wl['spec'].name}")
+    wl["ctx_lens"].copy_(ctx0)  # the commits advanced it
     t_attn = statistics.median(e[0].elapsed_time(e[1]) * 1e-3 for e in evs)
     t_acc = statistics.median(e[1].elapsed_time(e[2]) * 1e-3 for e in evs)
     return t_attn, t_acc, int((acc.long() + 1).sum().item()), acc.tolist()
@@ -501,12 +543,14 @@ def per_workload(args, dev, skip):
         wl = _to_device(W.make_workload(spec, device="cpu"), dev)
         attn_bytes, lm_bytes, lm_flop, _, _ = _work_bytes(wl)
         t_attn, t_acc, toks, acc = _time_step(wl, dev, args.per_workload_steps, 3)
+        qkv = _time_qkv(spec, wl, dev, launches=10)
         lm = _lm_roofline(lm_bytes, lm_flop, t_acc, hbm, bf16_sus, bf16, peak_src)
         res[name] = {"tokens_per_s": toks / (t_attn + t_acc), "us_per_step": (t_attn + t_acc) * 1e6,
                      "tokens_per_step": toks, "accepted_len": acc,
                      "verify_attention_us": t_attn * 1e6, "attention_hbm_frac": attn_bytes / t_attn / 1e9 / hbm,
                      "verify_accept_commit_us": t_acc * 1e6, "lm_head_bound": lm["bound"],
                      "lm_head_frac": lm["frac"], "lm_head_tensor_frac_of_sustained": lm["tensor"]["frac_of_sustained"],
+                     "qkv_rope_us": qkv["us"], "qkv_rope_hbm_frac": qkv["frac"],
                      "steps": args.per_workload_steps, "timing": "median of CUDA-event times per launch"}
         del wl
         torch.cuda.empty_cache()

@@ -16,6 +16,9 @@
  *   spade_kv_commit         context update m <- m + a + 1 (Algorithm 1) on the
  *                           KV cache: keep accepted slots, clear rejected ones
  *   spade_verify_accept_commit  the two calls above fused into one launch
+ *   spade_verify_qkv_rope   the verify block's QKV projection with rotary
+ *                           embedding, writing its K/V into the cache slots
+ *                           the attention reads
  *
  * Conventions shared by every call
  *  - Every pointer argument is a DEVICE pointer owned by the caller; the
@@ -64,6 +67,47 @@ typedef enum {
 #define SPADE_DEV_CAPACITY  0x2  /* ctx_lens[b] + n_draft[b] + 1 > cap                       */
 #define SPADE_DEV_TIMEOUT   0x4  /* a bounded device-side wait expired; outputs are invalid  */
 #define SPADE_DEV_FALLBACK  0x8  /* a residual had no positive mass; p was sampled instead   */
+
+/* ------------------------------------------------------------------------ */
+/* QKV projection + rotary embedding of the verify block (Sec. III-A/III-B)  */
+/* ------------------------------------------------------------------------ */
+/*
+ * The verifier's projection of the verify block's hidden states into queries,
+ * keys and values -- the input side of the attention in x_{l+1} = x_l +
+ * f_l(x_l) (Sec. III-A) for the d+1 positions scored in the single forward
+ * pass (Sec. III-B) -- with rotary position embedding, writing the block's
+ * keys and values into its cache slots, ready for spade_verify_attention:
+ *   y = x W^T (fp32 accumulation on the tensor cores), split into the head
+ *   slices q_h (h < Hq), k_g, v_g (g < Hkv);
+ *   q and k are rotated at the row's position pos = ctx_lens[b] + i (row
+ *   cu_q[b] + i): the pair (dimension j, j + D/2) turns counter-clockwise by
+ *   pos * rope_theta^(-2j/D); v is not rotated;
+ *   q_out[cu_q[b]+i, h, :] = q_h, k_cache[b, g, ctx_b+i, :] = k_g and
+ *   v_cache[b, g, ctx_b+i, :] = v_g, rounded to bf16.
+ *
+ *   x           bf16 [R, H] row-major (the verify rows' hidden states), H % 8 == 0
+ *   w_qkv       bf16 [(Hq + 2 Hkv) D, H] row-major (nn.Linear layout): the query
+ *               heads' rows, then the key heads', then the value heads';
+ *               (Hq + 2 Hkv) * D a multiple of 128
+ *   ctx_lens, n_draft, cu_q   int32 [B], [B], [B+1], as for the attention
+ *   q_out       bf16 [R, Hq, D] written
+ *   k_cache, v_cache  bf16 [B, Hkv, cap, D]: slots [ctx_b, ctx_b + n_draft[b]]
+ *               written, every other slot left as it is
+ *   B, R, H, Hq, Hkv, D, cap, max_k   sizes; D in {64, 128}; R <= 512
+ *   rope_theta  base of the rotary frequencies (10000 for Llama-2, 500000 for
+ *               Llama-3), finite and > 1
+ *   status      device int32: a sequence whose block is invalid
+ *               (SPADE_DEV_BAD_INDEX) or does not fit its cache
+ *               (SPADE_DEV_CAPACITY) is skipped; none of its rows is written
+ * Every pointer is a 16-byte aligned device pointer.  Allocates nothing and
+ * needs no workspace: the split-K partial sums meet in distributed shared
+ * memory inside the launch.  Launched with programmatic dependent launch.
+ */
+spade_status spade_verify_qkv_rope(const void *x, const void *w_qkv, const int32_t *ctx_lens,
+                                   const int32_t *n_draft, const int32_t *cu_q, void *q_out,
+                                   void *k_cache, void *v_cache, int32_t B, int32_t R, int32_t H,
+                                   int32_t Hq, int32_t Hkv, int32_t D, int32_t cap, int32_t max_k,
+                                   float rope_theta, int32_t *status, spade_stream_t stream);
 
 /* ------------------------------------------------------------------------ */
 /* Verify attention (Sec. III-B verification stage; Algorithm 1 cloud step)  */

@@ -10,6 +10,7 @@ Entry points (same names as the C ABI in include/spade.h):
     spade_verify_attention  verify-position attention against the KV cache
     spade_verify_accept     LM head + softmax + accept/reject + residual sampling
     spade_kv_commit         append accepted positions, roll back rejected ones
+    spade_verify_qkv_rope   QKV projection + rotary embedding of the verify block, K/V into the cache
 """
 from __future__ import annotations
 
@@ -23,6 +24,7 @@ from . import _build
 __all__ = [
     "SpadeError", "load", "build", "library_path",
     "spade_verify_attention", "spade_verify_accept", "spade_kv_commit", "spade_verify_attention_noalloc",
+    "spade_verify_qkv_rope",
     "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_accept_launches",
     "spade_accept_stats_layout", "read_accept_stats", "spade_verify_accept_commit", "spade_selftest_wait_timeout",
     "attn_workspace", "accept_workspace", "status_tensor", "check_status",
@@ -88,6 +90,8 @@ def load():
     lib.spade_accept_launches.argtypes = [_i32] * 4
     lib.spade_selftest_wait_timeout.restype = _i32
     lib.spade_selftest_wait_timeout.argtypes = [_vp, _i32, _vp]
+    lib.spade_verify_qkv_rope.restype = _i32
+    lib.spade_verify_qkv_rope.argtypes = [_vp] * 8 + [_i32] * 8 + [ctypes.c_float, _vp, _vp]
     lib.spade_kv_commit.restype = _i32
     lib.spade_kv_commit.argtypes = [_vp] * 5 + [_i32] * 4 + [_vp, _vp]
     lib.spade_status_string.restype = ctypes.c_char_p
@@ -307,6 +311,30 @@ def spade_verify_accept_commit(hidden, w_lm, draft_tokens, draft_probs, uniforms
         _stream(stream))
     _check_rc(rc)
     return accepted_len, next_token
+
+
+# ---------------------------------------------------------------------------
+def spade_verify_qkv_rope(x, w_qkv, ctx_lens, n_draft, cu_q, q_out, k_cache, v_cache, *, Hq, Hkv,
+                          rope_theta, max_k, status, stream=None):
+    """q, k, v of the verify block (rotary embedding at ctx + i); K/V into cache slots ctx .. ctx + k."""
+    _need(x, "x", torch.bfloat16, 2)
+    _need(w_qkv, "w_qkv", torch.bfloat16, 2)
+    _need(q_out, "q_out", torch.bfloat16, 3)
+    _need(k_cache, "k_cache", torch.bfloat16, 4)
+    _need(v_cache, "v_cache", torch.bfloat16, 4)
+    for t, n in ((ctx_lens, "ctx_lens"), (n_draft, "n_draft"), (cu_q, "cu_q"), (status, "status")):
+        _need(t, n, torch.int32, 1)
+    R, H = x.shape
+    B, Hkv2, cap, D = k_cache.shape
+    if Hkv2 != Hkv or tuple(v_cache.shape) != tuple(k_cache.shape) or tuple(q_out.shape) != (R, Hq, D) \
+            or tuple(w_qkv.shape) != ((Hq + 2 * Hkv) * D, H) or ctx_lens.numel() != B or n_draft.numel() != B \
+            or cu_q.numel() != B + 1:
+        raise ValueError("inconsistent qkv_rope shapes")
+    rc = load().spade_verify_qkv_rope(
+        _ptr(x), _ptr(w_qkv), _ptr(ctx_lens), _ptr(n_draft), _ptr(cu_q), _ptr(q_out), _ptr(k_cache), _ptr(v_cache),
+        B, R, H, Hq, Hkv, D, cap, int(max_k), float(rope_theta), _ptr(status), _stream(stream))
+    _check_rc(rc)
+    return q_out
 
 
 # ---------------------------------------------------------------------------

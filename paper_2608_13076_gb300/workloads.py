@@ -45,6 +45,7 @@ class WorkloadSpec:
     target_accept: float = 0.0  # stochastic: if > 0, tune noise so mean sum(min(p,q)) hits it
     greedy_draft: str = "match" # greedy drafts: "match" (match_prob) or "noisy_argmax"
     seed: int = 0
+    rope_theta: float = 10000.0  # base of the rotary frequencies of the model family
     extra: dict = field(default_factory=dict)
 
 
@@ -61,13 +62,13 @@ SPECS = {
                                          mode="stochastic", noise=0.5, seed=2002),
     "llama3_8b": WorkloadSpec("llama3_8b", B=8, Hq=32, Hkv=8, D=128, H=4096, V=128256,
                               ctx=(4096, 4096), k=(8, 8), mode="stochastic",
-                              target_accept=0.7, seed=1003),
+                              target_accept=0.7, seed=1003, rope_theta=500000.0),
     "long_70b": WorkloadSpec("long_70b", B=4, Hq=64, Hkv=8, D=128, H=8192, V=32000,
                              ctx=(32768, 32768), k=(4, 4), mode="greedy", match_prob=0.6,
-                             seed=1004),
+                             seed=1004, rope_theta=500000.0),
     "ragged": WorkloadSpec("ragged", B=64, Hq=40, Hkv=8, D=128, H=5120, V=152064,
                            ctx=(128, 8192), k=(1, 10), mode="mixed", match_prob=0.7,
-                           noise=0.5, seed=1005),
+                           noise=0.5, seed=1005, rope_theta=1000000.0),
 }
 
 
@@ -203,3 +204,13 @@ def make_workload(spec: WorkloadSpec, device="cpu", cache_pad: int = 0):
         draft_tokens=mv(drafts.to(torch.int32)), draft_probs=mv(draft_probs),
         uniforms=mv(uniforms), mode=mv(mode), sigma=sigma,
     )
+
+
+def make_qkv_inputs(spec: WorkloadSpec, R: int, device="cpu"):
+    """Inputs of the verify block's QKV projection: hidden states x [R, H] ~ N(0, 1) and
+    w_qkv [(Hq + 2 Hkv) D, H] ~ N(0, 1/H) in bf16 (so q, k, v ~ N(0, 1)), drawn on the CPU
+    from their own seed (the spec's + 500) and moved to ``device``."""
+    gen = torch.Generator(device="cpu").manual_seed(spec.seed + 500)
+    x = _bf16_normal(gen, (R, spec.H), 1.0, "cpu")
+    w = _bf16_normal(gen, ((spec.Hq + 2 * spec.Hkv) * spec.D, spec.H), 1.0 / math.sqrt(spec.H), "cpu")
+    return x.to(device), w.to(device)

@@ -199,6 +199,51 @@ def check_commit_windows(wl_before, k_after, v_after, ctx_after, acc):
     return B
 
 
+def gpu_qkv_rope(wl, x, w, q_out=None, status=None):
+    """The QKV projection + rotary embedding call (writes wl's caches in place)."""
+    dev = x.device
+    if q_out is None:
+        q_out = torch.full((wl["R"], wl["Hq"], wl["D"]), float("nan"), dtype=torch.bfloat16, device=dev)
+    if status is None:
+        status = spade.status_tensor(dev)
+    spade.spade_verify_qkv_rope(x, w, wl["ctx_lens"], wl["n_draft"], wl["cu_q"], q_out, wl["k_cache"],
+                                wl["v_cache"], Hq=wl["Hq"], Hkv=wl["Hkv"], rope_theta=wl["spec"].rope_theta,
+                                max_k=int(wl["n_draft"].max()), status=status)
+    return q_out, status
+
+
+def check_qkv_rope(wl, x, w, q_gpu, k_before, v_before, skip=()):
+    """q, and the K/V written into the verify slots, against ``O.verify_qkv_rope`` (the
+    attention rule per (row, head) vector); every other cache slot unchanged bit for bit.
+    Sequences in ``skip`` must be left entirely untouched (q rows still NaN).
+    Returns the worst tolerance ratio over q, k and v."""
+    ctx, kd, cu = to_np(wl["ctx_lens"]), to_np(wl["n_draft"]), to_np(wl["cu_q"])
+    q_ref, k_ref, v_ref = O.verify_qkv_rope(to_np(x), to_np(w), ctx, kd, cu, wl["Hq"], wl["Hkv"],
+                                            wl["spec"].rope_theta)
+    seq, pos = O.verify_positions(ctx, kd, cu)
+    keep = np.array([s not in skip for s in seq])
+    rows = [(r, h) for r in np.nonzero(keep)[0] for h in range(wl["Hq"])]
+    worst = 0.0
+    n, bad, wq = compare_attention(q_gpu, q_ref, rows=rows)
+    assert bad == 0, f"q: {bad} bad elements, worst {wq:.3g}"
+    worst = max(worst, wq)
+    dev = q_gpu.device
+    si = torch.from_numpy(seq[keep]).to(dev)
+    pi = torch.from_numpy(pos[keep]).to(dev)
+    for cache, before, ref, nm in ((wl["k_cache"], k_before, k_ref, "k"), (wl["v_cache"], v_before, v_ref, "v")):
+        got = cache[si, :, pi]  # [rows, Hkv, D]
+        kv_rows = [(r, g) for r in range(int(keep.sum())) for g in range(wl["Hkv"])]
+        n, bad, wk = compare_attention(got, ref[keep], rows=kv_rows)
+        assert bad == 0, f"{nm}: {bad} bad elements, worst {wk:.3g}"
+        worst = max(worst, wk)
+        expect = before.clone()
+        expect[si, :, pi] = cache[si, :, pi]
+        assert torch.equal(expect, cache), f"{nm} cache changed outside the verify slots"
+    if skip:
+        assert torch.isnan(q_gpu[torch.from_numpy(~keep).to(dev)].float()).all()
+    return worst
+
+
 def compare_accept(acc_gpu, tok_gpu, ref):
     """Bit-exact accept decisions outside flagged margins.
 

@@ -412,3 +412,68 @@ def test_long_greedy_sequence_in_two_pass_batch(dev):
     assert parity.compare_accept(acc, tok, ref)["mismatch_unflagged"] == 0
     assert int(ref["accepted_len"][0]) >= 30  # the greedy sequence b = 0 accepts deep
     parity.check_commit_windows(before, wl["k_cache"], wl["v_cache"], wl["ctx_lens"], acc)
+
+
+# ---------------------------------------------------------------------------
+# QKV projection + rotary embedding of the verify block (writes its K/V slots).
+
+QKV_SMALL = {
+    "qkv_gqa_d128": W.WorkloadSpec("qkv_gqa_d128", B=3, Hq=8, Hkv=2, D=128, H=520, V=1000, ctx=(50, 700),
+                                   k=(0, 7), mode="greedy", seed=51, rope_theta=500000.0),
+    "qkv_d64_ragged_k": W.WorkloadSpec("qkv_d64_ragged_k", B=5, Hq=6, Hkv=2, D=64, H=200, V=1000, ctx=(0, 300),
+                                       k=(1, 9), mode="greedy", seed=52),
+    "qkv_many_rows": W.WorkloadSpec("qkv_many_rows", B=40, Hq=4, Hkv=2, D=128, H=256, V=1000, ctx=(5, 3000),
+                                    k=(6, 9), mode="greedy", seed=53, rope_theta=1000000.0),
+}
+
+
+@pytest.mark.parametrize("name", sorted(QKV_SMALL) + FULL)
+def test_qkv_rope(dev, name):
+    spec = QKV_SMALL[name] if name in QKV_SMALL else W.SPECS[name]
+    wl = W.make_workload(spec, device=dev, cache_pad=3)
+    x, w = W.make_qkv_inputs(spec, wl["R"], device=dev)
+    k0, v0 = wl["k_cache"].clone(), wl["v_cache"].clone()
+    q, st = parity.gpu_qkv_rope(wl, x, w)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    worst = parity.check_qkv_rope(wl, x, w, q, k0, v0)
+    print(f"{name}: worst {worst:.3g} of tolerance")
+
+
+def test_qkv_rope_skips_invalid_sequences(dev):
+    """A sequence whose block does not fit its cache is reported and left untouched."""
+    spec = QKV_SMALL["qkv_gqa_d128"]
+    wl = W.make_workload(spec, device=dev)
+    wl["ctx_lens"][1] = wl["cap"]  # ctx + k + 1 > cap
+    x, w = W.make_qkv_inputs(spec, wl["R"], device=dev)
+    k0, v0 = wl["k_cache"].clone(), wl["v_cache"].clone()
+    q, st = parity.gpu_qkv_rope(wl, x, w)
+    torch.cuda.synchronize()
+    assert int(st.item()) == spade.DEV_CAPACITY
+    # The oracle is asked only about the valid sequences; sequence 1's slots (beyond its cache)
+    # are not compared, and its rows of q must still hold the NaN they were filled with.
+    ctx = wl["ctx_lens"].clone()
+    wl["ctx_lens"][1] = 0  # a harmless stand-in position for the oracle call; its rows are skipped
+    parity.check_qkv_rope(wl, x, w, q, k0, v0, skip=(1,))
+    wl["ctx_lens"].copy_(ctx)
+
+
+def test_qkv_then_attention_matches_oracle_chain(dev):
+    """The step as a model runs it: the QKV kernel writes the block's K/V, the attention reads
+    them; the attention output matches the oracle's attention over the oracle's q, K, V."""
+    spec = QKV_SMALL["qkv_gqa_d128"]
+    wl = W.make_workload(spec, device=dev)
+    x, w = W.make_qkv_inputs(spec, wl["R"], device=dev)
+    k0, v0 = parity.to_np(wl["k_cache"]), parity.to_np(wl["v_cache"])
+    q, st = parity.gpu_qkv_rope(wl, x, w)
+    wl["q"] = q
+    out, lse, st2 = parity.gpu_attention(wl)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0 and int(st2.item()) == 0
+    ctx, kd, cu = (parity.to_np(wl[k]) for k in ("ctx_lens", "n_draft", "cu_q"))
+    q_ref, k_ref, v_ref = O.verify_qkv_rope(parity.to_np(x), parity.to_np(w), ctx, kd, cu, wl["Hq"], wl["Hkv"],
+                                            spec.rope_theta)
+    kc, vc = O.kv_write(k0, v0, k_ref, v_ref, ctx, kd, cu)
+    ref, _ = O.verify_attention(q_ref, kc, vc, ctx, kd, cu)
+    n, bad, worst = parity.compare_attention(out, ref)
+    assert bad == 0, worst
