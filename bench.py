@@ -89,6 +89,13 @@ def _job_rate(tokens_local, t_local, ws, device):
     return tokens_local / t_local, t_local
 
 
+def _head_start(ms=3.0):
+    """Queues a spin kernel of about `ms` milliseconds so that the host can enqueue the
+    timed launches ahead of the GPU: a timed region must not contain GPU idle time spent
+    waiting for Python to issue the next launch."""
+    torch.cuda._sleep(int(ms * 2.0e6))  # cycles at about 2 GHz
+
+
 def _to_device(wl, dev):
     return {k: (v.to(dev) if isinstance(v, torch.Tensor) else v) for k, v in wl.items()}
 
@@ -274,6 +281,7 @@ def run_spade(args, ws, rank, local):
     torch.cuda.synchronize()
     with Clocks(local) as clk:
         t_wall0 = time.perf_counter()
+        _head_start(3.0)
         for s in range(args.steps):
             wl["ctx_lens"].copy_(ctx0)
             if flush:
@@ -393,6 +401,7 @@ def run_spade(args, ws, rank, local):
         acc_g = torch.zeros_like(acc)
         tok_g = torch.zeros_like(tok)
         ev1 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
+        _head_start(3.0)
         for i in range(13):
             if flush:
                 flush_buf.zero_()
@@ -465,14 +474,22 @@ def _time_qkv(spec, wl, dev, flush_buf=None, launches=20):
         flush_buf = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
     kc, vc = wl["k_cache"].clone(), wl["v_cache"].clone()  # the step's caches stay as they were
     stream = torch.cuda.current_stream()
+    def call():
+        spade.spade_verify_qkv_rope(x, w, wl["ctx_lens"], wl["n_draft"], wl["cu_q"], q, kc, vc, Hq=wl["Hq"],
+                                    Hkv=wl["Hkv"], rope_theta=spec.rope_theta, max_k=int(wl["n_draft"].max()),
+                                    status=status)
+
+    # The first launch of a shape also runs one-time host work (occupancy queries):
+    # finish it before the timed loop, which must not wait on the host.
+    call()
+    torch.cuda.synchronize()
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(launches)]
+    _head_start(3.0)
     for i in range(launches + 3):
         flush_buf.zero_()
         if i >= 3:
             ev[i - 3][0].record(stream)
-        spade.spade_verify_qkv_rope(x, w, wl["ctx_lens"], wl["n_draft"], wl["cu_q"], q, kc, vc, Hq=wl["Hq"],
-                                    Hkv=wl["Hkv"], rope_theta=spec.rope_theta, max_k=int(wl["n_draft"].max()),
-                                    status=status)
+        call()
         if i >= 3:
             ev[i - 3][1].record(stream)
     torch.cuda.synchronize()
@@ -508,6 +525,11 @@ def _time_step(wl, dev, steps, warmup):
     stream = torch.cuda.current_stream()
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
     for s in range(warmup + steps):
+        if s == 1:
+            # The first step of a shape runs one-time host work; the timed steps must not
+            # wait on the host, so the GPU gets a head start after it.
+            torch.cuda.synchronize()
+            _head_start(3.0)
         wl["ctx_lens"].copy_(ctx0)
         if flush:
             flush_buf.zero_()

@@ -243,31 +243,49 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
     cluster_sync();
-    const int items = nc * (kTileM / 2);
+    // Items are (row, 4 consecutive dimension pairs of one head): two float4
+    // loads per split CTA, all issued before any is used.
+    constexpr int kQuads = kTileM / 8;  // quads of pairs per accumulator column
+    const int items = nc * kQuads;
     const int i0 = items * rank / S, i1 = items * (rank + 1) / S;
     for (int it = i0 + tid; it < i1; it += kThreads) {
-      const int col = it / (kTileM / 2), pp = it % (kTileM / 2);
+      const int col = it / kQuads, qd = it % kQuads;
       const int r = c0 + col;
       if (r >= p.R) continue;
       const int b = s_rseq[r];
       if (b < 0) continue;
-      const int hloc = pp / half, j = pp % half;
-      const int d1 = hloc * p.D + j;
+      const int pp = qd * 4;  // first pair of the quad
+      const int hloc = pp / half, j0 = pp % half;
+      const int d1 = hloc * p.D + j0;
       const uint32_t off1 = static_cast<uint32_t>((col * kTileM + d1) * 4);
       const uint32_t off2 = off1 + static_cast<uint32_t>(half * 4);
-      float y1 = 0.f, y2 = 0.f;
-      for (int s = 0; s < S; ++s) {
-        y1 += ld_dsmem_f32(red_rank[s] + off1);
-        y2 += ld_dsmem_f32(red_rank[s] + off2);
+      float4 a[kMaxSplits], c[kMaxSplits];
+#pragma unroll
+      for (int s = 0; s < kMaxSplits; ++s) {
+        if (s < S) {
+          a[s] = ld_dsmem_f32x4(red_rank[s] + off1);
+          c[s] = ld_dsmem_f32x4(red_rank[s] + off2);
+        }
+      }
+      float y1[4] = {0.f, 0.f, 0.f, 0.f}, y2[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int s = 0; s < kMaxSplits; ++s) {
+        if (s < S) {
+          y1[0] += a[s].x; y1[1] += a[s].y; y1[2] += a[s].z; y1[3] += a[s].w;
+          y2[0] += c[s].x; y2[1] += c[s].y; y2[2] += c[s].z; y2[3] += c[s].w;
+        }
       }
       const int hg = tile * hpt + hloc;  // head among the Hq + 2 Hkv of the projection
       const int pos = s_rpos[r];
       if (hg < p.Hq + p.Hkv) {
-        float sn, cs;
-        sincosf(static_cast<float>(pos) * p.inv_freq[j], &sn, &cs);
-        const float o1 = y1 * cs - y2 * sn, o2 = y2 * cs + y1 * sn;
-        y1 = o1;
-        y2 = o2;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          float sn, cs;
+          sincosf(static_cast<float>(pos) * p.inv_freq[j0 + e], &sn, &cs);
+          const float o1 = y1[e] * cs - y2[e] * sn, o2 = y2[e] * cs + y1[e] * sn;
+          y1[e] = o1;
+          y2[e] = o2;
+        }
       }
       __nv_bfloat16 *dst;
       if (hg < p.Hq) {
@@ -277,8 +295,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         __nv_bfloat16 *cache = hg < p.Hq + p.Hkv ? p.k_cache : p.v_cache;
         dst = cache + ((static_cast<size_t>(b) * p.Hkv + hk) * p.cap + pos) * p.D;
       }
-      dst[j] = __float2bfloat16_rn(y1);
-      dst[j + half] = __float2bfloat16_rn(y2);
+      // 4 bf16 = 8 bytes at each half (j0 is a multiple of 4, rows 16-byte aligned).
+      *reinterpret_cast<uint2 *>(dst + j0) = make_uint2(pack_bf16(y1[0], y1[1]), pack_bf16(y1[2], y1[3]));
+      *reinterpret_cast<uint2 *>(dst + j0 + half) = make_uint2(pack_bf16(y2[0], y2[1]), pack_bf16(y2[2], y2[3]));
     }
     __syncwarp();
     cluster_sync();
