@@ -18,6 +18,8 @@ What it computes (the verifier side of one speculative-decoding iteration):
   the longest accepted prefix and the correction token (Algorithm 1).
 * ``kv_commit`` -- the context update m <- m + k + 1 of Algorithm 1 applied to
   a KV cache: accepted slots stay, rejected slots are cleared.
+* ``paged_gather`` / ``kv_commit_paged`` / ``kv_write_paged`` -- the same cache
+  operations on a paged cache (pools of fixed-size pages and a block table).
 * ``verify_qkv_rope`` / ``kv_write`` -- the projection of the verify block's
   hidden states into queries, keys and values with rotary position embedding,
   and the write of its keys and values into the block's cache slots: the
@@ -327,3 +329,53 @@ def kv_write(k_cache, v_cache, k, v, ctx_lens, n_draft, cu_q):
         kc[seq[r], :, pos[r]] = k[r]
         vc[seq[r], :, pos[r]] = v[r]
     return kc, vc
+
+
+# ----------------------------------------------------------------------------
+# Paged KV cache: pools [num_pages, Hkv, page, D] and a block table [B, max_pages]
+# ----------------------------------------------------------------------------
+def paged_slot(block_table, b, s, page):
+    """(page id, row in the page) of slot s of sequence b."""
+    return int(block_table[b][s // page]), s % page
+
+
+def paged_gather(pool, block_table, n_slots, page):
+    """Dense view [B, Hkv, n_slots, D] of a paged pool: slot s of sequence b is row
+    s % page of page block_table[b][s // page]."""
+    pool = np.asarray(pool)
+    B = len(block_table)
+    out = np.zeros((B, pool.shape[1], n_slots, pool.shape[3]), dtype=np.float64)
+    for b in range(B):
+        for s in range(n_slots):
+            pg, r = paged_slot(block_table, b, s, page)
+            out[b, :, s] = pool[pg, :, r]
+    return out
+
+
+def kv_commit_paged(k_pool, v_pool, block_table, ctx_lens, accepted_len, n_draft, page):
+    """``kv_commit`` on a paged cache: the rejected slots ctx_b + a_b + 1 .. ctx_b + k_b of
+    sequence b are cleared where the block table puts them; returns new (k_pool, v_pool,
+    ctx_lens) copies."""
+    k = np.array(k_pool, dtype=np.float64, copy=True)
+    v = np.array(v_pool, dtype=np.float64, copy=True)
+    ctx = np.array(ctx_lens, dtype=np.int64, copy=True)
+    for b in range(len(ctx)):
+        lo = int(ctx[b]) + int(accepted_len[b]) + 1
+        for s in range(lo, int(ctx[b]) + int(n_draft[b]) + 1):
+            pg, r = paged_slot(block_table, b, s, page)
+            k[pg, :, r] = 0
+            v[pg, :, r] = 0
+        ctx[b] = lo
+    return k, v, ctx
+
+
+def kv_write_paged(k_pool, v_pool, block_table, k, v, ctx_lens, n_draft, cu_q, page):
+    """``kv_write`` on a paged cache; returns new (k_pool, v_pool) copies."""
+    kp = np.array(k_pool, dtype=np.float64, copy=True)
+    vp = np.array(v_pool, dtype=np.float64, copy=True)
+    seq, pos = verify_positions(ctx_lens, n_draft, cu_q)
+    for r in range(len(seq)):
+        pg, row = paged_slot(block_table, int(seq[r]), int(pos[r]), page)
+        kp[pg, :, row] = k[r]
+        vp[pg, :, row] = v[r]
+    return kp, vp

@@ -456,6 +456,61 @@ def check_kv_write_slots(o):
                 assert (k2[b, :, slot] == -1.0).all() and (v2[b, :, slot] == -2.0).all()
 
 
+# ----------------------------------------------------------------------------
+# Paged KV cache
+# ----------------------------------------------------------------------------
+def check_paged_worked_example(o):
+    g = _golden()["paged"]
+    P = g["page"]
+    kp = np.arange(4 * 1 * P * 2, dtype=np.float64).reshape(4, 1, P, 2) + 1.0
+    vp = -kp
+    k2, v2, ctx = o.kv_commit_paged(kp, vp, g["block_table"], g["ctx"], g["accepted"], g["k"], P)
+    np.testing.assert_array_equal(ctx, g["new_ctx"])
+    cleared = {tuple(c) for c in g["cleared"]}
+    for pg in range(4):
+        for r in range(P):
+            if (pg, r) in cleared:
+                assert (k2[pg, :, r] == 0).all() and (v2[pg, :, r] == 0).all()
+            else:
+                assert (k2[pg, :, r] == kp[pg, :, r]).all() and (v2[pg, :, r] == vp[pg, :, r]).all()
+
+
+def check_paged_matches_dense(o, seed=13):
+    """Scattering dense caches into pages by a random table and gathering them back is the
+    identity; commit and write through the table equal the dense ones on the gathered view."""
+    rng = np.random.default_rng(seed)
+    B, Hkv, D, P, max_pages = 3, 2, 4, 4, 3
+    cap = P * max_pages
+    perm = rng.permutation(B * max_pages + 2)
+    table = perm[:B * max_pages].reshape(B, max_pages)
+    kd = np.array([2, 0, 3])
+    ctx = np.array([5, 0, 8])
+    cu = np.concatenate([[0], np.cumsum(kd + 1)])
+    dense_k = rng.standard_normal((B, Hkv, cap, D))
+    dense_v = rng.standard_normal((B, Hkv, cap, D))
+    kp = np.full((B * max_pages + 2, Hkv, P, D), np.nan)
+    vp = kp.copy()
+    for b in range(B):
+        for j in range(max_pages):
+            kp[table[b, j]] = dense_k[b, :, j * P:(j + 1) * P]
+            vp[table[b, j]] = dense_v[b, :, j * P:(j + 1) * P]
+    np.testing.assert_array_equal(o.paged_gather(kp, table, cap, P), dense_k)
+    acc = np.array([1, 0, 0])
+    k2, v2, c2 = o.kv_commit_paged(kp, vp, table, ctx, acc, kd, P)
+    kd2, vd2, cd2 = o.kv_commit(dense_k, dense_v, ctx, acc, kd)
+    np.testing.assert_array_equal(o.paged_gather(k2, table, cap, P), kd2)
+    np.testing.assert_array_equal(o.paged_gather(v2, table, cap, P), vd2)
+    np.testing.assert_array_equal(c2, cd2)
+    R = int(cu[-1])
+    kn = rng.standard_normal((R, Hkv, D))
+    vn = rng.standard_normal((R, Hkv, D))
+    k3, v3 = o.kv_write_paged(kp, vp, table, kn, vn, ctx, kd, cu, P)
+    kd3, vd3 = o.kv_write(dense_k, dense_v, kn, vn, ctx, kd, cu)
+    np.testing.assert_array_equal(o.paged_gather(k3, table, cap, P), kd3)
+    np.testing.assert_array_equal(o.paged_gather(v3, table, cap, P), vd3)
+    assert np.isnan(k3[perm[B * max_pages:]]).all()  # pages outside the table untouched
+
+
 ALL_CHECKS = [
     check_attention_worked_examples, check_attention_vs_sdpa, check_attention_special_cases,
     check_attention_gqa_mapping, check_logits_one_hot, check_acceptance_worked_examples,
@@ -463,4 +518,5 @@ ALL_CHECKS = [
     check_stochastic_output_law, check_progress_and_bounds, check_greedy_identity,
     check_kv_commit, check_rope_worked_examples, check_rope_vs_complex_rotation,
     check_rope_relative_position, check_qkv_projection_layout, check_kv_write_slots,
+    check_paged_worked_example, check_paged_matches_dense,
 ]

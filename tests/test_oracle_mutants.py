@@ -60,6 +60,13 @@ MUTANTS = {
     "keys_not_rotated": ("return rope(q, pos[:, None], theta), rope(k, pos[:, None], theta), v",
                          "return rope(q, pos[:, None], theta), k, v"),
     "kv_write_wrong_slot": ("kc[seq[r], :, pos[r]] = k[r]", "kc[seq[r], :, pos[r] - 1] = k[r]"),
+    # Paged cache addressing.
+    "paged_row_from_page_index": ("return int(block_table[b][s // page]), s % page",
+                                  "return int(block_table[b][s // page]), s // page"),
+    "paged_table_transposed": ("return int(block_table[b][s // page]), s % page",
+                               "return int(block_table[s // page][b]), s % page"),
+    "paged_commit_off_by_one": ("        lo = int(ctx[b]) + int(accepted_len[b]) + 1\n        for s in range(lo,",
+                                "        lo = int(ctx[b]) + int(accepted_len[b]) + 1\n        for s in range(lo + 1,"),
 }
 
 
