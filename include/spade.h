@@ -302,6 +302,50 @@ spade_status spade_kv_commit(void *k_cache, void *v_cache, int32_t *ctx_lens,
                              spade_stream_t stream);
 
 /* ------------------------------------------------------------------------ */
+/* Paged KV cache                                                            */
+/* ------------------------------------------------------------------------ */
+/*
+ * The same operations on a paged KV cache, for serving batches whose context
+ * lengths differ widely: keys and values live in pools of fixed-size pages,
+ *   k_pool, v_pool  bf16 [num_pages, Hkv, page_size, D] row-major, 16-byte aligned
+ *   block_table     int32 [B, max_pages]: block_table[b * max_pages + j] is the
+ *                   page that holds slots [j * page_size, (j + 1) * page_size)
+ *                   of sequence b (every KV head), 0 <= page < num_pages;
+ * so slot s of sequence b, KV head g, is row s % page_size of page
+ * block_table[b][s / page_size], head g.  A sequence can use up to
+ * max_pages * page_size slots (its capacity, the `cap` of the dense calls);
+ * page_size is a multiple of 64 for the attention.  Only the table entries of
+ * the pages a call touches are read; a touched entry outside [0, num_pages)
+ * sets SPADE_DEV_BAD_INDEX (the attention reads zeros for it; the commit and
+ * the QKV write skip that sequence).  Every other argument, and the result,
+ * is that of the dense call of the same name.  The fused
+ * spade_verify_accept_commit has no paged form: a paged step runs
+ * spade_verify_accept and then spade_kv_commit_paged.
+ */
+spade_status spade_verify_attention_paged(const void *q, const void *k_pool, const void *v_pool,
+                                          const int32_t *block_table, const int32_t *ctx_lens,
+                                          const int32_t *n_draft, const int32_t *cu_q, void *out,
+                                          float *lse, int32_t B, int32_t Hq, int32_t Hkv, int32_t D,
+                                          int32_t page_size, int32_t num_pages, int32_t max_pages,
+                                          int32_t max_k, int32_t R, void *workspace,
+                                          size_t workspace_bytes, int32_t *status,
+                                          spade_stream_t stream);
+
+spade_status spade_kv_commit_paged(void *k_pool, void *v_pool, const int32_t *block_table,
+                                   int32_t *ctx_lens, const int32_t *accepted_len,
+                                   const int32_t *n_draft, int32_t B, int32_t Hkv, int32_t D,
+                                   int32_t page_size, int32_t num_pages, int32_t max_pages,
+                                   int32_t *status, spade_stream_t stream);
+
+spade_status spade_verify_qkv_rope_paged(const void *x, const void *w_qkv, const int32_t *block_table,
+                                         const int32_t *ctx_lens, const int32_t *n_draft,
+                                         const int32_t *cu_q, void *q_out, void *k_pool, void *v_pool,
+                                         int32_t B, int32_t R, int32_t H, int32_t Hq, int32_t Hkv,
+                                         int32_t D, int32_t page_size, int32_t num_pages,
+                                         int32_t max_pages, int32_t max_k, float rope_theta,
+                                         int32_t *status, spade_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
 /* Diagnostics                                                               */
 /* ------------------------------------------------------------------------ */
 const char *spade_status_string(spade_status s);

@@ -24,7 +24,8 @@ from . import _build
 __all__ = [
     "SpadeError", "load", "build", "library_path",
     "spade_verify_attention", "spade_verify_accept", "spade_kv_commit", "spade_verify_attention_noalloc",
-    "spade_verify_qkv_rope",
+    "spade_verify_qkv_rope", "spade_verify_attention_paged", "spade_kv_commit_paged",
+    "spade_verify_qkv_rope_paged",
     "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_accept_launches",
     "spade_accept_stats_layout", "read_accept_stats", "spade_verify_accept_commit", "spade_selftest_wait_timeout",
     "attn_workspace", "accept_workspace", "status_tensor", "check_status",
@@ -92,6 +93,12 @@ def load():
     lib.spade_selftest_wait_timeout.argtypes = [_vp, _i32, _vp]
     lib.spade_verify_qkv_rope.restype = _i32
     lib.spade_verify_qkv_rope.argtypes = [_vp] * 8 + [_i32] * 8 + [ctypes.c_float, _vp, _vp]
+    lib.spade_verify_attention_paged.restype = _i32
+    lib.spade_verify_attention_paged.argtypes = [_vp] * 9 + [_i32] * 9 + [_vp, _sz, _vp, _vp]
+    lib.spade_kv_commit_paged.restype = _i32
+    lib.spade_kv_commit_paged.argtypes = [_vp] * 6 + [_i32] * 6 + [_vp, _vp]
+    lib.spade_verify_qkv_rope_paged.restype = _i32
+    lib.spade_verify_qkv_rope_paged.argtypes = [_vp] * 9 + [_i32] * 10 + [ctypes.c_float, _vp, _vp]
     lib.spade_kv_commit.restype = _i32
     lib.spade_kv_commit.argtypes = [_vp] * 5 + [_i32] * 4 + [_vp, _vp]
     lib.spade_status_string.restype = ctypes.c_char_p
@@ -333,6 +340,78 @@ def spade_verify_qkv_rope(x, w_qkv, ctx_lens, n_draft, cu_q, q_out, k_cache, v_c
     rc = load().spade_verify_qkv_rope(
         _ptr(x), _ptr(w_qkv), _ptr(ctx_lens), _ptr(n_draft), _ptr(cu_q), _ptr(q_out), _ptr(k_cache), _ptr(v_cache),
         B, R, H, Hq, Hkv, D, cap, int(max_k), float(rope_theta), _ptr(status), _stream(stream))
+    _check_rc(rc)
+    return q_out
+
+
+# ---------------------------------------------------------------------------
+# Paged KV cache: pools [num_pages, Hkv, page_size, D], block_table [B, max_pages].
+def _need_paged(k_pool, v_pool, block_table):
+    _need(k_pool, "k_pool", torch.bfloat16, 4)
+    _need(v_pool, "v_pool", torch.bfloat16, 4)
+    _need(block_table, "block_table", torch.int32, 2)
+    if tuple(v_pool.shape) != tuple(k_pool.shape):
+        raise ValueError("k_pool and v_pool shapes differ")
+    num_pages, Hkv, page_size, D = k_pool.shape
+    return num_pages, Hkv, page_size, D, block_table.shape[1]
+
+
+def spade_verify_attention_paged(q, k_pool, v_pool, block_table, ctx_lens, n_draft, cu_q, out, lse=None, *,
+                                 max_k, workspace, status, stream=None):
+    """spade_verify_attention on a paged cache (see include/spade.h)."""
+    _need(q, "q", torch.bfloat16, 3)
+    _need(out, "out", torch.bfloat16, 3)
+    num_pages, Hkv, page_size, D, max_pages = _need_paged(k_pool, v_pool, block_table)
+    for t, n in ((ctx_lens, "ctx_lens"), (n_draft, "n_draft"), (cu_q, "cu_q"), (status, "status")):
+        _need(t, n, torch.int32, 1)
+    if lse is not None:
+        _need(lse, "lse", torch.float32, 2)
+    _need(workspace, "workspace", torch.uint8, 1)
+    R, Hq, Dq = q.shape
+    B = ctx_lens.numel()
+    if Dq != D or tuple(out.shape) != (R, Hq, D) or block_table.shape[0] != B or n_draft.numel() != B \
+            or cu_q.numel() != B + 1:
+        raise ValueError("inconsistent paged attention shapes")
+    rc = load().spade_verify_attention_paged(
+        _ptr(q), _ptr(k_pool), _ptr(v_pool), _ptr(block_table), _ptr(ctx_lens), _ptr(n_draft), _ptr(cu_q), _ptr(out),
+        _ptr(lse), B, Hq, Hkv, D, page_size, num_pages, max_pages, int(max_k), R, _ptr(workspace), workspace.numel(),
+        _ptr(status), _stream(stream))
+    _check_rc(rc)
+    return out
+
+
+def spade_kv_commit_paged(k_pool, v_pool, block_table, ctx_lens, accepted_len, n_draft, *, status, stream=None):
+    """spade_kv_commit on a paged cache (see include/spade.h)."""
+    num_pages, Hkv, page_size, D, max_pages = _need_paged(k_pool, v_pool, block_table)
+    for t, n in ((ctx_lens, "ctx_lens"), (accepted_len, "accepted_len"), (n_draft, "n_draft"), (status, "status")):
+        _need(t, n, torch.int32, 1)
+    B = ctx_lens.numel()
+    if block_table.shape[0] != B:
+        raise ValueError("block_table must have one row per sequence")
+    rc = load().spade_kv_commit_paged(_ptr(k_pool), _ptr(v_pool), _ptr(block_table), _ptr(ctx_lens),
+                                      _ptr(accepted_len), _ptr(n_draft), B, Hkv, D, page_size, num_pages,
+                                      max_pages, _ptr(status), _stream(stream))
+    _check_rc(rc)
+
+
+def spade_verify_qkv_rope_paged(x, w_qkv, block_table, ctx_lens, n_draft, cu_q, q_out, k_pool, v_pool, *, Hq,
+                                rope_theta, max_k, status, stream=None):
+    """spade_verify_qkv_rope writing the block's K/V into a paged cache (see include/spade.h)."""
+    _need(x, "x", torch.bfloat16, 2)
+    _need(w_qkv, "w_qkv", torch.bfloat16, 2)
+    _need(q_out, "q_out", torch.bfloat16, 3)
+    num_pages, Hkv, page_size, D, max_pages = _need_paged(k_pool, v_pool, block_table)
+    for t, n in ((ctx_lens, "ctx_lens"), (n_draft, "n_draft"), (cu_q, "cu_q"), (status, "status")):
+        _need(t, n, torch.int32, 1)
+    R, H = x.shape
+    B = ctx_lens.numel()
+    if tuple(q_out.shape) != (R, Hq, D) or tuple(w_qkv.shape) != ((Hq + 2 * Hkv) * D, H) \
+            or block_table.shape[0] != B or n_draft.numel() != B or cu_q.numel() != B + 1:
+        raise ValueError("inconsistent paged qkv_rope shapes")
+    rc = load().spade_verify_qkv_rope_paged(
+        _ptr(x), _ptr(w_qkv), _ptr(block_table), _ptr(ctx_lens), _ptr(n_draft), _ptr(cu_q), _ptr(q_out),
+        _ptr(k_pool), _ptr(v_pool), B, R, H, Hq, Hkv, D, page_size, num_pages, max_pages, int(max_k),
+        float(rope_theta), _ptr(status), _stream(stream))
     _check_rc(rc)
     return q_out
 

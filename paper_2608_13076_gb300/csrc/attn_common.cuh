@@ -33,7 +33,25 @@ struct Params {
   int B, Hq, Hkv, G, cap, max_k, R, RB, num_ctas;
   int unit_cost;     // virtual slices charged at each unit's start (the schedule's cost model)
   float scale_log2;  // log2(e) / sqrt(D)
+  // Paged cache (block_table null: dense [B, Hkv, cap, D] caches).  The pools
+  // are [num_pages, Hkv, page_size, D]; block_table[b * max_pages + j] is the
+  // page of sequence b's slots [j * page_size, (j + 1) * page_size).
+  const int32_t *block_table;
+  int page_size, max_pages, num_pages;
 };
+
+// Pool row of the 64-key slice starting at key `key` of (b, kvh) in a paged
+// cache.  An out-of-range page id is reported and mapped past the last row,
+// where the tensor copy reads zeros.
+__device__ __forceinline__ int paged_row(const Params &p, int b, int kvh, int key) {
+  const int page = __ldg(p.block_table + static_cast<int64_t>(b) * p.max_pages + key / p.page_size);
+  const int64_t rows = static_cast<int64_t>(p.num_pages) * p.Hkv * p.page_size;
+  if (page < 0 || page >= p.num_pages) {
+    atomicOr(p.status, SPADE_DEV_BAD_INDEX);
+    return static_cast<int>(rows);
+  }
+  return static_cast<int>((static_cast<int64_t>(page) * p.Hkv + kvh) * p.page_size + key % p.page_size);
+}
 
 constexpr int round_up_c(int x, int a) { return (x + a - 1) / a * a; }
 

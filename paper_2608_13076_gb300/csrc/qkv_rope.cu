@@ -61,6 +61,10 @@ struct Params {
   int stages;   // ring depth
   uint32_t tmem_cols;
   float inv_freq[64];  // theta^(-2j/D), j < D/2, rounded from double on the host
+  // Paged caches (block_table null: dense [B, Hkv, cap, D]): pools
+  // [num_pages, Hkv, page_size, D], block_table [B, max_pages].
+  const int32_t *block_table;
+  int page_size, max_pages, num_pages;
 };
 
 // Shared-memory plan (offsets from a 1024-byte aligned base).
@@ -135,6 +139,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (bad) {
       if (blockIdx.x == 0) atomicOr(p.status, bad);
       continue;
+    }
+    if (p.block_table) {
+      // Every page the block writes must exist.
+      for (int i = 0; i <= k; ++i) {
+        const int pg = p.block_table[static_cast<int64_t>(b) * p.max_pages + (c + i) / p.page_size];
+        if (pg < 0 || pg >= p.num_pages) bad = SPADE_DEV_BAD_INDEX;
+      }
+      if (bad) {
+        if (blockIdx.x == 0) atomicOr(p.status, bad);
+        continue;
+      }
     }
     for (int i = 0; i <= k; ++i) {
       s_rseq[q0 + i] = b;
@@ -293,7 +308,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       } else {
         const int hk = hg < p.Hq + p.Hkv ? hg - p.Hq : hg - p.Hq - p.Hkv;
         __nv_bfloat16 *cache = hg < p.Hq + p.Hkv ? p.k_cache : p.v_cache;
-        dst = cache + ((static_cast<size_t>(b) * p.Hkv + hk) * p.cap + pos) * p.D;
+        if (p.block_table) {
+          const int pg = p.block_table[static_cast<int64_t>(b) * p.max_pages + pos / p.page_size];
+          dst = cache + ((static_cast<size_t>(pg) * p.Hkv + hk) * p.page_size + pos % p.page_size) * p.D;
+        } else {
+          dst = cache + ((static_cast<size_t>(b) * p.Hkv + hk) * p.cap + pos) * p.D;
+        }
       }
       // 4 bf16 = 8 bytes at each half (j0 is a multiple of 4, rows 16-byte aligned).
       *reinterpret_cast<uint2 *>(dst + j0) = make_uint2(pack_bf16(y1[0], y1[1]), pack_bf16(y1[2], y1[3]));
@@ -349,12 +369,20 @@ static int max_active_clusters(int splits, int smem) {
 
 using namespace spade;
 
-extern "C" spade_status spade_verify_qkv_rope(const void *x, const void *w_qkv, const int32_t *ctx_lens,
-                                              const int32_t *n_draft, const int32_t *cu_q, void *q_out,
-                                              void *k_cache, void *v_cache, int32_t B, int32_t R,
-                                              int32_t H, int32_t Hq, int32_t Hkv, int32_t D, int32_t cap,
-                                              int32_t max_k, float rope_theta, int32_t *status,
-                                              spade_stream_t stream) {
+namespace spade {
+namespace qkv {
+struct Paging {
+  const int32_t *block_table;
+  int page_size, max_pages, num_pages;
+};
+}  // namespace qkv
+}  // namespace spade
+
+static spade_status qkv_rope_impl(const void *x, const void *w_qkv, const int32_t *ctx_lens,
+                                  const int32_t *n_draft, const int32_t *cu_q, void *q_out, void *k_cache,
+                                  void *v_cache, int32_t B, int32_t R, int32_t H, int32_t Hq, int32_t Hkv,
+                                  int32_t D, int32_t cap, int32_t max_k, float rope_theta, int32_t *status,
+                                  spade_stream_t stream, const qkv::Paging *pg) {
   using namespace qkv;
   if (!x || !w_qkv || !ctx_lens || !n_draft || !cu_q || !q_out || !k_cache || !v_cache || !status)
     return fail(SPADE_ERR_INVALID_ARG, "spade_verify_qkv_rope: null pointer argument");
@@ -385,6 +413,10 @@ extern "C" spade_status spade_verify_qkv_rope(const void *x, const void *w_qkv, 
   p.v_cache = static_cast<__nv_bfloat16 *>(v_cache);
   p.status = status;
   p.B = B; p.R = R; p.H = H; p.Hq = Hq; p.Hkv = Hkv; p.D = D; p.cap = cap; p.max_k = max_k;
+  p.block_table = pg ? pg->block_table : nullptr;
+  p.page_size = pg ? pg->page_size : 0;
+  p.max_pages = pg ? pg->max_pages : 0;
+  p.num_pages = pg ? pg->num_pages : 0;
   p.KC = (H + kKChunk - 1) / kKChunk;
   p.Ncols = (R + 15) / 16 * 16;
   p.tmem_cols = 32;
@@ -444,4 +476,32 @@ extern "C" spade_status spade_verify_qkv_rope(const void *x, const void *w_qkv, 
   const cudaError_t e = cudaLaunchKernelEx(&cfg, qkv_rope_kernel, p, tw, tx0, tx1);
   if (e != cudaSuccess) return cuda_fail(e, "qkv_rope launch");
   return SPADE_OK;
+}
+
+extern "C" spade_status spade_verify_qkv_rope(const void *x, const void *w_qkv, const int32_t *ctx_lens,
+                                              const int32_t *n_draft, const int32_t *cu_q, void *q_out,
+                                              void *k_cache, void *v_cache, int32_t B, int32_t R,
+                                              int32_t H, int32_t Hq, int32_t Hkv, int32_t D, int32_t cap,
+                                              int32_t max_k, float rope_theta, int32_t *status,
+                                              spade_stream_t stream) {
+  return qkv_rope_impl(x, w_qkv, ctx_lens, n_draft, cu_q, q_out, k_cache, v_cache, B, R, H, Hq, Hkv, D, cap,
+                       max_k, rope_theta, status, stream, nullptr);
+}
+
+extern "C" spade_status spade_verify_qkv_rope_paged(const void *x, const void *w_qkv,
+                                                    const int32_t *block_table, const int32_t *ctx_lens,
+                                                    const int32_t *n_draft, const int32_t *cu_q, void *q_out,
+                                                    void *k_pool, void *v_pool, int32_t B, int32_t R,
+                                                    int32_t H, int32_t Hq, int32_t Hkv, int32_t D,
+                                                    int32_t page_size, int32_t num_pages, int32_t max_pages,
+                                                    int32_t max_k, float rope_theta, int32_t *status,
+                                                    spade_stream_t stream) {
+  if (!block_table) return fail(SPADE_ERR_INVALID_ARG, "spade_verify_qkv_rope_paged: null block_table");
+  if (page_size <= 0 || num_pages <= 0 || max_pages <= 0)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_verify_qkv_rope_paged: non-positive page geometry");
+  if (static_cast<int64_t>(max_pages) * page_size >= (int64_t(1) << 31))
+    return fail(SPADE_ERR_CAPACITY, "max_pages * page_size exceeds 2^31");
+  const qkv::Paging pg{block_table, page_size, max_pages, num_pages};
+  return qkv_rope_impl(x, w_qkv, ctx_lens, n_draft, cu_q, q_out, k_pool, v_pool, B, R, H, Hq, Hkv, D,
+                       max_pages * page_size, max_k, rope_theta, status, stream, &pg);
 }

@@ -32,11 +32,21 @@ extern "C" size_t spade_attn_workspace_size(int32_t B, int32_t Hq, int32_t Hkv, 
   return counters + (units + sms) * attn::slot_floats(D) * sizeof(float);
 }
 
-extern "C" spade_status spade_verify_attention(
+namespace spade {
+namespace attn {
+// Page geometry of a paged cache (see Params).
+struct Paging {
+  const int32_t *block_table;
+  int page_size, max_pages, num_pages;
+};
+}  // namespace attn
+}  // namespace spade
+
+static spade_status verify_attention_impl(
     const void *q, const void *k_cache, const void *v_cache, const int32_t *ctx_lens,
     const int32_t *n_draft, const int32_t *cu_q, void *out, float *lse, int32_t B, int32_t Hq,
     int32_t Hkv, int32_t D, int32_t cap, int32_t max_k, int32_t R, void *workspace,
-    size_t workspace_bytes, int32_t *status, spade_stream_t stream) {
+    size_t workspace_bytes, int32_t *status, spade_stream_t stream, const attn::Paging *pg) {
   if (!q || !k_cache || !v_cache || !ctx_lens || !n_draft || !cu_q || !out || !status)
     return fail(SPADE_ERR_INVALID_ARG, "spade_verify_attention: null pointer argument");
   if (B <= 0 || Hq <= 0 || Hkv <= 0 || cap <= 0 || max_k < 0 || R <= 0)
@@ -45,8 +55,10 @@ extern "C" spade_status spade_verify_attention(
   if (D != 64 && D != 128) return fail(SPADE_ERR_SHAPE, "head dim %d not supported (64 or 128)", D);
   if (B > attn::kMaxB) return fail(SPADE_ERR_SHAPE, "B = %d exceeds %d sequences per call", B, attn::kMaxB);
   if (R < B) return fail(SPADE_ERR_INVALID_ARG, "R = %d < B = %d", R, B);
-  if (static_cast<int64_t>(B) * Hkv * cap >= (int64_t(1) << 31))
-    return fail(SPADE_ERR_CAPACITY, "KV cache rows B*Hkv*cap exceed 2^31");
+  const int64_t cache_rows = pg ? static_cast<int64_t>(pg->num_pages) * Hkv * pg->page_size
+                                : static_cast<int64_t>(B) * Hkv * cap;
+  if (cache_rows >= (int64_t(1) << 31))
+    return fail(SPADE_ERR_CAPACITY, "KV cache rows (B or pages) * Hkv * slots exceed 2^31");
   if (!aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(q, 16) || !aligned(out, 16))
     return fail(SPADE_ERR_INVALID_ARG, "q, caches and out must be 16-byte aligned");
   int sms = 0;
@@ -73,6 +85,10 @@ extern "C" spade_status spade_verify_attention(
   p.status = status;
   p.B = B; p.Hq = Hq; p.Hkv = Hkv; p.G = G; p.cap = cap; p.max_k = max_k; p.R = R; p.RB = RB;
   p.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(D));
+  p.block_table = pg ? pg->block_table : nullptr;
+  p.page_size = pg ? pg->page_size : 0;
+  p.max_pages = pg ? pg->max_pages : 0;
+  p.num_pages = pg ? pg->num_pages : 0;
   // The tensor-memory kernel charges each unit's epilogue and pipeline restart
   // to the CTA that starts it; a 64-dim slice moves half the bytes of a
   // 128-dim one, so the same restart costs twice the slices.
@@ -81,7 +97,7 @@ extern "C" spade_status spade_verify_attention(
   const int64_t max_chunks = static_cast<int64_t>(units) * ((cap + attn::kChunk - 1) / attn::kChunk);
   p.num_ctas = static_cast<int>(max_chunks < sms ? max_chunks : sms);
 
-  const uint64_t rows = static_cast<uint64_t>(B) * Hkv * cap;
+  const uint64_t rows = static_cast<uint64_t>(cache_rows);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e;
   {
@@ -98,6 +114,34 @@ extern "C" spade_status spade_verify_attention(
   }
   if (e != cudaSuccess) return cuda_fail(e, "verify_attention launch");
   return SPADE_OK;
+}
+
+extern "C" spade_status spade_verify_attention(
+    const void *q, const void *k_cache, const void *v_cache, const int32_t *ctx_lens,
+    const int32_t *n_draft, const int32_t *cu_q, void *out, float *lse, int32_t B, int32_t Hq,
+    int32_t Hkv, int32_t D, int32_t cap, int32_t max_k, int32_t R, void *workspace,
+    size_t workspace_bytes, int32_t *status, spade_stream_t stream) {
+  return verify_attention_impl(q, k_cache, v_cache, ctx_lens, n_draft, cu_q, out, lse, B, Hq, Hkv, D,
+                               cap, max_k, R, workspace, workspace_bytes, status, stream, nullptr);
+}
+
+extern "C" spade_status spade_verify_attention_paged(
+    const void *q, const void *k_pool, const void *v_pool, const int32_t *block_table,
+    const int32_t *ctx_lens, const int32_t *n_draft, const int32_t *cu_q, void *out, float *lse,
+    int32_t B, int32_t Hq, int32_t Hkv, int32_t D, int32_t page_size, int32_t num_pages,
+    int32_t max_pages, int32_t max_k, int32_t R, void *workspace, size_t workspace_bytes,
+    int32_t *status, spade_stream_t stream) {
+  if (!block_table) return fail(SPADE_ERR_INVALID_ARG, "spade_verify_attention_paged: null block_table");
+  if (page_size <= 0 || num_pages <= 0 || max_pages <= 0)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_verify_attention_paged: non-positive page geometry");
+  if (page_size % attn::kChunk)
+    return fail(SPADE_ERR_SHAPE, "page size %d must be a multiple of %d", page_size, attn::kChunk);
+  if (static_cast<int64_t>(max_pages) * page_size >= (int64_t(1) << 31))
+    return fail(SPADE_ERR_CAPACITY, "max_pages * page_size exceeds 2^31");
+  const attn::Paging pg{block_table, page_size, max_pages, num_pages};
+  return verify_attention_impl(q, k_pool, v_pool, ctx_lens, n_draft, cu_q, out, lse, B, Hq, Hkv, D,
+                               max_pages * page_size, max_k, R, workspace, workspace_bytes, status,
+                               stream, &pg);
 }
 
 // ---------------------------------------------------------------------------

@@ -328,16 +328,30 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int st = it % kStages;
           const uint32_t ph = (it / kStages) & 1;
           const int nsl = min(2, si.n_here - 2 * c);
-          const int key_row = row0 + (si.g.ci + 2 * c) * kChunk;
+          const int key0 = (si.g.ci + 2 * c) * kChunk;
+          // Cache rows of the chunk's slices: contiguous in a dense cache; in a
+          // paged one each slice lies in one page (page sizes are multiples of
+          // 64), found through the block table before the stage wait so that
+          // the table load overlaps it.
+          int row_a = row0 + key0, row_b = row_a + kChunk;
+          if (p.block_table) {
+            row_a = paged_row(p, si.g.b, si.g.kvh, key0);
+            row_b = nsl == 2 ? paged_row(p, si.g.b, si.g.kvh, key0 + kChunk) : 0;
+          }
           uint8_t *tile = ring + st * kTile;
           if (!mbar_wait(&bars[bar_empty + st], ph ^ 1, s_abort)) expired = true;
           if (*s_abort) continue;
           mbar_arrive_expect_tx(&bars[bar_full + st], nsl * (kSlab / kDMax) * kD);
-          if (nsl == 2) {
-            tma_load_3d(tile, tm2, 0, key_row, 0, &bars[bar_full + st], pol);
+          if (nsl == 2 && row_b == row_a + kChunk) {
+            tma_load_3d(tile, tm2, 0, row_a, 0, &bars[bar_full + st], pol);
           } else {
-            tma_load_3d(tile, tm1, 0, key_row, 0, &bars[bar_full + st], pol);
-            if constexpr (kD == kDMax) tma_load_3d(tile + kSlab, tm1, 0, key_row, 1, &bars[bar_full + st], pol);
+            // One 64-key box per slice and slab; the second slice lands 64 rows in.
+            for (int i = 0; i < nsl; ++i) {
+              const int row = i ? row_b : row_a;
+              uint8_t *dst = tile + i * kChunk * 128;
+              tma_load_3d(dst, tm1, 0, row, 0, &bars[bar_full + st], pol);
+              if constexpr (kD == kDMax) tma_load_3d(dst + kSlab, tm1, 0, row, 1, &bars[bar_full + st], pol);
+            }
           }
           issued = it + 1;
         }

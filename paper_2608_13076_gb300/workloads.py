@@ -214,3 +214,32 @@ def make_qkv_inputs(spec: WorkloadSpec, R: int, device="cpu"):
     x = _bf16_normal(gen, (R, spec.H), 1.0, "cpu")
     w = _bf16_normal(gen, ((spec.Hq + 2 * spec.Hkv) * spec.D, spec.H), 1.0 / math.sqrt(spec.H), "cpu")
     return x.to(device), w.to(device)
+
+
+def to_paged(wl, page_size: int, seed: int = 0, spare_pages: int = 3, device=None):
+    """The workload's dense caches scattered into paged pools.
+
+    Each sequence's cap slots are cut into pages of ``page_size`` slots, placed in a pool
+    at positions given by a seeded random permutation (so neighbouring pages of a sequence
+    are far apart), with ``spare_pages`` extra pages no sequence uses, filled with NaN.
+    Returns dict(k_pool, v_pool [num_pages, Hkv, page_size, D] bf16, block_table [B, max_pages]
+    int32, page_size, num_pages, max_pages) on ``device`` (default: the caches' device).
+    """
+    dev = wl["k_cache"].device if device is None else torch.device(device)
+    B, Hkv, cap, D = wl["k_cache"].shape
+    max_pages = (cap + page_size - 1) // page_size
+    num_pages = B * max_pages + spare_pages
+    gen = torch.Generator(device="cpu").manual_seed(seed)
+    perm = torch.randperm(num_pages, generator=gen)
+    table = perm[:B * max_pages].reshape(B, max_pages).to(torch.int32)
+    pools = []
+    for cache in (wl["k_cache"], wl["v_cache"]):
+        c = cache.cpu()
+        padded = torch.zeros((B, Hkv, max_pages * page_size, D), dtype=c.dtype)
+        padded[:, :, :cap] = c
+        pool = torch.full((num_pages, Hkv, page_size, D), float("nan"), dtype=c.dtype)
+        blocks = padded.reshape(B, Hkv, max_pages, page_size, D).permute(0, 2, 1, 3, 4)
+        pool[table.reshape(-1).long()] = blocks.reshape(B * max_pages, Hkv, page_size, D)
+        pools.append(pool.to(dev))
+    return dict(k_pool=pools[0], v_pool=pools[1], block_table=table.to(dev), page_size=page_size,
+                num_pages=num_pages, max_pages=max_pages)

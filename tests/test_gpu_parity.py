@@ -477,3 +477,106 @@ def test_qkv_then_attention_matches_oracle_chain(dev):
     ref, _ = O.verify_attention(q_ref, kc, vc, ctx, kd, cu)
     n, bad, worst = parity.compare_attention(out, ref)
     assert bad == 0, worst
+
+
+# ---------------------------------------------------------------------------
+# Paged KV cache: the same step through a block table.
+
+PAGED = [
+    ("gqa_mixed", 64), ("gqa_mixed", 128), ("long_split", 256), ("many_rows", 64), ("d64_stochastic", 128),
+    ("empty_context", 64),
+]
+
+
+@pytest.mark.parametrize("name,page", PAGED, ids=[f"{n}-p{p}" for n, p in PAGED])
+def test_paged_attention_equals_dense(dev, name, page):
+    """Paged attention over shuffled pages gives bit for bit the dense attention's output on the
+    same data (same schedule, same tensor-core products), and matches the oracle."""
+    wl = W.make_workload(SMALL[name], device=dev, cache_pad=70)
+    pg = W.to_paged(wl, page, seed=5)
+    out, lse, st = parity.gpu_attention(wl)
+    max_k = int(wl["n_draft"].max())
+    out_p = torch.full_like(out, float("nan"))
+    lse_p = torch.full_like(lse, float("nan"))
+    st_p = spade.status_tensor(dev)
+    ws = spade.attn_workspace(wl["B"], wl["Hq"], wl["Hkv"], wl["D"], pg["max_pages"] * page, max_k, device=dev)
+    spade.spade_verify_attention_paged(wl["q"], pg["k_pool"], pg["v_pool"], pg["block_table"], wl["ctx_lens"],
+                                       wl["n_draft"], wl["cu_q"], out_p, lse_p, max_k=max_k, workspace=ws, status=st_p)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0 and int(st_p.item()) == 0
+    assert torch.equal(out_p, out) and torch.equal(lse_p, lse)
+    kd = O.paged_gather(parity.to_np(pg["k_pool"]), parity.to_np(pg["block_table"]), wl["cap"], page)
+    vd = O.paged_gather(parity.to_np(pg["v_pool"]), parity.to_np(pg["block_table"]), wl["cap"], page)
+    ref, _ = O.verify_attention(parity.to_np(wl["q"]), kd, vd, parity.to_np(wl["ctx_lens"]),
+                                parity.to_np(wl["n_draft"]), parity.to_np(wl["cu_q"]))
+    n, bad, worst = parity.compare_attention(out_p, ref)
+    assert bad == 0, worst
+
+
+@pytest.mark.parametrize("name", ["llama3_8b", "ragged"])
+def test_paged_attention_full_size(dev, name):
+    """The benchmark shapes through 128-slot pages: equal to the dense attention bit for bit."""
+    wl = W.make_workload(W.SPECS[name], device=dev)
+    pg = W.to_paged(wl, 128, seed=9)
+    out, lse, st = parity.gpu_attention(wl)
+    max_k = int(wl["n_draft"].max())
+    out_p = torch.empty_like(out)
+    lse_p = torch.empty_like(lse)
+    st_p = spade.status_tensor(dev)
+    ws = spade.attn_workspace(wl["B"], wl["Hq"], wl["Hkv"], wl["D"], pg["max_pages"] * 128, max_k, device=dev)
+    spade.spade_verify_attention_paged(wl["q"], pg["k_pool"], pg["v_pool"], pg["block_table"], wl["ctx_lens"],
+                                       wl["n_draft"], wl["cu_q"], out_p, lse_p, max_k=max_k, workspace=ws, status=st_p)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0 and int(st_p.item()) == 0
+    assert torch.equal(out_p, out) and torch.equal(lse_p, lse)
+
+
+@pytest.mark.parametrize("page", [64, 128, 16])
+def test_paged_commit(dev, page):
+    wl = W.make_workload(SMALL["many_rows"], device=dev, cache_pad=5)
+    pg = W.to_paged(wl, page, seed=6)
+    acc, tok, st = parity.gpu_accept(wl)
+    k0, v0 = parity.to_np(pg["k_pool"]), parity.to_np(pg["v_pool"])
+    ctx = wl["ctx_lens"].clone()
+    spade.spade_kv_commit_paged(pg["k_pool"], pg["v_pool"], pg["block_table"], ctx, acc, wl["n_draft"], status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0
+    rk, rv, rctx = O.kv_commit_paged(k0, v0, parity.to_np(pg["block_table"]), parity.to_np(wl["ctx_lens"]),
+                                     parity.to_np(acc), parity.to_np(wl["n_draft"]), page)
+    assert np.array_equal(parity.to_np(ctx), rctx)
+    np.testing.assert_array_equal(parity.to_np(pg["k_pool"]), rk)   # NaN spare pages compare equal
+    np.testing.assert_array_equal(parity.to_np(pg["v_pool"]), rv)
+
+
+def test_paged_qkv_rope(dev):
+    spec = QKV_SMALL["qkv_gqa_d128"]
+    wl = W.make_workload(spec, device=dev, cache_pad=40)
+    pg = W.to_paged(wl, 64, seed=7)
+    x, w = W.make_qkv_inputs(spec, wl["R"], device=dev)
+    k0, v0 = parity.to_np(pg["k_pool"]), parity.to_np(pg["v_pool"])
+    q = torch.full((wl["R"], wl["Hq"], wl["D"]), float("nan"), dtype=torch.bfloat16, device=dev)
+    st = spade.status_tensor(dev)
+    spade.spade_verify_qkv_rope_paged(x, w, pg["block_table"], wl["ctx_lens"], wl["n_draft"], wl["cu_q"], q,
+                                      pg["k_pool"], pg["v_pool"], Hq=wl["Hq"], rope_theta=spec.rope_theta,
+                                      max_k=int(wl["n_draft"].max()), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    ctx, kd, cu = (parity.to_np(wl[k]) for k in ("ctx_lens", "n_draft", "cu_q"))
+    q_ref, k_ref, v_ref = O.verify_qkv_rope(parity.to_np(x), parity.to_np(w), ctx, kd, cu, wl["Hq"], wl["Hkv"],
+                                            spec.rope_theta)
+    n, bad, worst = parity.compare_attention(q, q_ref)
+    assert bad == 0, worst
+    rk, rv = O.kv_write_paged(k0, v0, parity.to_np(pg["block_table"]), k_ref, v_ref, ctx, kd, cu, 64)
+    gk, gv = parity.to_np(pg["k_pool"]), parity.to_np(pg["v_pool"])
+    seq, pos = O.verify_positions(ctx, kd, cu)
+    table = parity.to_np(pg["block_table"])
+    written = np.zeros(gk.shape[:1] + gk.shape[2:3], dtype=bool)  # [page, row]
+    for r in range(len(seq)):
+        pgi, row = O.paged_slot(table, int(seq[r]), int(pos[r]), 64)
+        written[pgi, row] = True
+        for got, ref in ((gk[pgi, :, row], k_ref[r]), (gv[pgi, :, row], v_ref[r])):
+            n, bad, worst = parity.compare_attention(torch.from_numpy(got[None]), ref[None])
+            assert bad == 0, worst
+    keep = ~written
+    np.testing.assert_array_equal(gk.transpose(0, 2, 1, 3)[keep], k0.transpose(0, 2, 1, 3)[keep])
+    np.testing.assert_array_equal(gv.transpose(0, 2, 1, 3)[keep], v0.transpose(0, 2, 1, 3)[keep])
