@@ -488,13 +488,26 @@ PAGED = [
 ]
 
 
+def _pool_to_dense(pool, table):
+    """[B, Hkv, max_pages * page, D] view of a paged pool (a plain gather on the device)."""
+    B, mp = table.shape
+    g = pool[table.reshape(-1).long()]                     # [B * mp, Hkv, page, D]
+    g = g.reshape(B, mp, *pool.shape[1:]).permute(0, 2, 1, 3, 4)
+    return g.reshape(B, pool.shape[1], mp * pool.shape[2], pool.shape[3]).contiguous()
+
+
 @pytest.mark.parametrize("name,page", PAGED, ids=[f"{n}-p{p}" for n, p in PAGED])
 def test_paged_attention_equals_dense(dev, name, page):
     """Paged attention over shuffled pages gives bit for bit the dense attention's output on the
     same data (same schedule, same tensor-core products), and matches the oracle."""
     wl = W.make_workload(SMALL[name], device=dev, cache_pad=70)
     pg = W.to_paged(wl, page, seed=5)
-    out, lse, st = parity.gpu_attention(wl)
+    # The dense reference gets the paged call's capacity (max_pages * page): the grid is sized
+    # from the capacity, and equal schedules give equal roundings.
+    dense = dict(wl, cap=pg["max_pages"] * page,
+                 k_cache=_pool_to_dense(pg["k_pool"], pg["block_table"]),
+                 v_cache=_pool_to_dense(pg["v_pool"], pg["block_table"]))
+    out, lse, st = parity.gpu_attention(dense)
     max_k = int(wl["n_draft"].max())
     out_p = torch.full_like(out, float("nan"))
     lse_p = torch.full_like(lse, float("nan"))
