@@ -170,7 +170,7 @@ def _top2_margin(l):
 
 
 def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
-                  margin=1e-3):
+                  margin=1e-3, temperature=None):
     """Accept/reject of every sequence, given its verifier logits.
 
     logits [R, V] (rows as in ``verify_attention``); draft_tokens [R-B] with
@@ -185,6 +185,10 @@ def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_dra
       flag_sample [B]    the sampled token's u*Z lies within margin*r(x) of an
                          edge of its CDF interval (stochastic only);
       fallback [B]       residual had no mass, p used instead.
+
+    ``temperature`` [B] (optional): the verifier samples from p = softmax(l / T_b)
+    (the paper mentions sampling for diversity, Sec. III-A, without fixing it);
+    greedy decisions, which take the argmax, are unaffected.
     """
     B = len(n_draft)
     acc = np.zeros(B, dtype=np.int64)
@@ -197,6 +201,7 @@ def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_dra
         r0 = int(cu_q[b])
         d0 = r0 - b
         stochastic = int(mode[b]) == STOCHASTIC
+        t_b = 1.0 if temperature is None else float(temperature[b])
         a = 0
         for i in range(k):
             l = _f64(logits[r0 + i])
@@ -206,7 +211,7 @@ def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_dra
                 if _top2_margin(l) < margin:
                     flag_dec[b] = True
             else:
-                p = softmax(l)
+                p = softmax(l / t_b)
                 qd = float(draft_probs[d0 + i][d])
                 u = float(uniforms[r0 + i])
                 if qd > 0.0:
@@ -226,7 +231,7 @@ def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_dra
             if _top2_margin(lr) < margin:
                 flag_dec[b] = True
         else:
-            p = softmax(lr)
+            p = softmax(lr / t_b)
             if a < k:
                 r, Z, fb = residual_distribution(p, draft_probs[d0 + a])
             else:

@@ -511,6 +511,45 @@ def check_paged_matches_dense(o, seed=13):
     assert np.isnan(k3[perm[B * max_pages:]]).all()  # pages outside the table untouched
 
 
+# ----------------------------------------------------------------------------
+# Temperature of the verifier's distribution
+# ----------------------------------------------------------------------------
+def check_temperature_worked_example(o):
+    g = _golden()["temperature"]
+    l = np.asarray(g["logits"])
+    T = g["T"]
+    logits = np.stack([l, l])
+    a = g["accept"]
+    q = np.asarray(a["q"])[None]
+    res = o.verify_accept(logits, [a["draft"]], q, [a["u_accept"], 0.5], [1], [0, 2], [1], temperature=[T])
+    assert res["accepted_len"][0] == 1
+    res = o.verify_accept(logits, [a["draft"]], q, [a["u_reject"], 0.5], [1], [0, 2], [1], temperature=[T])
+    assert res["accepted_len"][0] == 0
+    for u, x in g["bonus"]:
+        res = o.verify_accept(l[None], [], np.zeros((0, 3)), [u], [1], [0, 1], [0], temperature=[T])
+        assert res["next_token"][0] == x, (u, x)
+    # Greedy decisions ignore the temperature.
+    res = o.verify_accept(logits, [1], None, [0.5, 0.5], [0], [0, 2], [1], temperature=[T])
+    assert res["accepted_len"][0] == 1 and res["next_token"][0] == 1
+
+
+def check_temperature_output_law(o, n=40000, seed=14):
+    """Rejection sampling at temperature T reproduces softmax(l / T) (Sec. III-C with p at T)."""
+    rng = np.random.default_rng(seed)
+    V, k, T = 6, 1, 0.5
+    L = rng.standard_normal((k + 1, V))
+    P = np.exp(L / T)
+    P /= P.sum(axis=1, keepdims=True)
+    Q = rng.dirichlet(np.ones(V), size=k)
+    drafts = rng.choice(V, size=n, p=Q[0])
+    u = rng.random(n * (k + 1))
+    res = o.verify_accept(np.tile(L, (n, 1)), drafts, np.tile(Q, (n, 1)), u, np.ones(n, int),
+                          np.arange(n + 1) * (k + 1), np.full(n, k), temperature=np.full(n, T))
+    first = np.where(res["accepted_len"] >= 1, drafts, res["next_token"])
+    _, pv = stats.chisquare(np.bincount(first, minlength=V), P[0] * n)
+    assert pv > 1e-3, pv
+
+
 ALL_CHECKS = [
     check_attention_worked_examples, check_attention_vs_sdpa, check_attention_special_cases,
     check_attention_gqa_mapping, check_logits_one_hot, check_acceptance_worked_examples,
@@ -518,5 +557,6 @@ ALL_CHECKS = [
     check_stochastic_output_law, check_progress_and_bounds, check_greedy_identity,
     check_kv_commit, check_rope_worked_examples, check_rope_vs_complex_rotation,
     check_rope_relative_position, check_qkv_projection_layout, check_kv_write_slots,
-    check_paged_worked_example, check_paged_matches_dense,
+    check_paged_worked_example, check_paged_matches_dense, check_temperature_worked_example,
+    check_temperature_output_law,
 ]

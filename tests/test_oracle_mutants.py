@@ -60,6 +60,9 @@ MUTANTS = {
     "keys_not_rotated": ("return rope(q, pos[:, None], theta), rope(k, pos[:, None], theta), v",
                          "return rope(q, pos[:, None], theta), k, v"),
     "kv_write_wrong_slot": ("kc[seq[r], :, pos[r]] = k[r]", "kc[seq[r], :, pos[r] - 1] = k[r]"),
+    # Temperature of p.
+    "temperature_multiplies": ("p = softmax(l / t_b)", "p = softmax(l * t_b)"),
+    "temperature_ignored_in_sampling": ("p = softmax(lr / t_b)", "p = softmax(lr)"),
     # Paged cache addressing.
     "paged_row_from_page_index": ("return int(block_table[b][s // page]), s % page",
                                   "return int(block_table[b][s // page]), s // page"),
