@@ -222,6 +222,27 @@ spade_status spade_verify_accept(const void *hidden, const void *w_lm,
                                  size_t workspace_bytes, int32_t *status,
                                  spade_stream_t stream);
 
+/*
+ * spade_verify_accept with a softmax temperature per sequence: the verifier's
+ * distribution is p = softmax(logits / temperature[b]) in the accept test and
+ * in the residual / bonus draw (sampling "for diversity", Sec. III-A; the
+ * test and p' of Sec. III-C are unchanged otherwise).  Greedy sequences take
+ * the argmax, which no positive temperature changes.  draft_probs is the draft
+ * model's distribution at its own temperature, as the caller produced it.
+ *   temperature  float32 [B] device array, each finite and > 0 (a value that
+ *                is not is taken as 1 and sets SPADE_DEV_BAD_INDEX)
+ * The row statistics of spade_accept_stats_layout are then those of l / T.
+ * Every other argument is that of spade_verify_accept.
+ */
+spade_status spade_verify_accept_temperature(const void *hidden, const void *w_lm,
+                                             const int32_t *draft_tokens, const float *draft_probs,
+                                             const float *uniforms, const int32_t *mode,
+                                             const float *temperature, const int32_t *cu_q,
+                                             const int32_t *n_draft, int32_t *accepted_len,
+                                             int32_t *next_token, int32_t B, int32_t R, int32_t H,
+                                             int32_t V, void *workspace, size_t workspace_bytes,
+                                             int32_t *status, spade_stream_t stream);
+
 /* Bytes of workspace spade_verify_accept needs (0 on invalid sizes). */
 size_t spade_accept_workspace_size(int32_t B, int32_t R, int32_t H, int32_t V);
 

@@ -85,6 +85,8 @@ def load():
     lib.spade_verify_accept_commit.argtypes = [_vp] * 13 + [_i32] * 7 + [_vp, _sz, _vp, _vp]
     lib.spade_accept_workspace_size.restype = _sz
     lib.spade_accept_workspace_size.argtypes = [_i32] * 4
+    lib.spade_verify_accept_temperature.restype = _i32
+    lib.spade_verify_accept_temperature.argtypes = [_vp] * 11 + [_i32] * 4 + [_vp, _sz, _vp, _vp]
     lib.spade_accept_stats_layout.restype = _i32
     lib.spade_accept_stats_layout.argtypes = [_i32] * 4 + [_vp, _vp, _vp]
     lib.spade_accept_launches.restype = _i32
@@ -258,8 +260,9 @@ def accept_workspace(B, R, H, V, device="cuda"):
 
 
 def spade_verify_accept(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
-                        accepted_len, next_token, *, workspace, status, stream=None):
-    """Greedy / rejection-sampling verification of every sequence (see include/spade.h)."""
+                        accepted_len, next_token, *, workspace, status, stream=None, temperature=None):
+    """Greedy / rejection-sampling verification of every sequence (see include/spade.h); with
+    ``temperature`` ([B] float32) the verifier's p is softmax(logits / T)."""
     _need(hidden, "hidden", torch.bfloat16, 2)
     _need(w_lm, "w_lm", torch.bfloat16, 2)
     _need(uniforms, "uniforms", torch.float32, 1)
@@ -277,10 +280,19 @@ def spade_verify_accept(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode,
         raise ValueError("inconsistent accept shapes")
     if draft_probs is not None and tuple(draft_probs.shape) != (R - B, V):
         raise ValueError("draft_probs must be [R - B, V]")
-    rc = load().spade_verify_accept(
-        _ptr(hidden), _ptr(w_lm), _ptr(draft_tokens), _ptr(draft_probs), _ptr(uniforms), _ptr(mode),
-        _ptr(cu_q), _ptr(n_draft), _ptr(accepted_len), _ptr(next_token), B, R, H, V,
-        _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream))
+    if temperature is None:
+        rc = load().spade_verify_accept(
+            _ptr(hidden), _ptr(w_lm), _ptr(draft_tokens), _ptr(draft_probs), _ptr(uniforms), _ptr(mode),
+            _ptr(cu_q), _ptr(n_draft), _ptr(accepted_len), _ptr(next_token), B, R, H, V,
+            _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream))
+    else:
+        _need(temperature, "temperature", torch.float32, 1)
+        if temperature.numel() != B:
+            raise ValueError("temperature must be [B]")
+        rc = load().spade_verify_accept_temperature(
+            _ptr(hidden), _ptr(w_lm), _ptr(draft_tokens), _ptr(draft_probs), _ptr(uniforms), _ptr(mode),
+            _ptr(temperature), _ptr(cu_q), _ptr(n_draft), _ptr(accepted_len), _ptr(next_token), B, R, H, V,
+            _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream))
     _check_rc(rc)
     return accepted_len, next_token
 

@@ -97,6 +97,7 @@ struct Params {
   int4 *samp;        // [B]: sample specs written by kStatsOnly, read by kPresampled:
                      //      draft_probs row (-1: sample p), uniform bits, output index, row
   int *samp_count;   // number of specs
+  const float *temperature;  // [B] softmax temperature of each sequence, or null (all 1)
   __nv_bfloat16 *hidden_s;      // [B, H]: gathered hidden rows of the samples
   const __nv_bfloat16 *hidden;  // the call's hidden rows (gather source)
   // Fused KV commit (null kc: not requested): clear the rejected draft slots of
@@ -225,6 +226,18 @@ __device__ __forceinline__ void stat_merge(float &m, float &s, int &i, float om,
   }
   if (om > m || (om == m && oi < i)) i = oi;
   m = M;
+}
+
+// 1 / T for sequence b: p = softmax(l / T).  A temperature that is not
+// positive and finite is reported and taken as 1.
+__device__ __forceinline__ float inv_temp(const Params &p, int b) {
+  if (p.temperature == nullptr || b < 0) return 1.f;
+  const float t = __ldg(p.temperature + b);
+  if (!(t > 0.f) || !(t < INFINITY)) {
+    atomicOr(p.status, SPADE_DEV_BAD_INDEX);
+    return 1.f;
+  }
+  return 1.f / t;
 }
 
 // Float-float numbers (hi + lo, about 48 significant bits) for the sums that
@@ -780,12 +793,15 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             __syncwarp();
             const int n = r0 + lane;
             if (lane < nc && n < p.R) {
+              // Logits at the row's temperature, l / T (T = 1 without temperatures).
+              const int sq = p.kind == kPresampled ? (n < *p.samp_count ? p.samp[n].z : -1) : s_seq[n];
+              const float it = inv_temp(p, sq);
               float x[32];
               float m = -INFINITY;
               int mi = 0;
 #pragma unroll
               for (int i = 0; i < 32; ++i) {
-                x[i] = T[i * 33 + lane];
+                x[i] = T[i * 33 + lane] * it;
                 if (x[i] > m) { m = x[i]; mi = i; }
               }
               float sm = 0.f;
@@ -795,7 +811,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               }
               stat_merge(rm[cj], rs[cj], ri[cj], m, sm, m == -INFINITY ? INT_MAX : vlane0 + mi);
               const int d = s_draft[n];
-              if (d >= vlane0 && d < vlane0 + 32 && d < v_hi) p.ldraft[n] = T[(d - vlane0) * 33 + lane];
+              if (d >= vlane0 && d < vlane0 + 32 && d < v_hi) p.ldraft[n] = T[(d - vlane0) * 33 + lane] * it;
             }
             __syncwarp();
           }
@@ -1130,7 +1146,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             // broadcasts them.  The loop body has no divergent branch: tiles
             // past the slice re-read its last tile and store zeros.
             int n_l = -1, hq_l = 0;
-            float m_l = 0.f, is_l = 0.f;
+            float m_l = 0.f, is_l = 0.f, it_l = 1.f;
             if (lane < ng) {
               const int b = s_slist[g0 + lane];
               n_l = (attempt == 0 || s_usep[b]) ? s_rstar[b] : -1;
@@ -1138,6 +1154,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               if (n_l >= 0) {
                 m_l = g_m[n_l];
                 is_l = 1.f / g_s[n_l];
+                it_l = inv_temp(p, s_outb[b]);
               }
             }
 #pragma unroll 1
@@ -1145,6 +1162,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               const int n = __shfl_sync(0xffffffffu, n_l, gi);
               const bool hasq = __shfl_sync(0xffffffffu, hq_l, gi) != 0;
               const float M = __shfl_sync(0xffffffffu, m_l, gi), invS = __shfl_sync(0xffffffffu, is_l, gi);
+              const float IT = __shfl_sync(0xffffffffu, it_l, gi);  // 1 / T of the row
               uint32_t raw[kTiles];
               if (n >= 0) {
 #pragma unroll
@@ -1169,7 +1187,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
 #pragma unroll
               for (int t = 0; t < kTiles; ++t) {
                 const int e = t * kTileV + q4 * 32 + lane;  // < kFastSlice: inside the row's buffers
-                const float pv = ex2((__uint_as_float(raw[t]) - M) * kLog2e) * invS;
+                const float pv = ex2((__uint_as_float(raw[t]) * IT - M) * kLog2e) * invS;
                 const float rv = hasq ? fmaxf(0.f, pv - qv[t]) : pv;
                 rrow[(e >> 5) * kSegPad + (e & 31)] = e < slen ? rv : 0.f;
               }
@@ -1220,7 +1238,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           if (nb == 0) break;
           const float *qrow[kG];
           int nrow[kG];
-          float M[kG], invS[kG];
+          float M[kG], invS[kG], IT[kG];
           ff2 z[kG], zp[kG];
   #pragma unroll
           for (int g = 0; g < kG; ++g) {
@@ -1229,6 +1247,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             qrow[g] = (attempt == 0 && s_qidx[b] >= 0) ? p.draft_probs + static_cast<size_t>(s_qidx[b]) * p.V : nullptr;
             M[g] = g_m[nrow[g]];
             invS[g] = 1.f / g_s[nrow[g]];
+            IT[g] = inv_temp(p, s_outb[b]);
             z[g] = ff2{0.f, 0.f};
             zp[g] = ff2{0.f, 0.f};
           }
@@ -1258,7 +1277,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               for (int j = 0; j < 8; ++j) {
                 const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
                 if (g < nb && j < nj && v < v_hi) {
-                  const float pv = ex2((__uint_as_float(raw[g][j]) - M[g]) * kLog2e) * invS[g];
+                  const float pv = ex2((__uint_as_float(raw[g][j]) * IT[g] - M[g]) * kLog2e) * invS[g];
                   zp[g] = ff_add_f(zp[g], pv);
                   z[g] = ff_add_f(z[g], qrow[g] ? fmaxf(0.f, pv - qv[g][j]) : pv);
                 }
@@ -1380,6 +1399,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         const bool usep = s_usep[b] != 0;
         const float *qrow = (s_qidx[b] >= 0 && !usep) ? p.draft_probs + static_cast<size_t>(s_qidx[b]) * p.V : nullptr;
         const float M = g_m[n], invS = 1.f / g_s[n];
+        const float IT = inv_temp(p, s_outb[b]);  // 1 / T of the row
         // (1) mass of every 32-entry segment (tile j, lane quarter q4) of the slice:
         //     from phase C's shared-memory sums, else recomputed.
         if (fastc) {
@@ -1408,7 +1428,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
             float rv = 0.f;
             if (j < nj && v < v_hi) {
-              const float pv = ex2((__uint_as_float(raw[j]) - M) * kLog2e) * invS;
+              const float pv = ex2((__uint_as_float(raw[j]) * IT - M) * kLog2e) * invS;
               rv = qrow ? fmaxf(0.f, pv - qv[j]) : pv;
             }
             const ff2 seg = warp_sum_ff(ff2{rv, 0.f});
@@ -1447,7 +1467,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           tmem_wait_ld();
           float rv = 0.f;
           if (v < v_hi) {
-            const float pv = ex2((__uint_as_float(raw) - M) * kLog2e) * invS;
+            const float pv = ex2((__uint_as_float(raw) * IT - M) * kLog2e) * invS;
             rv = qrow ? fmaxf(0.f, pv - qv) : pv;
           }
           const ff2 incl = warp_scan_ff(ff2{rv, 0.f}, lane);
@@ -1840,7 +1860,8 @@ static spade_status verify_accept_impl(const void *hidden, const void *w_lm,
                                        int32_t *accepted_len, int32_t *next_token, int32_t B,
                                        int32_t R, int32_t H, int32_t V, void *workspace,
                                        size_t workspace_bytes, int32_t *status,
-                                       spade_stream_t stream, const CommitArgs *cm) {
+                                       spade_stream_t stream, const CommitArgs *cm,
+                                       const float *temperature = nullptr) {
   using namespace accept;
   if (!hidden || !w_lm || !uniforms || !mode || !cu_q || !n_draft || !accepted_len ||
       !next_token || !status || (R > B && !draft_tokens))
@@ -1866,6 +1887,7 @@ static spade_status verify_accept_impl(const void *hidden, const void *w_lm,
   Params p{};
   p.draft_tokens = draft_tokens;
   p.draft_probs = draft_probs;
+  p.temperature = temperature;
   p.qbulk = draft_probs != nullptr && aligned(draft_probs, 16) && V % 4 == 0;
   p.uniforms = uniforms;
   p.mode = mode;
@@ -1943,4 +1965,15 @@ extern "C" spade_status spade_verify_accept_commit(
   return accept::verify_accept_impl(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q,
                                     n_draft, accepted_len, next_token, B, R, H, V, workspace,
                                     workspace_bytes, status, stream, &cm);
+}
+
+extern "C" spade_status spade_verify_accept_temperature(
+    const void *hidden, const void *w_lm, const int32_t *draft_tokens, const float *draft_probs,
+    const float *uniforms, const int32_t *mode, const float *temperature, const int32_t *cu_q,
+    const int32_t *n_draft, int32_t *accepted_len, int32_t *next_token, int32_t B, int32_t R, int32_t H,
+    int32_t V, void *workspace, size_t workspace_bytes, int32_t *status, spade_stream_t stream) {
+  if (!temperature) return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_temperature: null temperature");
+  return accept::verify_accept_impl(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
+                                    accepted_len, next_token, B, R, H, V, workspace, workspace_bytes, status,
+                                    stream, nullptr, temperature);
 }

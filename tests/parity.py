@@ -49,7 +49,7 @@ def gpu_attention(wl, workspace=None, status=None):
     return out, lse, status
 
 
-def gpu_accept(wl, workspace=None, status=None):
+def gpu_accept(wl, workspace=None, status=None, temperature=None):
     dev = wl["hidden"].device
     B = wl["B"]
     acc = torch.full((B,), -7, dtype=torch.int32, device=dev)
@@ -60,7 +60,7 @@ def gpu_accept(wl, workspace=None, status=None):
         status = spade.status_tensor(dev)
     spade.spade_verify_accept(wl["hidden"], wl["w_lm"], wl["draft_tokens"], wl["draft_probs"],
                               wl["uniforms"], wl["mode"], wl["cu_q"], wl["n_draft"], acc, tok,
-                              workspace=workspace, status=status)
+                              workspace=workspace, status=status, temperature=temperature)
     return acc, tok, status
 
 
@@ -85,10 +85,10 @@ def oracle_logits(wl):
     return O.lm_logits(to_np(wl["hidden"]), to_np(wl["w_lm"]))
 
 
-def oracle_accept_from_logits(wl, logits):
+def oracle_accept_from_logits(wl, logits, temperature=None):
     return O.verify_accept(logits, to_np(wl["draft_tokens"]), to_np(wl["draft_probs"]),
                            to_np(wl["uniforms"]), to_np(wl["mode"]), to_np(wl["cu_q"]),
-                           to_np(wl["n_draft"]))
+                           to_np(wl["n_draft"]), temperature=temperature)
 
 
 def oracle_attention(wl, rows=None):

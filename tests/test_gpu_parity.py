@@ -593,3 +593,53 @@ def test_paged_qkv_rope(dev):
     keep = ~written
     np.testing.assert_array_equal(gk.transpose(0, 2, 1, 3)[keep], k0.transpose(0, 2, 1, 3)[keep])
     np.testing.assert_array_equal(gv.transpose(0, 2, 1, 3)[keep], v0.transpose(0, 2, 1, 3)[keep])
+
+
+# ---------------------------------------------------------------------------
+# Temperature of the verifier's distribution: p = softmax(l / T_b).
+
+TEMP = {
+    "temp_resident": W.WorkloadSpec("temp_resident", B=6, Hq=4, Hkv=4, D=64, H=256, V=5000, ctx=(1, 64),
+                                    k=(1, 6), mode="mixed", seed=61),
+    "temp_wide_slices": W.WorkloadSpec("temp_wide_slices", B=3, Hq=4, Hkv=4, D=64, H=256, V=160000, ctx=(1, 64),
+                                       k=(1, 3), mode="stochastic", seed=62),
+    "temp_two_pass": W.WorkloadSpec("temp_two_pass", B=40, Hq=4, Hkv=4, D=64, H=256, V=9100, ctx=(1, 64),
+                                    k=(6, 9), mode="mixed", seed=63),
+}
+
+
+@pytest.mark.parametrize("name", sorted(TEMP) + ["llama3_8b"])
+def test_accept_temperature(dev, name):
+    spec = TEMP.get(name) or W.SPECS[name]
+    wl = W.make_workload(spec, device=dev)
+    g = torch.Generator().manual_seed(5)
+    T = (0.3 + 1.7 * torch.rand(wl["B"], generator=g)).to(torch.float32)
+    acc, tok, st = parity.gpu_accept(wl, temperature=T.to(dev))
+    ws = None
+    torch.cuda.synchronize()
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0
+    logits = parity.oracle_logits(wl)
+    ref = parity.oracle_accept_from_logits(wl, logits, temperature=T.numpy())
+    cmp = parity.compare_accept(acc, tok, ref)
+    assert cmp["mismatch_unflagged"] == 0, cmp
+    assert cmp["flagged"] <= _flag_bound(wl["B"]), cmp
+    # The decisions depend on T: the same call at T = 1 disagrees somewhere (stochastic rows).
+    ref1 = parity.oracle_accept_from_logits(wl, logits)
+    assert not (np.array_equal(ref1["accepted_len"], ref["accepted_len"])
+                and np.array_equal(ref1["next_token"], ref["next_token"]))
+
+
+def test_accept_temperature_row_stats(dev):
+    """The on-chip statistics are those of l / T (max, log-sum-exp, draft logit)."""
+    spec = TEMP["temp_resident"]
+    wl = W.make_workload(spec, device=dev)
+    T = torch.linspace(0.4, 1.9, wl["B"], dtype=torch.float32)
+    ws = spade.accept_workspace(wl["B"], wl["R"], wl["H"], wl["V"], device=dev)
+    acc, tok, st = parity.gpu_accept(wl, workspace=ws, temperature=T.to(dev))
+    torch.cuda.synchronize()
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0
+    logits = parity.oracle_logits(wl)
+    seq, _ = O.verify_positions(parity.to_np(wl["ctx_lens"]), parity.to_np(wl["n_draft"]), parity.to_np(wl["cu_q"]))
+    scaled = logits / T.numpy().astype(np.float64)[seq][:, None]
+    rs = parity.compare_row_stats(spade.read_accept_stats(ws, wl["B"], wl["R"], wl["H"], wl["V"]), scaled, wl)
+    assert rs["max"] <= 1 and rs["lse"] <= 1 and rs["draft_logit"] <= 1 and rs["argmax_mismatch"] == 0, rs
