@@ -455,6 +455,8 @@ def run_spade(args, ws, rank, local):
         base, par = cpu_baseline(wl_cpu, acc.cpu(), tok.cpu())
         line["cpu_baseline"] = base
         line["parity"] = par
+    if rank == 0 and ws == 1 and not args.no_loop:
+        line["speculative_loop"] = loop_report(dev)
     if rank == 0 and ws == 1 and not args.no_per_workload:
         line["per_workload"] = per_workload(args, dev, skip=args.workload)
     return line
@@ -577,6 +579,34 @@ def per_workload(args, dev, skip):
         del wl
         torch.cuda.empty_cache()
     return res
+
+
+def loop_report(dev, B=8, max_new=64):
+    """Algorithm 1 with the toy verifier (one layer through the library) for draft lengths
+    0 (plain decoding), 1, 2, 4, 8: verifier calls per generated token and the acceptance
+    rate, greedy and stochastic -- the synthetic analogue of the paper's cloud-call counts."""
+    import numpy as np
+
+    from paper_2608_13076_gb300 import speculative as S
+
+    ver = S.ToyVerifier(S.ToyConfig(), B, cap=2048, seed=3, device=dev)
+    g = np.random.default_rng(4)
+    prompts = [list(g.integers(0, ver.cfg.V - 1, size=int(n))) for n in g.integers(8, 64, size=B)]
+    out = {"model": "toy verifier: V 2048, H 512, GQA 8/2, D 64, one layer; drafter: its residual path",
+           "sequences": B, "max_new": max_new}
+    for name, mode in (("greedy", S.GREEDY), ("stochastic", S.STOCHASTIC)):
+        rows = []
+        for d in (0, 1, 2, 4, 8):
+            t0 = time.perf_counter()
+            res = S.speculative_decode(ver, prompts, d=d, max_new=max_new, mode=mode, seed=11)
+            wall = time.perf_counter() - t0
+            toks = sum(len(t) for t in res.tokens)
+            rows.append({"d": d, "verifier_calls": sum(res.calls_per_seq), "tokens": toks,
+                         "tokens_per_call": toks / max(1, sum(res.calls_per_seq)),
+                         "acceptance": res.accepted / res.drafted if res.drafted else None,
+                         "batch_calls": res.calls, "wall_s": wall})
+        out[name] = rows
+    return out
 
 
 def _npf(t):
@@ -703,6 +733,7 @@ def main():
     ap.add_argument("--no-per-workload", action="store_true",
                     help="skip the device timing of the suite's other workloads")
     ap.add_argument("--per-workload-steps", type=int, default=20)
+    ap.add_argument("--no-loop", action="store_true", help="skip the decoding-loop report")
     ap.add_argument("--separate-commit", action="store_true",
                     help="run the KV commit as its own launch instead of inside the LM-head kernel")
     args = ap.parse_args()
