@@ -504,6 +504,7 @@ def _time_qkv(spec, wl, dev, flush_buf=None, launches=20):
     flop = 2.0 * R * (Hq + 2 * Hkv) * D * H
     return {"kernel": "qkv_rope_kernel", "us": t * 1e6, "bound": "hbm", "achieved": nbytes / t / 1e9, "peak": hbm,
             "unit": "GB/s", "frac": nbytes / t / 1e9 / hbm, "algorithmic_bytes": nbytes, "tflops": flop / t / 1e12,
+            "traffic": _traffic("qkv_rope_kernel", spec.name),
             "launches": launches, "l2": "flushed before each launch",
             "note": "not part of the timed step (the step's q and cache slots are inputs); measured after it"}
 
