@@ -476,10 +476,11 @@ def _time_qkv(spec, wl, dev, flush_buf=None, launches=20):
         flush_buf = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
     kc, vc = wl["k_cache"].clone(), wl["v_cache"].clone()  # the step's caches stay as they were
     stream = torch.cuda.current_stream()
+    max_k = int(wl["n_draft"].max())  # read once: a device read inside the loop would synchronise it
+
     def call():
         spade.spade_verify_qkv_rope(x, w, wl["ctx_lens"], wl["n_draft"], wl["cu_q"], q, kc, vc, Hq=wl["Hq"],
-                                    Hkv=wl["Hkv"], rope_theta=spec.rope_theta, max_k=int(wl["n_draft"].max()),
-                                    status=status)
+                                    Hkv=wl["Hkv"], rope_theta=spec.rope_theta, max_k=max_k, status=status)
 
     # The first launch of a shape also runs one-time host work (occupancy queries):
     # finish it before the timed loop, which must not wait on the host.
