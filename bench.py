@@ -477,10 +477,12 @@ def _time_qkv(spec, wl, dev, flush_buf=None, launches=20):
     kc, vc = wl["k_cache"].clone(), wl["v_cache"].clone()  # the step's caches stay as they were
     stream = torch.cuda.current_stream()
     max_k = int(wl["n_draft"].max())  # read once: a device read inside the loop would synchronise it
+    ws = spade.qkv_workspace(wl["R"], wl["Hq"], wl["Hkv"], wl["D"], device=dev)
 
     def call():
         spade.spade_verify_qkv_rope(x, w, wl["ctx_lens"], wl["n_draft"], wl["cu_q"], q, kc, vc, Hq=wl["Hq"],
-                                    Hkv=wl["Hkv"], rope_theta=spec.rope_theta, max_k=max_k, status=status)
+                                    Hkv=wl["Hkv"], rope_theta=spec.rope_theta, max_k=max_k, workspace=ws,
+                                    status=status)
 
     # The first launch of a shape also runs one-time host work (occupancy queries):
     # finish it before the timed loop, which must not wait on the host.

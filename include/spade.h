@@ -99,15 +99,25 @@ typedef enum {
  *   status      device int32: a sequence whose block is invalid
  *               (SPADE_DEV_BAD_INDEX) or does not fit its cache
  *               (SPADE_DEV_CAPACITY) is skipped; none of its rows is written
- * Every pointer is a 16-byte aligned device pointer.  Allocates nothing and
- * needs no workspace: the split-K partial sums meet in distributed shared
- * memory inside the launch.  Launched with programmatic dependent launch.
+ *   workspace   device scratch of at least spade_qkv_workspace_size(R, Hq, Hkv, D)
+ *               bytes, 256-byte aligned, ZEROED ONCE by the caller after
+ *               allocation; every call that completes leaves its counters
+ *               zeroed again.  Calls that share a workspace must be ordered.
+ * Every pointer is a 16-byte aligned device pointer.  The contraction is split
+ * over every SM; the split parts' fp32 sums meet in the workspace and are
+ * added in a fixed order, so results do not depend on timing.  Launched with
+ * programmatic dependent launch.
  */
 spade_status spade_verify_qkv_rope(const void *x, const void *w_qkv, const int32_t *ctx_lens,
                                    const int32_t *n_draft, const int32_t *cu_q, void *q_out,
                                    void *k_cache, void *v_cache, int32_t B, int32_t R, int32_t H,
                                    int32_t Hq, int32_t Hkv, int32_t D, int32_t cap, int32_t max_k,
-                                   float rope_theta, int32_t *status, spade_stream_t stream);
+                                   float rope_theta, void *workspace, size_t workspace_bytes,
+                                   int32_t *status, spade_stream_t stream);
+
+/* Bytes of workspace spade_verify_qkv_rope (and its paged form) needs for these
+ * sizes on the current device (0 on invalid sizes). */
+size_t spade_qkv_workspace_size(int32_t R, int32_t Hq, int32_t Hkv, int32_t D);
 
 /* ------------------------------------------------------------------------ */
 /* Verify attention (Sec. III-B verification stage; Algorithm 1 cloud step)  */
@@ -364,7 +374,8 @@ spade_status spade_verify_qkv_rope_paged(const void *x, const void *w_qkv, const
                                          int32_t B, int32_t R, int32_t H, int32_t Hq, int32_t Hkv,
                                          int32_t D, int32_t page_size, int32_t num_pages,
                                          int32_t max_pages, int32_t max_k, float rope_theta,
-                                         int32_t *status, spade_stream_t stream);
+                                         void *workspace, size_t workspace_bytes, int32_t *status,
+                                         spade_stream_t stream);
 
 /* ------------------------------------------------------------------------ */
 /* Diagnostics                                                               */

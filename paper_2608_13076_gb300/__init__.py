@@ -24,7 +24,7 @@ from . import _build
 __all__ = [
     "SpadeError", "load", "build", "library_path",
     "spade_verify_attention", "spade_verify_accept", "spade_kv_commit", "spade_verify_attention_noalloc",
-    "spade_verify_qkv_rope", "spade_verify_attention_paged", "spade_kv_commit_paged",
+    "spade_verify_qkv_rope", "spade_qkv_workspace_size", "qkv_workspace", "spade_verify_attention_paged", "spade_kv_commit_paged",
     "spade_verify_qkv_rope_paged",
     "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_accept_launches",
     "spade_accept_stats_layout", "read_accept_stats", "spade_verify_accept_commit", "spade_selftest_wait_timeout",
@@ -94,13 +94,15 @@ def load():
     lib.spade_selftest_wait_timeout.restype = _i32
     lib.spade_selftest_wait_timeout.argtypes = [_vp, _i32, _vp]
     lib.spade_verify_qkv_rope.restype = _i32
-    lib.spade_verify_qkv_rope.argtypes = [_vp] * 8 + [_i32] * 8 + [ctypes.c_float, _vp, _vp]
+    lib.spade_verify_qkv_rope.argtypes = [_vp] * 8 + [_i32] * 8 + [ctypes.c_float, _vp, _sz, _vp, _vp]
+    lib.spade_qkv_workspace_size.restype = _sz
+    lib.spade_qkv_workspace_size.argtypes = [_i32] * 4
     lib.spade_verify_attention_paged.restype = _i32
     lib.spade_verify_attention_paged.argtypes = [_vp] * 9 + [_i32] * 9 + [_vp, _sz, _vp, _vp]
     lib.spade_kv_commit_paged.restype = _i32
     lib.spade_kv_commit_paged.argtypes = [_vp] * 6 + [_i32] * 6 + [_vp, _vp]
     lib.spade_verify_qkv_rope_paged.restype = _i32
-    lib.spade_verify_qkv_rope_paged.argtypes = [_vp] * 9 + [_i32] * 10 + [ctypes.c_float, _vp, _vp]
+    lib.spade_verify_qkv_rope_paged.argtypes = [_vp] * 9 + [_i32] * 10 + [ctypes.c_float, _vp, _sz, _vp, _vp]
     lib.spade_kv_commit.restype = _i32
     lib.spade_kv_commit.argtypes = [_vp] * 5 + [_i32] * 4 + [_vp, _vp]
     lib.spade_status_string.restype = ctypes.c_char_p
@@ -333,8 +335,20 @@ def spade_verify_accept_commit(hidden, w_lm, draft_tokens, draft_probs, uniforms
 
 
 # ---------------------------------------------------------------------------
+def spade_qkv_workspace_size(R, Hq, Hkv, D):
+    return int(load().spade_qkv_workspace_size(R, Hq, Hkv, D))
+
+
+def qkv_workspace(R, Hq, Hkv, D, device="cuda"):
+    """A zeroed workspace for spade_verify_qkv_rope (zeroed once; calls keep its counters zeroed)."""
+    n = spade_qkv_workspace_size(R, Hq, Hkv, D)
+    if n == 0:
+        raise SpadeError(-1, "spade_qkv_workspace_size returned 0: " + load().spade_last_error().decode())
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
 def spade_verify_qkv_rope(x, w_qkv, ctx_lens, n_draft, cu_q, q_out, k_cache, v_cache, *, Hq, Hkv,
-                          rope_theta, max_k, status, stream=None):
+                          rope_theta, max_k, workspace, status, stream=None):
     """q, k, v of the verify block (rotary embedding at ctx + i); K/V into cache slots ctx .. ctx + k."""
     _need(x, "x", torch.bfloat16, 2)
     _need(w_qkv, "w_qkv", torch.bfloat16, 2)
@@ -349,9 +363,11 @@ def spade_verify_qkv_rope(x, w_qkv, ctx_lens, n_draft, cu_q, q_out, k_cache, v_c
             or tuple(w_qkv.shape) != ((Hq + 2 * Hkv) * D, H) or ctx_lens.numel() != B or n_draft.numel() != B \
             or cu_q.numel() != B + 1:
         raise ValueError("inconsistent qkv_rope shapes")
+    _need(workspace, "workspace", torch.uint8, 1)
     rc = load().spade_verify_qkv_rope(
         _ptr(x), _ptr(w_qkv), _ptr(ctx_lens), _ptr(n_draft), _ptr(cu_q), _ptr(q_out), _ptr(k_cache), _ptr(v_cache),
-        B, R, H, Hq, Hkv, D, cap, int(max_k), float(rope_theta), _ptr(status), _stream(stream))
+        B, R, H, Hq, Hkv, D, cap, int(max_k), float(rope_theta), _ptr(workspace), workspace.numel(), _ptr(status),
+        _stream(stream))
     _check_rc(rc)
     return q_out
 
@@ -407,7 +423,7 @@ def spade_kv_commit_paged(k_pool, v_pool, block_table, ctx_lens, accepted_len, n
 
 
 def spade_verify_qkv_rope_paged(x, w_qkv, block_table, ctx_lens, n_draft, cu_q, q_out, k_pool, v_pool, *, Hq,
-                                rope_theta, max_k, status, stream=None):
+                                rope_theta, max_k, workspace, status, stream=None):
     """spade_verify_qkv_rope writing the block's K/V into a paged cache (see include/spade.h)."""
     _need(x, "x", torch.bfloat16, 2)
     _need(w_qkv, "w_qkv", torch.bfloat16, 2)
@@ -420,10 +436,11 @@ def spade_verify_qkv_rope_paged(x, w_qkv, block_table, ctx_lens, n_draft, cu_q, 
     if tuple(q_out.shape) != (R, Hq, D) or tuple(w_qkv.shape) != ((Hq + 2 * Hkv) * D, H) \
             or block_table.shape[0] != B or n_draft.numel() != B or cu_q.numel() != B + 1:
         raise ValueError("inconsistent paged qkv_rope shapes")
+    _need(workspace, "workspace", torch.uint8, 1)
     rc = load().spade_verify_qkv_rope_paged(
         _ptr(x), _ptr(w_qkv), _ptr(block_table), _ptr(ctx_lens), _ptr(n_draft), _ptr(cu_q), _ptr(q_out),
         _ptr(k_pool), _ptr(v_pool), B, R, H, Hq, Hkv, D, page_size, num_pages, max_pages, int(max_k),
-        float(rope_theta), _ptr(status), _stream(stream))
+        float(rope_theta), _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream))
     _check_rc(rc)
     return q_out
 

@@ -10,18 +10,22 @@
 //    tcgen05.mma kind::f16 (bf16 in, fp32 in tensor memory) with W's output
 //    rows on the MMA M side (128-row tiles: one head of dimension 128, or two
 //    of dimension 64, per tile) and the R verify rows on N.  At R = 72 the
-//    work is bound by streaming W from HBM (50 MB for the Llama-3-8B layer),
-//    so the grid is filled by splitting K: the `splits` CTAs of one tile form
-//    a thread-block cluster, each accumulates its share of the k-chunks, and
-//    the partial sums meet through distributed shared memory -- no workspace,
-//    no second launch.
+//    work is bound by streaming W from HBM (50 MB for the Llama-3-8B layer).
+//  * Stream-K over (tile, k-chunk) units: the units are laid end to end and
+//    cut into one equal range per SM, so every SM streams the same share of W
+//    whatever the tile count.  A CTA's range covers pieces of one to three
+//    tiles ("segments"); each segment accumulates in one of two tensor-memory
+//    buffers (the next segment's MMAs start while the last one is drained),
+//    and its fp32 partial goes to the CTA's own workspace slot.  The CTA that
+//    completes a tile last sums the tile's partials in CTA order -- the same
+//    order every call, so results do not depend on arrival order -- rotates
+//    query and key pairs (dimension j with j + D/2, angle pos *
+//    theta^(-2j/D), pos = ctx_b + i) and stores bf16: queries to q_out, keys
+//    and values to cache slot ctx_b + i of their sequence (or, for a paged
+//    cache, where the block table puts that slot).
 //  * Warp roles: warp 0 streams W and x tiles with TMA into a ring of stages;
 //    warp 1 issues the MMAs (one elected thread) and owns the tensor memory;
-//    warps 2-5 move the accumulator to shared memory and, after the cluster
-//    barrier, sum the partials of their share of (row, dimension pair) items,
-//    rotate query and key pairs (dimension j with j + D/2, angle pos *
-//    theta^(-2j/D), pos = ctx_b + i) and store bf16: queries to q_out, keys and
-//    values to cache slot ctx_b + i of their sequence.
+//    warps 2-5 drain accumulators, publish partials and run the reduction.
 //  * Programmatic dependent launch: barriers, tensor memory and tensor-map
 //    prefetch come before the wait on the previous kernel; the attention that
 //    follows may be scheduled while this kernel finishes.
@@ -39,27 +43,32 @@ constexpr int kTileM = 128;                     // W rows per tile (MMA M)
 constexpr int kKChunk = 64;                     // k elements per 128-byte swizzled row
 constexpr int kWBytes = kTileM * kKChunk * 2;   // 16 KB: one W tile x one k-chunk
 constexpr int kMaxR = 512;                      // verify rows per call
-constexpr int kMaxSplits = 8;                   // portable cluster size
 constexpr int kEpiWarps = 4;
+constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr int kThreads = 32 * (2 + kEpiWarps);
-constexpr int kRedCols = 256;                   // accumulator columns reduced per round
 constexpr int kSmemBudget = 220 * 1024;
 constexpr int kMaxStages = 8;
+
 
 struct Params {
   const int32_t *ctx_lens;
   const int32_t *n_draft;
   const int32_t *cu_q;
   __nv_bfloat16 *q_out;    // [R, Hq, D]
-  __nv_bfloat16 *k_cache;  // [B, Hkv, cap, D]
-  __nv_bfloat16 *v_cache;  // [B, Hkv, cap, D]
+  __nv_bfloat16 *k_cache;  // [B, Hkv, cap, D] (or a pool, see block_table)
+  __nv_bfloat16 *v_cache;
   int32_t *status;
+  float *partials;         // [num_ctas + tiles slots][Ncols][128] fp32 (workspace)
+  int32_t *counters;       // [tiles], zero between calls (workspace)
   int B, R, H, Hq, Hkv, D, cap, max_k;
-  int splits;   // CTAs per tile (cluster size), each with a contiguous share of the k-chunks
+  int tiles;    // (Hq + 2 Hkv) D / 128
   int KC;       // k-chunks (ceil(H / 64))
+  int units;    // tiles * KC
+  int num_ctas;
   int Ncols;    // R rounded up to 16: MMA N (two MMAs of <= 256 when above 256)
   int stages;   // ring depth
-  uint32_t tmem_cols;
+  int nbuf;     // accumulator buffers (2 when two fit in tensor memory)
+  uint32_t buf_cols, tmem_cols;
   float inv_freq[64];  // theta^(-2j/D), j < D/2, rounded from double on the host
   // Paged caches (block_table null: dense [B, Hkv, cap, D]): pools
   // [num_pages, Hkv, page_size, D], block_table [B, max_pages].
@@ -69,7 +78,7 @@ struct Params {
 
 // Shared-memory plan (offsets from a 1024-byte aligned base).
 struct Layout {
-  int stage_bytes, ring, rseq, rpos, bars, misc, total;
+  int stage_bytes, ring, rseq, rpos, bars, misc, freq, total;
 };
 __host__ __device__ inline Layout layout(int Ncols, int stages) {
   Layout L;
@@ -77,10 +86,145 @@ __host__ __device__ inline Layout layout(int Ncols, int stages) {
   L.ring = 0;
   L.rseq = stages * L.stage_bytes;   // int32 [kMaxR]: sequence of each row (-1: skip)
   L.rpos = L.rseq + kMaxR * 4;       // int32 [kMaxR]: position of each row
-  L.bars = L.rpos + kMaxR * 4;       // full[stages], empty[stages], acc
-  L.misc = L.bars + (2 * kMaxStages + 2) * 8;  // tmem base, abort flag
-  L.total = L.misc + 64 + 1024;      // + slack for the 1024-byte alignment
+  L.bars = L.rpos + kMaxR * 4;       // full[stages], empty[stages], acc_full[2], acc_empty[2]
+  L.misc = L.bars + (2 * kMaxStages + 4) * 8;  // tmem base, abort flag, last-arrival flag
+  L.freq = L.misc + 64;              // float [64]: rotary frequencies (per-thread indices
+                                     // into the parameter array would serialise)
+  L.total = L.freq + 64 * 4 + 1024;  // + slack for the 1024-byte alignment
   return L;
+}
+
+// Unit range [u0, u1) of CTA i, and the CTA whose range holds unit u.
+__host__ __device__ inline int range_lo(int units, int n, int i) {
+  return static_cast<int>(static_cast<int64_t>(units) * i / n);
+}
+__device__ inline int unit_owner(int units, int n, int u) {
+  return static_cast<int>((static_cast<int64_t>(u + 1) * n + units - 1) / units - 1);
+}
+
+// Arrival of one partial at its tile's counter (one thread, after a barrier
+// that orders the partial's stores before it): release publishes this CTA's
+// partial; for the last arrival, acquire makes every other one visible.
+__device__ __forceinline__ bool arrive_tile(int32_t *counter, int nparts) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;" : "=r"(old) : "l"(counter) : "memory");
+  return old == nparts - 1;
+}
+
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory"); }
+
+
+// Sine and cosine of pos * f: the product as an exact pair (a + e == pos * f),
+// reduced to [-pi, pi] with 2 pi split in two parts (Cody and Waite's method),
+// then the SFU's sine and cosine (accurate to a few 1e-7 on that interval).
+__device__ __forceinline__ void rope_angle(int pos, float f, float *sn, float *cs) {
+  const float x = static_cast<float>(pos);  // exact: positions are below 2^24
+  const float a = x * f;
+  const float e = fmaf(x, f, -a);
+  const float k = rintf(a * 0.15915494309189535f);           // 1 / (2 pi)
+  float r = fmaf(-k, 6.28318548202514648f, a);               // 2 pi rounded to float
+  r = fmaf(-k, -1.7484555314695172e-07f, r);                 // 2 pi minus that
+  __sincosf(r + e, sn, cs);
+}
+
+// The reduction of tile t once every part has been published: for each verify
+// row and each 4 consecutive dimension pairs of a head (thread th of nth takes
+// items th, th + nth, ...), the sum of the partials of CTAs c_first ..
+// c_first + nparts - 1 in that order, the rotation of query and key pairs and
+// the bf16 stores (q_out, or the cache slot ctx_b + i of the row's sequence).
+__device__ __noinline__ void reduce_tile(const Params &p, const int32_t *s_rseq, const int32_t *s_rpos,
+                                         const float *s_freq, int t, int c_first, int nparts, int th,
+                                         int nth) {
+  // Every field used below in a local: the stores through dst could alias
+  // the parameter block as far as the compiler knows, and it would reload them.
+  const int D = p.D, R = p.R, Hq = p.Hq, Hkv = p.Hkv, cap = p.cap, Ncols = p.Ncols;
+  const int max_pages = p.max_pages, page_size = p.page_size;
+  const int32_t *block_table = p.block_table;
+  __nv_bfloat16 *q_out = p.q_out, *k_cache = p.k_cache, *v_cache = p.v_cache;
+  const float *partials = p.partials;
+  const int half = D / 2;
+  const int hpt = kTileM / D;  // heads per tile
+  // Items: (row, 4 consecutive dimension pairs of one head); partials summed
+  // in CTA order c_first .. c_last, every load of an item issued first.
+  constexpr int kQuads = kTileM / 8;
+  const float *base = partials + static_cast<size_t>(c_first + t) * Ncols * kTileM;
+  const size_t slot = static_cast<size_t>(Ncols) * kTileM;
+  // Each thread takes kIB items at a time and issues the loads of every item
+  // and two parts before using any: the reduction is bound by L2 latency.
+  constexpr int kIB = 4;
+  const int nitems = R * kQuads;
+  for (int it0 = th; it0 < nitems; it0 += nth * kIB) {
+    int rr[kIB], d1[kIB], hl[kIB], jj[kIB], bb[kIB];
+    float y1[kIB][4], y2[kIB][4];
+#pragma unroll
+    for (int i = 0; i < kIB; ++i) {
+      const int it = it0 + i * nth;
+      rr[i] = it < nitems ? it / kQuads : 0;
+      const int pp = (it % kQuads) * 4;
+      hl[i] = pp / half;
+      jj[i] = pp % half;
+      d1[i] = hl[i] * D + jj[i];
+      bb[i] = it < nitems ? s_rseq[rr[i]] : -1;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) y1[i][e] = y2[i][e] = 0.f;
+    }
+    for (int s0 = 0; s0 < nparts; s0 += 2) {
+      float4 a[kIB][2], c[kIB][2];
+#pragma unroll
+      for (int i = 0; i < kIB; ++i)
+#pragma unroll
+        for (int s = 0; s < 2; ++s)
+          if (bb[i] >= 0 && s0 + s < nparts) {
+            const float *ps = base + (s0 + s) * slot + rr[i] * kTileM + d1[i];
+            a[i][s] = __ldcg(reinterpret_cast<const float4 *>(ps));
+            c[i][s] = __ldcg(reinterpret_cast<const float4 *>(ps + half));
+          }
+#pragma unroll
+      for (int i = 0; i < kIB; ++i)
+#pragma unroll
+        for (int s = 0; s < 2; ++s)
+          if (bb[i] >= 0 && s0 + s < nparts) {
+            y1[i][0] += a[i][s].x; y1[i][1] += a[i][s].y; y1[i][2] += a[i][s].z; y1[i][3] += a[i][s].w;
+            y2[i][0] += c[i][s].x; y2[i][1] += c[i][s].y; y2[i][2] += c[i][s].z; y2[i][3] += c[i][s].w;
+          }
+    }
+#pragma unroll
+    for (int i = 0; i < kIB; ++i) {
+      const int b = bb[i];
+      if (b < 0) continue;
+      const int r = rr[i], j0 = jj[i];
+      const int hg = t * hpt + hl[i];  // head among the Hq + 2 Hkv of the projection
+      const int pos = s_rpos[r];
+      if (hg < Hq + Hkv) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          float sn, cs;
+          rope_angle(pos, s_freq[j0 + e], &sn, &cs);
+          const float o1 = y1[i][e] * cs - y2[i][e] * sn, o2 = y2[i][e] * cs + y1[i][e] * sn;
+          y1[i][e] = o1;
+          y2[i][e] = o2;
+        }
+      }
+      __nv_bfloat16 *dst;
+      if (hg < Hq) {
+        dst = q_out + (static_cast<size_t>(r) * Hq + hg) * D;
+      } else {
+        const int hk = hg < Hq + Hkv ? hg - Hq : hg - Hq - Hkv;
+        __nv_bfloat16 *cache = hg < Hq + Hkv ? k_cache : v_cache;
+        if (block_table) {
+          const int pg = block_table[static_cast<int64_t>(b) * max_pages + pos / page_size];
+          dst = cache + ((static_cast<size_t>(pg) * Hkv + hk) * page_size + pos % page_size) * D;
+        } else {
+          dst = cache + ((static_cast<size_t>(b) * Hkv + hk) * cap + pos) * D;
+        }
+      }
+      // 4 bf16 = 8 bytes at each half (j0 a multiple of 4, rows 16-byte aligned).
+      *reinterpret_cast<uint2 *>(dst + j0) =
+          make_uint2(pack_bf16(y1[i][0], y1[i][1]), pack_bf16(y1[i][2], y1[i][3]));
+      *reinterpret_cast<uint2 *>(dst + j0 + half) =
+          make_uint2(pack_bf16(y2[i][0], y2[i][1]), pack_bf16(y2[i][2], y2[i][3]));
+    }
+  }
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -93,21 +237,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   int32_t *s_rpos = reinterpret_cast<int32_t *>(smem + L.rpos);
   uint64_t *bar_full = reinterpret_cast<uint64_t *>(smem + L.bars);
   uint64_t *bar_empty = bar_full + kMaxStages;
-  uint64_t *bar_acc = bar_empty + kMaxStages;
+  uint64_t *acc_full = bar_empty + kMaxStages;  // [2]
+  uint64_t *acc_empty = acc_full + 2;           // [2]
   uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + L.misc);
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L.misc + 8);
+  volatile int *s_last = reinterpret_cast<volatile int *>(smem + L.misc + 16);
+  float *s_freq = reinterpret_cast<float *>(smem + L.freq);
+  volatile int *s_fin = reinterpret_cast<volatile int *>(smem + L.misc + 32);  // last tile, c_first, nparts
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const int lane = tid & 31;
-  const int S = p.splits;
-  const int rank = static_cast<int>(blockIdx.x) % S;  // == %cluster_ctarank (clusters along x)
-  const int tile = static_cast<int>(blockIdx.x) / S;
-  const int kc0 = p.KC * rank / S, kc1 = p.KC * (rank + 1) / S;
-  const int nk = kc1 - kc0;
+  const int u0 = range_lo(p.units, p.num_ctas, blockIdx.x);
+  const int u1 = range_lo(p.units, p.num_ctas, blockIdx.x + 1);
 
   // ---- set-up that reads no input -----------------------------------------
-  if (tid == 0) *s_abort = 0;
+  if (tid == 0) { *s_abort = 0; s_fin[0] = -1; }
+  for (int j = tid; j < 64; j += kThreads) s_freq[j] = p.inv_freq[j];
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tm_w);
     tma_prefetch_desc(&tm_x0);
@@ -118,7 +264,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(&bar_full[s], 1);
         mbar_init(&bar_empty[s], 1);
       }
-      mbar_init(bar_acc, 1);
+      for (int b = 0; b < 2; ++b) {
+        mbar_init(&acc_full[b], 1);
+        mbar_init(&acc_empty[b], kEpiWarps);
+      }
       fence_mbar_init();
     }
     __syncwarp();
@@ -136,20 +285,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     int bad = 0;
     if (c < 0 || k < 0 || k > p.max_k || q0 < 0 || q1 > p.R || q1 - q0 != k + 1) bad = SPADE_DEV_BAD_INDEX;
     else if (static_cast<int64_t>(c) + k + 1 > p.cap) bad = SPADE_DEV_CAPACITY;
-    if (bad) {
-      if (blockIdx.x == 0) atomicOr(p.status, bad);
-      continue;
-    }
-    if (p.block_table) {
+    if (!bad && p.block_table) {
       // Every page the block writes must exist.
       for (int i = 0; i <= k; ++i) {
         const int pg = p.block_table[static_cast<int64_t>(b) * p.max_pages + (c + i) / p.page_size];
         if (pg < 0 || pg >= p.num_pages) bad = SPADE_DEV_BAD_INDEX;
       }
-      if (bad) {
-        if (blockIdx.x == 0) atomicOr(p.status, bad);
-        continue;
-      }
+    }
+    if (bad) {
+      if (blockIdx.x == 0) atomicOr(p.status, bad);
+      continue;
     }
     for (int i = 0; i <= k; ++i) {
       s_rseq[q0 + i] = b;
@@ -168,20 +313,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ============================ producer: TMA ============================
     if (lane == 0) {
       const uint64_t pol_w = l2_policy_evict_first();  // W streams once
-      const uint64_t pol_x = l2_policy_evict_last();   // x is re-read by every tile
+      const uint64_t pol_x = l2_policy_evict_last();   // x is re-read for every unit
       const uint32_t bytes = kWBytes + p.Ncols * 128;
       bool expired = false;
       int issued = 0;
-      for (int i = 0; i < nk; ++i) {
+      for (int u = u0, i = 0; u < u1; ++u, ++i) {
         const int st = i % p.stages;
         const uint32_t ph = (i / p.stages) & 1;
         if (!mbar_wait(&bar_empty[st], ph ^ 1, s_abort)) expired = true;
         if (*s_abort) break;
         issued = i + 1;
         uint8_t *stage = smem + L.ring + st * L.stage_bytes;
-        const int kx = (kc0 + i) * kKChunk;
+        const int t = u / p.KC, kx = (u - t * p.KC) * kKChunk;
         mbar_arrive_expect_tx(&bar_full[st], bytes);
-        tma_load_2d(stage, &tm_w, kx, tile * kTileM, &bar_full[st], pol_w);
+        tma_load_2d(stage, &tm_w, kx, t * kTileM, &bar_full[st], pol_w);
         tma_load_2d(stage + kWBytes, &tm_x0, kx, 0, &bar_full[st], pol_x);
         if (n1) tma_load_2d(stage + kWBytes + n0 * 128, &tm_x1, kx, n0, &bar_full[st], pol_x);
       }
@@ -198,129 +343,89 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t idesc0 = idesc_bf16_f32(kTileM, n0);
       const uint32_t idesc1 = idesc_bf16_f32(kTileM, n1 ? n1 : 16);
       bool expired = false;
-      for (int i = 0; i < nk; ++i) {
-        const int st = i % p.stages;
-        const uint32_t ph = (i / p.stages) & 1;
-        if (!mbar_wait(&bar_full[st], ph, s_abort)) expired = true;
+      int i = 0, seg = 0;
+      for (int u = u0; u < u1; ++seg) {
+        const int t = u / p.KC;
+        const int se = min(u1, (t + 1) * p.KC);
+        const int buf = seg % p.nbuf, use = seg / p.nbuf;
+        // The buffer's previous segment has been drained by the epilogue warps.
+        if (use > 0 && !mbar_wait(&acc_empty[buf], (use - 1) & 1, s_abort)) expired = true;
         tc_fence_after();
-        if (!*s_abort) {
-          const uint32_t a = smem_base + L.ring + st * L.stage_bytes;
-          const uint32_t b = a + kWBytes;
+        const uint32_t acc_addr = tmem + static_cast<uint32_t>(buf) * p.buf_cols;
+        for (const int us = u; u < se; ++u, ++i) {
+          const int st = i % p.stages;
+          const uint32_t ph = (i / p.stages) & 1;
+          if (!mbar_wait(&bar_full[st], ph, s_abort)) expired = true;
+          tc_fence_after();
+          if (!*s_abort) {
+            const uint32_t a = smem_base + L.ring + st * L.stage_bytes;
+            const uint32_t b = a + kWBytes;
 #pragma unroll
-          for (int kk = 0; kk < kKChunk / 16; ++kk) {
-            const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
-            tc_mma_f16(tmem, smem_desc_sw128(a + kk * 32), smem_desc_sw128(b + kk * 32), idesc0, acc);
-            if (n1)
-              tc_mma_f16(tmem + 256, smem_desc_sw128(a + kk * 32), smem_desc_sw128(b + n0 * 128 + kk * 32),
-                         idesc1, acc);
+            for (int kk = 0; kk < kKChunk / 16; ++kk) {
+              const uint32_t acc = (u > us || kk > 0) ? 1u : 0u;
+              tc_mma_f16(acc_addr, smem_desc_sw128(a + kk * 32), smem_desc_sw128(b + kk * 32), idesc0, acc);
+              if (n1)
+                tc_mma_f16(acc_addr + 256, smem_desc_sw128(a + kk * 32),
+                           smem_desc_sw128(b + n0 * 128 + kk * 32), idesc1, acc);
+            }
           }
+          tc_commit(&bar_empty[st]);
         }
-        tc_commit(&bar_empty[st]);
+        tc_commit(&acc_full[buf]);
       }
-      tc_commit(bar_acc);  // arrives once every MMA above is done (at once if none)
       if (expired) atomicOr(p.status, SPADE_DEV_TIMEOUT);
     }
-  }
-
-
-  // ======================= epilogue (every thread) =========================
-  // Rounds of up to 256 accumulator columns: warps 2-5 move their tensor-memory
-  // lane quadrant to shared memory (the ring is free once the MMAs are done),
-  // the cluster barrier makes every CTA's partial visible, then the cluster's
-  // CTAs share the round's (row, dimension pair) items: each sums the partials
-  // of the split-K CTAs from distributed shared memory, rotates query and key
-  // pairs and stores bf16; a second barrier keeps every CTA's partial alive
-  // until all have read it.
-  float *red = reinterpret_cast<float *>(smem + L.ring);  // [kRedCols][128]
-  uint32_t red_rank[kMaxSplits];
-#pragma unroll
-  for (int s = 0; s < kMaxSplits; ++s) red_rank[s] = s < S ? cluster_map(red, s) : 0u;
-  const int hpt = kTileM / p.D;  // heads per tile
-  const int half = p.D / 2;
-  bool acc_ready = false;
-  for (int c0 = 0; c0 < p.Ncols; c0 += kRedCols) {
-    const int nc = min(kRedCols, p.Ncols - c0);
-    if (warp >= 2) {
-      const int q4 = warp & 3;  // tensor-memory lane quadrant this warp may access
-      if (!acc_ready) {
-        if (!mbar_wait(bar_acc, 0, s_abort)) atomicOr(p.status, SPADE_DEV_TIMEOUT);
-        tc_fence_after();
-        acc_ready = true;
-      }
-      const uint32_t tl = tmem + (static_cast<uint32_t>(q4 * 32) << 16) + static_cast<uint32_t>(c0);
-      for (int c = 0; c < nc; c += 8) {
+  } else {
+    // ===================== epilogue warps: drain, publish, reduce ==========
+    const int et = tid - 64;         // 0..127
+    const int q4 = warp & 3;         // tensor-memory lane quadrant this warp may access
+    bool expired = false;
+    int seg = 0;
+    for (int u = u0; u < u1; ++seg) {
+      const int t = u / p.KC;
+      const int se = min(u1, (t + 1) * p.KC);
+      const int buf = seg % p.nbuf, use = seg / p.nbuf;
+      if (!mbar_wait(&acc_full[buf], use & 1, s_abort)) expired = true;
+      tc_fence_after();
+      // Accumulator -> this CTA's slot [Ncols][128] of the tile's partials.
+      float *part = p.partials + static_cast<size_t>(blockIdx.x + t) * p.Ncols * kTileM;
+      const uint32_t tl = tmem + (static_cast<uint32_t>(q4 * 32) << 16) + static_cast<uint32_t>(buf) * p.buf_cols;
+      for (int c = 0; c < p.Ncols; c += 8) {
         uint32_t v[8];
         tmem_ld8(tl + c, v);
         tmem_wait_ld();
 #pragma unroll
-        for (int e = 0; e < 8; ++e) red[(c + e) * kTileM + q4 * 32 + lane] = __uint_as_float(v[e]);
+        for (int e = 0; e < 8; ++e) __stcg(part + (c + e) * kTileM + q4 * 32 + lane, __uint_as_float(v[e]));
       }
-    }
-    __syncwarp();
-    cluster_sync();
-    // Items are (row, 4 consecutive dimension pairs of one head): two float4
-    // loads per split CTA, all issued before any is used.
-    constexpr int kQuads = kTileM / 8;  // quads of pairs per accumulator column
-    const int items = nc * kQuads;
-    const int i0 = items * rank / S, i1 = items * (rank + 1) / S;
-    for (int it = i0 + tid; it < i1; it += kThreads) {
-      const int col = it / kQuads, qd = it % kQuads;
-      const int r = c0 + col;
-      if (r >= p.R) continue;
-      const int b = s_rseq[r];
-      if (b < 0) continue;
-      const int pp = qd * 4;  // first pair of the quad
-      const int hloc = pp / half, j0 = pp % half;
-      const int d1 = hloc * p.D + j0;
-      const uint32_t off1 = static_cast<uint32_t>((col * kTileM + d1) * 4);
-      const uint32_t off2 = off1 + static_cast<uint32_t>(half * 4);
-      float4 a[kMaxSplits], c[kMaxSplits];
-#pragma unroll
-      for (int s = 0; s < kMaxSplits; ++s) {
-        if (s < S) {
-          a[s] = ld_dsmem_f32x4(red_rank[s] + off1);
-          c[s] = ld_dsmem_f32x4(red_rank[s] + off2);
-        }
-      }
-      float y1[4] = {0.f, 0.f, 0.f, 0.f}, y2[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int s = 0; s < kMaxSplits; ++s) {
-        if (s < S) {
-          y1[0] += a[s].x; y1[1] += a[s].y; y1[2] += a[s].z; y1[3] += a[s].w;
-          y2[0] += c[s].x; y2[1] += c[s].y; y2[2] += c[s].z; y2[3] += c[s].w;
-        }
-      }
-      const int hg = tile * hpt + hloc;  // head among the Hq + 2 Hkv of the projection
-      const int pos = s_rpos[r];
-      if (hg < p.Hq + p.Hkv) {
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          float sn, cs;
-          sincosf(static_cast<float>(pos) * p.inv_freq[j0 + e], &sn, &cs);
-          const float o1 = y1[e] * cs - y2[e] * sn, o2 = y2[e] * cs + y1[e] * sn;
-          y1[e] = o1;
-          y2[e] = o2;
-        }
-      }
-      __nv_bfloat16 *dst;
-      if (hg < p.Hq) {
-        dst = p.q_out + (static_cast<size_t>(r) * p.Hq + hg) * p.D;
-      } else {
-        const int hk = hg < p.Hq + p.Hkv ? hg - p.Hq : hg - p.Hq - p.Hkv;
-        __nv_bfloat16 *cache = hg < p.Hq + p.Hkv ? p.k_cache : p.v_cache;
-        if (p.block_table) {
-          const int pg = p.block_table[static_cast<int64_t>(b) * p.max_pages + pos / p.page_size];
-          dst = cache + ((static_cast<size_t>(pg) * p.Hkv + hk) * p.page_size + pos % p.page_size) * p.D;
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[buf]);
+      // Publish; the CTA that completes the tile reduces it.
+      const int c_first = unit_owner(p.units, p.num_ctas, t * p.KC);
+      const int c_last = unit_owner(p.units, p.num_ctas, (t + 1) * p.KC - 1);
+      const int nparts = c_last - c_first + 1;
+      epi_bar();
+      if (et == 0) *s_last = nparts == 1 ? 1 : arrive_tile(&p.counters[t], nparts);
+      epi_bar();
+      if (*s_last) {
+        if (se == u1) {
+          // The CTA's last tile: reduced below by every thread of the CTA.
+          if (et == 0) { s_fin[0] = t; s_fin[1] = c_first; s_fin[2] = nparts; }
         } else {
-          dst = cache + ((static_cast<size_t>(b) * p.Hkv + hk) * p.cap + pos) * p.D;
+          reduce_tile(p, s_rseq, s_rpos, s_freq, t, c_first, nparts, et, kEpiThreads);
+          if (et == 0 && nparts > 1) p.counters[t] = 0;  // every part has arrived: reset for the next call
         }
       }
-      // 4 bf16 = 8 bytes at each half (j0 is a multiple of 4, rows 16-byte aligned).
-      *reinterpret_cast<uint2 *>(dst + j0) = make_uint2(pack_bf16(y1[0], y1[1]), pack_bf16(y1[2], y1[3]));
-      *reinterpret_cast<uint2 *>(dst + j0 + half) = make_uint2(pack_bf16(y2[0], y2[1]), pack_bf16(y2[2], y2[3]));
+      u = se;
     }
-    __syncwarp();
-    cluster_sync();
+    if (expired) atomicOr(p.status, SPADE_DEV_TIMEOUT);
+  }
+  // The CTA's last tile, if this CTA completed it, with every thread.
+  __syncwarp();
+  __syncthreads();
+  if (s_fin[0] >= 0) {
+    reduce_tile(p, s_rseq, s_rpos, s_freq, s_fin[0], s_fin[1], s_fin[2], tid, kThreads);
+    if (tid == 0 && s_fin[2] > 1) p.counters[s_fin[0]] = 0;  // every part has arrived: reset for the next call
   }
   tc_fence_before();
   __syncthreads();
@@ -335,54 +440,33 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 namespace spade {
 namespace qkv {
-
-// Clusters of `splits` CTAs (with `smem` bytes each) that the device can hold
-// at once; 0 if the query fails.
-static int max_active_clusters(int splits, int smem) {
-  static int cache[kMaxSplits + 1][2] = {};
-  static int cached_smem[kMaxSplits + 1] = {};
-  if (cached_smem[splits] == smem && cache[splits][0]) return cache[splits][1];
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(splits);
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = smem;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = splits;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, qkv_rope_kernel, &cfg) != cudaSuccess) {
-    cudaGetLastError();
-    n = 0;
-  }
-  cache[splits][0] = 1;
-  cache[splits][1] = n;
-  cached_smem[splits] = smem;
-  return n;
+struct Paging {
+  const int32_t *block_table;
+  int page_size, max_pages, num_pages;
+};
+static size_t workspace_bytes_for(int R, int tiles, int sms) {
+  const size_t ncols = static_cast<size_t>((R + 15) / 16 * 16);
+  return round_up(static_cast<size_t>(tiles) * 4, 256) + static_cast<size_t>(sms + tiles) * ncols * kTileM * 4;
 }
-
 }  // namespace qkv
 }  // namespace spade
 
 using namespace spade;
 
-namespace spade {
-namespace qkv {
-struct Paging {
-  const int32_t *block_table;
-  int page_size, max_pages, num_pages;
-};
-}  // namespace qkv
-}  // namespace spade
+extern "C" size_t spade_qkv_workspace_size(int32_t R, int32_t Hq, int32_t Hkv, int32_t D) {
+  if (R <= 0 || R > qkv::kMaxR || Hq <= 0 || Hkv <= 0 || (D != 64 && D != 128) || (Hq + 2 * Hkv) * D % qkv::kTileM)
+    return 0;
+  int sms = 0;
+  if (device_info(&sms, nullptr) != SPADE_OK) return 0;
+  return qkv::workspace_bytes_for(R, (Hq + 2 * Hkv) * D / qkv::kTileM, sms);
+}
 
 static spade_status qkv_rope_impl(const void *x, const void *w_qkv, const int32_t *ctx_lens,
                                   const int32_t *n_draft, const int32_t *cu_q, void *q_out, void *k_cache,
                                   void *v_cache, int32_t B, int32_t R, int32_t H, int32_t Hq, int32_t Hkv,
-                                  int32_t D, int32_t cap, int32_t max_k, float rope_theta, int32_t *status,
-                                  spade_stream_t stream, const qkv::Paging *pg) {
+                                  int32_t D, int32_t cap, int32_t max_k, float rope_theta, void *workspace,
+                                  size_t workspace_bytes, int32_t *status, spade_stream_t stream,
+                                  const qkv::Paging *pg) {
   using namespace qkv;
   if (!x || !w_qkv || !ctx_lens || !n_draft || !cu_q || !q_out || !k_cache || !v_cache || !status)
     return fail(SPADE_ERR_INVALID_ARG, "spade_verify_qkv_rope: null pointer argument");
@@ -403,6 +487,11 @@ static spade_status qkv_rope_impl(const void *x, const void *w_qkv, const int32_
   int sms = 0;
   spade_status st = device_info(&sms, nullptr);
   if (st != SPADE_OK) return st;
+  const int tiles = (Hq + 2 * Hkv) * D / kTileM;
+  const size_t need = workspace_bytes_for(R, tiles, sms);
+  if (!workspace || workspace_bytes < need || !aligned(workspace, 256))
+    return fail(SPADE_ERR_WORKSPACE, "qkv workspace needs %zu bytes, 256-byte aligned (got %zu)", need,
+                workspace_bytes);
 
   Params p{};
   p.ctx_lens = ctx_lens;
@@ -412,44 +501,35 @@ static spade_status qkv_rope_impl(const void *x, const void *w_qkv, const int32_
   p.k_cache = static_cast<__nv_bfloat16 *>(k_cache);
   p.v_cache = static_cast<__nv_bfloat16 *>(v_cache);
   p.status = status;
+  p.counters = static_cast<int32_t *>(workspace);
+  p.partials = reinterpret_cast<float *>(static_cast<uint8_t *>(workspace) + round_up(static_cast<size_t>(tiles) * 4, 256));
   p.B = B; p.R = R; p.H = H; p.Hq = Hq; p.Hkv = Hkv; p.D = D; p.cap = cap; p.max_k = max_k;
   p.block_table = pg ? pg->block_table : nullptr;
   p.page_size = pg ? pg->page_size : 0;
   p.max_pages = pg ? pg->max_pages : 0;
   p.num_pages = pg ? pg->num_pages : 0;
+  p.tiles = tiles;
   p.KC = (H + kKChunk - 1) / kKChunk;
+  p.units = tiles * p.KC;
+  p.num_ctas = p.units < sms ? p.units : sms;
   p.Ncols = (R + 15) / 16 * 16;
-  p.tmem_cols = 32;
-  while (p.tmem_cols < static_cast<uint32_t>(p.Ncols)) p.tmem_cols *= 2;
+  p.buf_cols = 32;
+  while (p.buf_cols < static_cast<uint32_t>(p.Ncols)) p.buf_cols *= 2;
+  p.nbuf = p.buf_cols * 2 <= 512 ? 2 : 1;
+  p.tmem_cols = p.buf_cols * p.nbuf;
   for (int j = 0; j < D / 2; ++j) p.inv_freq[j] = static_cast<float>(pow(static_cast<double>(rope_theta), -2.0 * j / D));
-  const int tiles = (Hq + 2 * Hkv) * D / kTileM;
-  // Ring: as many stages as fit, at least two, holding at least one round of
-  // the reduction buffer (256 columns x 128 rows of fp32) once the MMAs are done.
   const int stage = kWBytes + p.Ncols * 128;
-  const int fixed = layout(p.Ncols, 0).total;
-  p.stages = (kSmemBudget - fixed) / stage;
+  p.stages = (kSmemBudget - layout(p.Ncols, 0).total) / stage;
   if (p.stages > kMaxStages) p.stages = kMaxStages;
-  const int red = (p.Ncols < kRedCols ? p.Ncols : kRedCols) * kTileM * 4;
-  if (p.stages < 2 || p.stages * stage < red)
-    return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
+  if (p.stages < 2) return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
   const int smem = layout(p.Ncols, p.stages).total;
   static bool configured = false;
   if (!configured) {
     // The plan above never exceeds kSmemBudget (alignment slack included).
-    cudaError_t e = cudaFuncSetAttribute(qkv_rope_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         kSmemBudget);
+    cudaError_t e = cudaFuncSetAttribute(qkv_rope_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(qkv_rope)");
     configured = true;
   }
-  // Split K over a cluster of CTAs per tile so the grid fills the SMs, as
-  // long as every cluster of the grid fits on the device at once.
-  int S = sms / tiles;
-  if (S > kMaxSplits) S = kMaxSplits;
-  if (S > p.KC) S = p.KC;
-  if (S < 1) S = 1;
-  while (S > 1 && max_active_clusters(S, smem) < tiles) --S;
-  p.splits = S;
-
   CUtensorMap tw, tx0, tx1;
   const int n0 = p.Ncols > 256 ? 256 : p.Ncols;
   const int n1 = p.Ncols - n0;
@@ -458,21 +538,16 @@ static spade_status qkv_rope_impl(const void *x, const void *w_qkv, const int32_
       !encode_tmap_bf16_sw128(&tx0, x, H, R, static_cast<uint64_t>(H) * 2, kKChunk, n0) ||
       !encode_tmap_bf16_sw128(&tx1, x, H, R, static_cast<uint64_t>(H) * 2, kKChunk, n1 ? n1 : 16))
     return SPADE_ERR_CUDA;
-
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(tiles * S);
+  cfg.gridDim = dim3(p.num_ctas);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = reinterpret_cast<cudaStream_t>(stream);
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = S;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 2;
+  cfg.numAttrs = 1;
   const cudaError_t e = cudaLaunchKernelEx(&cfg, qkv_rope_kernel, p, tw, tx0, tx1);
   if (e != cudaSuccess) return cuda_fail(e, "qkv_rope launch");
   return SPADE_OK;
@@ -482,10 +557,10 @@ extern "C" spade_status spade_verify_qkv_rope(const void *x, const void *w_qkv, 
                                               const int32_t *n_draft, const int32_t *cu_q, void *q_out,
                                               void *k_cache, void *v_cache, int32_t B, int32_t R,
                                               int32_t H, int32_t Hq, int32_t Hkv, int32_t D, int32_t cap,
-                                              int32_t max_k, float rope_theta, int32_t *status,
-                                              spade_stream_t stream) {
+                                              int32_t max_k, float rope_theta, void *workspace,
+                                              size_t workspace_bytes, int32_t *status, spade_stream_t stream) {
   return qkv_rope_impl(x, w_qkv, ctx_lens, n_draft, cu_q, q_out, k_cache, v_cache, B, R, H, Hq, Hkv, D, cap,
-                       max_k, rope_theta, status, stream, nullptr);
+                       max_k, rope_theta, workspace, workspace_bytes, status, stream, nullptr);
 }
 
 extern "C" spade_status spade_verify_qkv_rope_paged(const void *x, const void *w_qkv,
@@ -494,7 +569,8 @@ extern "C" spade_status spade_verify_qkv_rope_paged(const void *x, const void *w
                                                     void *k_pool, void *v_pool, int32_t B, int32_t R,
                                                     int32_t H, int32_t Hq, int32_t Hkv, int32_t D,
                                                     int32_t page_size, int32_t num_pages, int32_t max_pages,
-                                                    int32_t max_k, float rope_theta, int32_t *status,
+                                                    int32_t max_k, float rope_theta, void *workspace,
+                                                    size_t workspace_bytes, int32_t *status,
                                                     spade_stream_t stream) {
   if (!block_table) return fail(SPADE_ERR_INVALID_ARG, "spade_verify_qkv_rope_paged: null block_table");
   if (page_size <= 0 || num_pages <= 0 || max_pages <= 0)
@@ -503,5 +579,5 @@ extern "C" spade_status spade_verify_qkv_rope_paged(const void *x, const void *w
     return fail(SPADE_ERR_CAPACITY, "max_pages * page_size exceeds 2^31");
   const qkv::Paging pg{block_table, page_size, max_pages, num_pages};
   return qkv_rope_impl(x, w_qkv, ctx_lens, n_draft, cu_q, q_out, k_pool, v_pool, B, R, H, Hq, Hkv, D,
-                       max_pages * page_size, max_k, rope_theta, status, stream, &pg);
+                       max_pages * page_size, max_k, rope_theta, workspace, workspace_bytes, status, stream, &pg);
 }

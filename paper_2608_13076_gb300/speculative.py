@@ -29,8 +29,8 @@ from dataclasses import dataclass
 
 import torch
 
-from . import (accept_workspace, attn_workspace, spade_verify_accept_commit, spade_verify_attention,
-               spade_verify_qkv_rope, status_tensor)
+from . import (accept_workspace, attn_workspace, qkv_workspace, spade_verify_accept_commit,
+               spade_verify_attention, spade_verify_qkv_rope, status_tensor)
 
 GREEDY = 0
 STOCHASTIC = 1
@@ -80,7 +80,9 @@ class ToyVerifier:
         x = self.emb[tokens].contiguous()
         q = torch.empty((x.shape[0], self.cfg.Hq, self.cfg.D), dtype=torch.bfloat16, device=self.device)
         spade_verify_qkv_rope(x, self.w_qkv, ctx, kd, cu_q, q, self.k_cache, self.v_cache, Hq=self.cfg.Hq,
-                              Hkv=self.cfg.Hkv, rope_theta=self.cfg.rope_theta, max_k=max_k, status=self.status)
+                              Hkv=self.cfg.Hkv, rope_theta=self.cfg.rope_theta, max_k=max_k,
+                              workspace=qkv_workspace(x.shape[0], self.cfg.Hq, self.cfg.Hkv, self.cfg.D,
+                                                      device=self.device), status=self.status)
 
     def verify(self, tokens, kd, cu_q, drafts, draft_probs, uniforms, mode, max_k):
         """One verify call over the blocks (row cu_q[b] + i holds token i of sequence b's
@@ -91,7 +93,8 @@ class ToyVerifier:
         x = self.emb[tokens].contiguous()
         q = torch.empty((R, c.Hq, c.D), dtype=torch.bfloat16, device=self.device)
         spade_verify_qkv_rope(x, self.w_qkv, self.ctx, kd, cu_q, q, self.k_cache, self.v_cache, Hq=c.Hq,
-                              Hkv=c.Hkv, rope_theta=c.rope_theta, max_k=max_k, status=self.status)
+                              Hkv=c.Hkv, rope_theta=c.rope_theta, max_k=max_k,
+                              workspace=qkv_workspace(R, c.Hq, c.Hkv, c.D, device=self.device), status=self.status)
         out = torch.empty_like(q)
         ws = attn_workspace(self.B, c.Hq, c.Hkv, c.D, self.cap, max_k, device=self.device)
         spade_verify_attention(q, self.k_cache, self.v_cache, self.ctx, kd, cu_q, out, None, max_k=max_k,

@@ -208,7 +208,9 @@ def gpu_qkv_rope(wl, x, w, q_out=None, status=None):
         status = spade.status_tensor(dev)
     spade.spade_verify_qkv_rope(x, w, wl["ctx_lens"], wl["n_draft"], wl["cu_q"], q_out, wl["k_cache"],
                                 wl["v_cache"], Hq=wl["Hq"], Hkv=wl["Hkv"], rope_theta=wl["spec"].rope_theta,
-                                max_k=int(wl["n_draft"].max()), status=status)
+                                max_k=int(wl["n_draft"].max()),
+                                workspace=spade.qkv_workspace(wl["R"], wl["Hq"], wl["Hkv"], wl["D"], device=dev),
+                                status=status)
     return q_out, status
 
 

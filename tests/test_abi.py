@@ -113,10 +113,10 @@ def test_stats_layout_rejects_bad_arguments(lib):
 def test_qkv_rope_validation_before_device_work(lib):
     p = ctypes.c_void_p(16)
     f = lib.spade_verify_qkv_rope
-    assert f(*([None] * 8), 1, 5, 512, 8, 8, 128, 300, 4, ctypes.c_float(1e4), None, None) == 1  # null
-    assert f(*([p] * 8), 1, 5, 512, 8, 8, 96, 300, 4, ctypes.c_float(1e4), p, None) == 2          # D = 96
-    assert f(*([p] * 8), 1, 5, 512, 6, 4, 128, 300, 4, ctypes.c_float(1e4), p, None) == 2         # Hq % Hkv
-    assert f(*([p] * 8), 1, 5, 500, 8, 8, 128, 300, 4, ctypes.c_float(1e4), p, None) == 2         # H % 8
-    assert f(*([p] * 8), 1, 5, 512, 3, 3, 64, 300, 4, ctypes.c_float(1e4), p, None) == 2          # (Hq+2Hkv)D % 128
-    assert f(*([p] * 8), 1, 600, 512, 8, 8, 128, 900, 4, ctypes.c_float(1e4), p, None) == 2       # R > 512
-    assert f(*([p] * 8), 1, 5, 512, 8, 8, 128, 300, 4, ctypes.c_float(0.5), p, None) == 1         # theta <= 1
+    assert f(*([None] * 8), 1, 5, 512, 8, 8, 128, 300, 4, ctypes.c_float(1e4), None, 0, None, None) == 1  # null
+    assert f(*([p] * 8), 1, 5, 512, 8, 8, 96, 300, 4, ctypes.c_float(1e4), p, 1 << 20, p, None) == 2          # D = 96
+    assert f(*([p] * 8), 1, 5, 512, 6, 4, 128, 300, 4, ctypes.c_float(1e4), p, 1 << 20, p, None) == 2         # Hq % Hkv
+    assert f(*([p] * 8), 1, 5, 500, 8, 8, 128, 300, 4, ctypes.c_float(1e4), p, 1 << 20, p, None) == 2         # H % 8
+    assert f(*([p] * 8), 1, 5, 512, 3, 3, 64, 300, 4, ctypes.c_float(1e4), p, 1 << 20, p, None) == 2          # (Hq+2Hkv)D % 128
+    assert f(*([p] * 8), 1, 600, 512, 8, 8, 128, 900, 4, ctypes.c_float(1e4), p, 1 << 20, p, None) == 2       # R > 512
+    assert f(*([p] * 8), 1, 5, 512, 8, 8, 128, 300, 4, ctypes.c_float(0.5), p, 1 << 20, p, None) == 1         # theta <= 1

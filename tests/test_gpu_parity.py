@@ -571,7 +571,9 @@ def test_paged_qkv_rope(dev):
     st = spade.status_tensor(dev)
     spade.spade_verify_qkv_rope_paged(x, w, pg["block_table"], wl["ctx_lens"], wl["n_draft"], wl["cu_q"], q,
                                       pg["k_pool"], pg["v_pool"], Hq=wl["Hq"], rope_theta=spec.rope_theta,
-                                      max_k=int(wl["n_draft"].max()), status=st)
+                                      max_k=int(wl["n_draft"].max()),
+                                      workspace=spade.qkv_workspace(wl["R"], wl["Hq"], wl["Hkv"], wl["D"], device=dev),
+                                      status=st)
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     ctx, kd, cu = (parity.to_np(wl[k]) for k in ("ctx_lens", "n_draft", "cu_q"))
