@@ -164,13 +164,36 @@ def inverse_cdf(r, Z, u):
     return x, margin
 
 
+def nucleus(p, top_p):
+    """Top-p truncation of a distribution (sampling "for diversity", Sec. III-A, left open
+    by the paper): S = {x : p(x) >= tau}, tau the probability of the token at which the
+    cumulative mass in descending order first reaches top_p (tokens tied with it included);
+    returns (p on S renormalised, mass margin, log gap): the distance of top_p to the nearer
+    end of the boundary token's step of the cumulative mass, and ln p of the boundary token
+    minus ln p of the next one (small values: a boundary that rounding could move)."""
+    p = _f64(p)
+    if top_p >= 1.0:
+        return p, np.inf, np.inf
+    order = np.argsort(-p, kind="stable")
+    c = np.cumsum(p[order])
+    j = int(np.nonzero(c >= top_p)[0][0]) if np.any(c >= top_p) else len(p) - 1
+    tau = p[order[j]]
+    keep = p >= tau
+    pt = np.where(keep, p, 0.0)
+    pt = pt / pt.sum()
+    below = c[j - 1] if j > 0 else 0.0
+    nxt = p[order[j + 1]] if j + 1 < len(p) else 0.0
+    gap = np.log(tau) - np.log(nxt) if nxt > 0 else np.inf
+    return pt, min(c[j] - top_p, top_p - below), gap
+
+
 def _top2_margin(l):
     top = np.partition(l, -2)[-2:] if l.shape[0] > 1 else np.array([-np.inf, l[0]])
     return float(top[1] - top[0])
 
 
 def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
-                  margin=1e-3, temperature=None):
+                  margin=1e-3, temperature=None, top_p=None):
     """Accept/reject of every sequence, given its verifier logits.
 
     logits [R, V] (rows as in ``verify_attention``); draft_tokens [R-B] with
@@ -188,7 +211,10 @@ def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_dra
 
     ``temperature`` [B] (optional): the verifier samples from p = softmax(l / T_b)
     (the paper mentions sampling for diversity, Sec. III-A, without fixing it);
-    greedy decisions, which take the argmax, are unaffected.
+    greedy decisions, which take the argmax, are unaffected.  ``top_p`` [B] (optional): p is
+    then truncated to its nucleus (``nucleus``) for stochastic sequences; a nucleus boundary
+    within the margin (1e-3 of mass, 1e-4 of log probability) at a deciding row flags the
+    sequence's decision.
     """
     B = len(n_draft)
     acc = np.zeros(B, dtype=np.int64)
@@ -202,6 +228,14 @@ def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_dra
         d0 = r0 - b
         stochastic = int(mode[b]) == STOCHASTIC
         t_b = 1.0 if temperature is None else float(temperature[b])
+        tp_b = 1.0 if top_p is None else float(top_p[b])
+
+        def dist(l_row):
+            pn, mass_margin, log_gap = nucleus(softmax(l_row / t_b), tp_b)
+            if mass_margin < margin or log_gap < 0.1 * margin:
+                flag_dec[b] = True
+            return pn
+
         a = 0
         for i in range(k):
             l = _f64(logits[r0 + i])
@@ -211,7 +245,7 @@ def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_dra
                 if _top2_margin(l) < margin:
                     flag_dec[b] = True
             else:
-                p = softmax(l / t_b)
+                p = dist(l)
                 qd = float(draft_probs[d0 + i][d])
                 u = float(uniforms[r0 + i])
                 if qd > 0.0:
@@ -231,7 +265,7 @@ def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_dra
             if _top2_margin(lr) < margin:
                 flag_dec[b] = True
         else:
-            p = softmax(lr / t_b)
+            p = dist(lr)
             if a < k:
                 r, Z, fb = residual_distribution(p, draft_probs[d0 + a])
             else:

@@ -550,6 +550,53 @@ def check_temperature_output_law(o, n=40000, seed=14):
     assert pv > 1e-3, pv
 
 
+# ----------------------------------------------------------------------------
+# Top-p truncation of the verifier's distribution
+# ----------------------------------------------------------------------------
+def check_top_p_worked_example(o):
+    g = _golden()["top_p"]
+    P = np.asarray(g["p"])
+    l = np.log(P)
+    pt, _, _ = o.nucleus(P, g["top_p"])
+    np.testing.assert_allclose(pt, g["nucleus"], rtol=0, atol=1e-15)
+    ex = g["exact_reach"]
+    np.testing.assert_allclose(o.nucleus(P, ex["top_p"])[0], ex["nucleus"], rtol=0, atol=1e-15, err_msg=ex["why"])
+    tp = [g["top_p"]]
+    for ex in g["accept"]:
+        res = o.verify_accept(np.stack([l, l]), [ex["draft"]], np.asarray(ex["q"])[None], [ex["u"], 0.5], [1],
+                              [0, 2], [1], top_p=tp)
+        assert res["accepted_len"][0] == ex["accepted"], ex["why"]
+    rq = np.asarray(g["residual"]["q"])[None]
+    for u, x in g["residual"]["cases"]:
+        res = o.verify_accept(np.stack([l, l]), [g["residual"]["draft"]], rq, [0.0, u], [1], [0, 2], [1], top_p=tp)
+        assert res["accepted_len"][0] == 0 and res["next_token"][0] == x, (u, x)
+    for u, x in g["bonus"]:
+        res = o.verify_accept(l[None], [], np.zeros((0, 4)), [u], [1], [0, 1], [0], top_p=tp)
+        assert res["next_token"][0] == x, (u, x)
+    # top_p = 1 is no truncation.
+    np.testing.assert_array_equal(o.nucleus(P, 1.0)[0], P)
+
+
+def check_top_p_output_law(o, n=40000, seed=15):
+    """Rejection sampling with a nucleus reproduces the truncated, renormalised p."""
+    rng = np.random.default_rng(seed)
+    V, k, tp = 8, 1, 0.8
+    L = rng.standard_normal((k + 1, V)) * 1.5
+    P0 = np.exp(L[0]) / np.exp(L[0]).sum()
+    Pt, _, _ = o.nucleus(P0, tp)
+    Q = rng.dirichlet(np.ones(V), size=k)
+    drafts = rng.choice(V, size=n, p=Q[0])
+    u = rng.random(n * (k + 1))
+    res = o.verify_accept(np.tile(L, (n, 1)), drafts, np.tile(Q, (n, 1)), u, np.ones(n, int),
+                          np.arange(n + 1) * (k + 1), np.full(n, k), top_p=np.full(n, tp))
+    first = np.where(res["accepted_len"] >= 1, drafts, res["next_token"])
+    counts = np.bincount(first, minlength=V)
+    assert (counts[Pt == 0] == 0).all()
+    keep = Pt > 0
+    _, pv = stats.chisquare(counts[keep], Pt[keep] * n)
+    assert pv > 1e-3, pv
+
+
 ALL_CHECKS = [
     check_attention_worked_examples, check_attention_vs_sdpa, check_attention_special_cases,
     check_attention_gqa_mapping, check_logits_one_hot, check_acceptance_worked_examples,
@@ -558,5 +605,5 @@ ALL_CHECKS = [
     check_kv_commit, check_rope_worked_examples, check_rope_vs_complex_rotation,
     check_rope_relative_position, check_qkv_projection_layout, check_kv_write_slots,
     check_paged_worked_example, check_paged_matches_dense, check_temperature_worked_example,
-    check_temperature_output_law,
+    check_temperature_output_law, check_top_p_worked_example, check_top_p_output_law,
 ]

@@ -61,8 +61,13 @@ MUTANTS = {
                          "return rope(q, pos[:, None], theta), k, v"),
     "kv_write_wrong_slot": ("kc[seq[r], :, pos[r]] = k[r]", "kc[seq[r], :, pos[r] - 1] = k[r]"),
     # Temperature of p.
-    "temperature_multiplies": ("p = softmax(l / t_b)", "p = softmax(l * t_b)"),
-    "temperature_ignored_in_sampling": ("p = softmax(lr / t_b)", "p = softmax(lr)"),
+    "temperature_multiplies": ("nucleus(softmax(l_row / t_b), tp_b)", "nucleus(softmax(l_row * t_b), tp_b)"),
+    "temperature_ignored": ("nucleus(softmax(l_row / t_b), tp_b)", "nucleus(softmax(l_row), tp_b)"),
+    # Top-p truncation.
+    "nucleus_ascending": ("order = np.argsort(-p, kind=\"stable\")", "order = np.argsort(p, kind=\"stable\")"),
+    "nucleus_strict_reach": ("j = int(np.nonzero(c >= top_p)[0][0])", "j = int(np.nonzero(c > top_p)[0][0])"),
+    "nucleus_not_renormalised": ("    pt = pt / pt.sum()\n", ""),
+    "nucleus_drops_ties": ("keep = p >= tau", "keep = p > tau"),
     # Paged cache addressing.
     "paged_row_from_page_index": ("return int(block_table[b][s // page]), s % page",
                                   "return int(block_table[b][s // page]), s // page"),
