@@ -253,6 +253,44 @@ spade_status spade_verify_accept_temperature(const void *hidden, const void *w_l
                                              int32_t V, void *workspace, size_t workspace_bytes,
                                              int32_t *status, spade_stream_t stream);
 
+/*
+ * spade_verify_accept with the verifier's sampling options and an optional
+ * fused KV commit: the general form of the calls above.
+ *
+ * temperature [B] (float32, device; may be null: all 1): p = softmax(l / T_b)
+ *   for sequence b, as in spade_verify_accept_temperature.
+ * top_p [B] (float32, device; may be null: no truncation): stochastic sequences
+ *   take p truncated to its nucleus, S_b = {x : p(x) >= tau_b} with tau_b the
+ *   probability of the token at which the mass of p in descending order first
+ *   reaches top_p[b] (tokens tied with it included), renormalised on S_b --
+ *   for the accept test, the residual max(0, p - q) and the bonus draw alike
+ *   (Sec. III-A samples the verifier's distribution for diversity; the paper
+ *   fixes no truncation, this is the usual nucleus rule).  top_p[b] = 1 leaves
+ *   p whole; a value outside (0, 1] is reported (SPADE_DEV_BAD_INDEX) and
+ *   taken as 1.  Greedy sequences are unaffected.  tau_b is located by a
+ *   four-round 32-bin search over integer keys of l / T (2^16 per unit of
+ *   log-probability, from 31.5 below the row maximum; the last bit is not
+ *   resolved), so tokens whose log-probability lies within 3.1e-5 below the
+ *   boundary token's may also be in S_b, and tokens more than 31.5 below the
+ *   maximum (at most V e^-31.5 of p) never are.  Needs the one-launch path
+ *   (spade_accept_launches == 1): SPADE_ERR_SHAPE otherwise.  The row
+ *   statistics of spade_accept_stats_layout stay those of the whole p (the
+ *   accept bit there is the untruncated test).
+ * k_cache, v_cache, ctx_lens, Hkv, D, cap: as in spade_verify_accept_commit,
+ *   or all three pointers null for no commit.
+ * Every other argument is that of spade_verify_accept.
+ */
+spade_status spade_verify_accept_sampling(const void *hidden, const void *w_lm,
+                                          const int32_t *draft_tokens, const float *draft_probs,
+                                          const float *uniforms, const int32_t *mode,
+                                          const float *temperature, const float *top_p,
+                                          const int32_t *cu_q, const int32_t *n_draft,
+                                          int32_t *accepted_len, int32_t *next_token, void *k_cache,
+                                          void *v_cache, int32_t *ctx_lens, int32_t B, int32_t R,
+                                          int32_t H, int32_t V, int32_t Hkv, int32_t D, int32_t cap,
+                                          void *workspace, size_t workspace_bytes, int32_t *status,
+                                          spade_stream_t stream);
+
 /* Bytes of workspace spade_verify_accept needs (0 on invalid sizes). */
 size_t spade_accept_workspace_size(int32_t B, int32_t R, int32_t H, int32_t V);
 

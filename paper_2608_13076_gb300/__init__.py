@@ -27,7 +27,8 @@ __all__ = [
     "spade_verify_qkv_rope", "spade_qkv_workspace_size", "qkv_workspace", "spade_verify_attention_paged", "spade_kv_commit_paged",
     "spade_verify_qkv_rope_paged",
     "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_accept_launches",
-    "spade_accept_stats_layout", "read_accept_stats", "spade_verify_accept_commit", "spade_selftest_wait_timeout",
+    "spade_accept_stats_layout", "read_accept_stats", "spade_verify_accept_commit",
+    "spade_verify_accept_sampling", "spade_selftest_wait_timeout",
     "attn_workspace", "accept_workspace", "status_tensor", "check_status",
     "DEV_BAD_INDEX", "DEV_CAPACITY", "DEV_TIMEOUT", "DEV_FALLBACK",
 ]
@@ -87,6 +88,8 @@ def load():
     lib.spade_accept_workspace_size.argtypes = [_i32] * 4
     lib.spade_verify_accept_temperature.restype = _i32
     lib.spade_verify_accept_temperature.argtypes = [_vp] * 11 + [_i32] * 4 + [_vp, _sz, _vp, _vp]
+    lib.spade_verify_accept_sampling.restype = _i32
+    lib.spade_verify_accept_sampling.argtypes = [_vp] * 15 + [_i32] * 7 + [_vp, _sz, _vp, _vp]
     lib.spade_accept_stats_layout.restype = _i32
     lib.spade_accept_stats_layout.argtypes = [_i32] * 4 + [_vp, _vp, _vp]
     lib.spade_accept_launches.restype = _i32
@@ -330,6 +333,53 @@ def spade_verify_accept_commit(hidden, w_lm, draft_tokens, draft_probs, uniforms
         _ptr(cu_q), _ptr(n_draft), _ptr(accepted_len), _ptr(next_token), _ptr(k_cache), _ptr(v_cache),
         _ptr(ctx_lens), B, R, H, V, Hkv, D, cap, _ptr(workspace), workspace.numel(), _ptr(status),
         _stream(stream))
+    _check_rc(rc)
+    return accepted_len, next_token
+
+
+def spade_verify_accept_sampling(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
+                                 accepted_len, next_token, *, workspace, status, temperature=None, top_p=None,
+                                 k_cache=None, v_cache=None, ctx_lens=None, stream=None):
+    """spade_verify_accept with per-sequence ``temperature`` and ``top_p`` ([B] float32, either
+    may be None) and, with k_cache / v_cache / ctx_lens given, the fused KV commit
+    (see include/spade.h)."""
+    _need(hidden, "hidden", torch.bfloat16, 2)
+    _need(w_lm, "w_lm", torch.bfloat16, 2)
+    _need(uniforms, "uniforms", torch.float32, 1)
+    for t, n in ((draft_tokens, "draft_tokens"), (mode, "mode"), (cu_q, "cu_q"), (n_draft, "n_draft"),
+                 (accepted_len, "accepted_len"), (next_token, "next_token"), (status, "status")):
+        _need(t, n, torch.int32, 1)
+    if draft_probs is not None:
+        _need(draft_probs, "draft_probs", torch.float32, 2)
+    _need(workspace, "workspace", torch.uint8, 1)
+    R, H = hidden.shape
+    V, H2 = w_lm.shape
+    B = n_draft.numel()
+    if H2 != H or uniforms.numel() != R or draft_tokens.numel() != R - B or cu_q.numel() != B + 1 \
+            or mode.numel() != B or accepted_len.numel() != B or next_token.numel() != B:
+        raise ValueError("inconsistent accept shapes")
+    if draft_probs is not None and tuple(draft_probs.shape) != (R - B, V):
+        raise ValueError("draft_probs must be [R - B, V]")
+    for t, n in ((temperature, "temperature"), (top_p, "top_p")):
+        if t is not None:
+            _need(t, n, torch.float32, 1)
+            if t.numel() != B:
+                raise ValueError(f"{n} must be [B]")
+    Hkv = D = cap = 0
+    if (k_cache is None) != (v_cache is None) or (k_cache is None) != (ctx_lens is None):
+        raise ValueError("give all of k_cache, v_cache, ctx_lens or none")
+    if k_cache is not None:
+        _need(k_cache, "k_cache", torch.bfloat16, 4)
+        _need(v_cache, "v_cache", torch.bfloat16, 4)
+        _need(ctx_lens, "ctx_lens", torch.int32, 1)
+        Bc, Hkv, cap, D = k_cache.shape
+        if Bc != B or tuple(v_cache.shape) != tuple(k_cache.shape) or ctx_lens.numel() != B:
+            raise ValueError("inconsistent cache shapes")
+    rc = load().spade_verify_accept_sampling(
+        _ptr(hidden), _ptr(w_lm), _ptr(draft_tokens), _ptr(draft_probs), _ptr(uniforms), _ptr(mode),
+        _ptr(temperature), _ptr(top_p), _ptr(cu_q), _ptr(n_draft), _ptr(accepted_len), _ptr(next_token),
+        _ptr(k_cache), _ptr(v_cache), _ptr(ctx_lens), B, R, H, V, Hkv, D, cap, _ptr(workspace),
+        workspace.numel(), _ptr(status), _stream(stream))
     _check_rc(rc)
     return accepted_len, next_token
 

@@ -98,6 +98,10 @@ struct Params {
                      //      draft_probs row (-1: sample p), uniform bits, output index, row
   int *samp_count;   // number of specs
   const float *temperature;  // [B] softmax temperature of each sequence, or null (all 1)
+  const float *top_p;        // [B] nucleus mass of each sequence, or null (no truncation)
+  unsigned *nhist;           // [R][NC][kNucBins]: each CTA's bin masses of the nucleus search
+                             // (fixed point, 2^31 = all of p)
+  uint4 *nstate;             // [kReplicas][R]: key prefix, mass above the prefix's range, its upper mass
   __nv_bfloat16 *hidden_s;      // [B, H]: gathered hidden rows of the samples
   const __nv_bfloat16 *hidden;  // the call's hidden rows (gather source)
   // Fused KV commit (null kc: not requested): clear the rejected draft slots of
@@ -176,6 +180,10 @@ __device__ __forceinline__ unsigned ld_relaxed(const unsigned *p) {
 // for several microseconds, a handful per line do not.  The barrier's
 // generation word is replicated the same way, one 128-byte line per copy.
 constexpr int kReplicas = 8;
+constexpr int kNucBinBits = 5;                 // key bits decided per round of the nucleus search
+constexpr int kNucBins = 1 << kNucBinBits;     // bins per round
+constexpr int kNucRounds = 4;                  // all 20 key bits, see nuc_key
+constexpr int kNucSubs = 4;                    // independent bin copies per lane (see phase B (3b))
 constexpr int kGenWord = 32;      // words between the arrival count and each generation copy
 constexpr int kBarBytes = 2048;  // barrier words at the workspace's start
 static_assert(kGenWord * (kReplicas + 1) * 4 <= kBarBytes, "barrier words fit their region");
@@ -238,6 +246,41 @@ __device__ __forceinline__ float inv_temp(const Params &p, int b) {
     return 1.f;
   }
   return 1.f / t;
+}
+
+// Top-p (nucleus) threshold search over the scaled logits l of a row.  The
+// nucleus is S = {x : l_x >= tau}, tau the largest logit value whose upper
+// mass F(tau) = sum_{l_x >= tau} p_x reaches top_p (tokens tied with the
+// boundary are in).  The search runs on integer keys
+//   L(l) = floor((l - base) * 2^15),  base = m - 31.5  (m: the row maximum),
+// a monotone map of l onto [0, 2^20) for every l >= base (p below base is at
+// most V e^-31.5); each of kNucRounds rounds fixes 5 more bits of the key of
+// the boundary, keeping the highest bin whose upper mass still reaches top_p.
+// The nucleus is then {x : L(l_x) >= L_tau}: the same key decides the bins,
+// the accept test and the sampling, so all three agree bit for bit.  Logits
+// within one key step (2^-15 = 3.1e-5 in l) are not told apart.
+constexpr float kNucSpan = 31.5f;
+constexpr int kNucKeyBits = 20;
+constexpr float kNucScale = 32768.f;  // key steps per unit of l
+// y = fma(l, 2^15, -base 2^15) equals (l - base) rounded, times 2^15 (scaling
+// by a power of two commutes with rounding); adding 2^23 rounded toward -inf
+// leaves floor(y) in the low mantissa bits for 0 <= y < 2^23 (no conversion
+// instruction), and a negative key for y < 0.  Monotone in l throughout.
+// nb65 = -base * 2^15 (exact).  nuc_key_bits is the float's bit pattern,
+// 0x4B000000 + L for L >= 0 (the constant's low 24 bits are zero, so shifts
+// of the pattern and of L differ by a constant).
+constexpr int kNucKeyBias = 0x4B000000;
+__device__ __forceinline__ int nuc_key_bits(float l, float nb65) {
+  return __float_as_int(__fadd_rd(__fmaf_rn(l, kNucScale, nb65), 8388608.f));
+}
+__device__ __forceinline__ int nuc_key(float l, float base) {
+  return nuc_key_bits(l, -kNucScale * base) - kNucKeyBias;
+}
+// top_p of sequence b when it truncates p (0 < top_p < 1), else 1.
+__device__ __forceinline__ float seq_top_p(const Params &p, int b) {
+  if (p.top_p == nullptr || b < 0) return 1.f;
+  const float t = __ldg(p.top_p + b);
+  return (t > 0.f && t < 1.f) ? t : 1.f;
 }
 
 // Float-float numbers (hi + lo, about 48 significant bits) for the sums that
@@ -933,7 +976,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   float2 *s_tw = reinterpret_cast<float2 *>(s_zw + kMaxB * kEpiWarps);  // [tiles][kEpiWarps]
   int *s_slist = reinterpret_cast<int *>(s_tw + kMaxTilesPerCta * kEpiWarps);  // [B] sampled sequences
   int *s_slpos = s_slist + kMaxB;                           // [B] position in s_slist, -1: none
-  float *f_R = reinterpret_cast<float *>(s_slpos + kMaxB);  // [kFG][kFastSegs][kSegPad] residual terms
+  int *g_tkey = s_slpos + kMaxB;                            // [R] nucleus key threshold (INT_MIN: all of p)
+  float *f_R = reinterpret_cast<float *>(g_tkey + kMaxR);   // [kFG][kFastSegs][kSegPad] residual terms
   float *f_Q = f_R + kFG * kFastSegs * kSegPad;             // [kFG][kQStride] q of staged rows
   float2 *f_seg = reinterpret_cast<float2 *>(f_Q + kFG * kQStride);  // [kFastSeqs][kFastSegs]
   uint32_t q_phase = 0;
@@ -944,13 +988,276 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     g_s[n] = g.y;
     g_arg[n] = __float_as_int(g.z);
     s_ok[n] = __float_as_int(g.w);
+    g_tkey[n] = INT_MIN;
   }
   for (int b = tid; p.kind != kPresampled && b < p.B; b += kThreads) {
     const int md = s_md[b];
     if (md != 0 && md != 1 && c == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
     s_stoch[b] = (md == 1) && p.draft_probs != nullptr;
+    if (p.top_p != nullptr && c == 0) {
+      const float t = __ldg(p.top_p + b);
+      if (!(t > 0.f && t <= 1.f)) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
+    }
   }
   block_sync();
+  if (p.top_p != nullptr && p.kind == kResident) {
+    // (3b) Top-p: the nucleus of every row of a stochastic sequence with
+    //      top_p < 1 (see nuc_key).  Per round: every CTA bins its slice of
+    //      each listed row and stores the bins to its own slot of the
+    //      workspace (plain stores: 152 CTAs adding into the same lines
+    //      serialise for hundreds of microseconds); after a grid barrier the
+    //      CTA owning a row sums the slots, takes the bin and publishes the
+    //      longer key prefix in kReplicas copies; after a second barrier every
+    //      CTA reads it.  Bin masses are fixed point (2^31 = all of p, each
+    //      term rounded to nearest): integer sums, the same in any order.
+    //      Scratch:
+    //      the phase-C staging area, idle until then.
+    int *s_nl = reinterpret_cast<int *>(f_R);                  // [R] listed rows, ascending
+    int *s_npre = s_nl + kMaxR;                                // [R] key prefix of row n (-1: not listed)
+    unsigned *s_nab = reinterpret_cast<unsigned *>(s_npre + kMaxR);  // [R] mass above the prefix; at the end, F
+    float *s_hp = reinterpret_cast<float *>(s_nab + kMaxR);   // [kEpiWarps][kNucSubs][kNucBins][32] lane-private bins
+    if (warp == 0) {
+      int base = 0;
+      for (int n0 = 0; n0 < p.R; n0 += 32) {
+        const int n = n0 + lane;
+        const int b = n < p.R ? s_seq[n] : -1;
+        const bool want = b >= 0 && s_md[b] == 1 && p.draft_probs != nullptr && seq_top_p(p, b) < 1.f &&
+                          isfinite(g_m[n]) && g_s[n] > 0.f;
+        const unsigned bal = __ballot_sync(0xffffffffu, want);
+        if (want) s_nl[base + __popc(bal & ((1u << lane) - 1u))] = n;
+        base += __popc(bal);
+      }
+      if (lane == 0) s_seg[8] = base;
+    }
+    block_sync();
+    const int nl = s_seg[8];
+    for (int n = tid; n < kMaxR; n += kThreads) {
+      s_npre[n] = -1;
+      s_nab[n] = 0u;
+    }
+    block_sync();
+    for (int i = tid; i < nl; i += kThreads) s_npre[s_nl[i]] = 0;
+    block_sync();
+#pragma unroll 1
+    for (int r = 0; nl > 0 && r < kNucRounds; ++r) {
+      const int sh = kNucKeyBits - kNucBinBits * (r + 1);  // this round's bin: key bits [sh, sh + 5)
+      if (warp >= 2) {
+        // Rows in chunks of 32.  Each warp loads its lane quarter of every
+        // tile (lane = vocabulary entry, 32 columns in four 8-column loads,
+        // the next tile's loads in flight while this one is binned) and
+        // transposes it through its shared buffer, so that lane i owns row
+        // 32 j + i.  Its bins are fp32 sums kept in kNucSubs copies: value u of
+        // a batch goes to copy u % kNucSubs, so the read-add-write of four
+        // values never waits on another's write (shared-memory atomics cost
+        // tens of cycles per instruction here); each copy's sums follow a
+        // fixed order.  Layout bin-major, lane-minor: lane i's words all sit
+        // in bank i, so no access conflicts.
+        const int ew = warp - 2, q4 = warp & 3;
+        const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
+        float *T = s_tbuf + ew * (32 * 33);
+        float *hp = s_hp + ew * (kNucSubs * kNucBins * 32) + lane;
+#pragma unroll 1
+        for (int r0 = 0; r0 < p.R; r0 += 32) {
+          const int n = r0 + lane;
+          const int pre = n < p.R ? s_npre[n] : -1;
+          const bool has = pre >= 0;
+          if (__ballot_sync(0xffffffffu, has) == 0u) continue;  // the same on every warp
+          const int nn = has ? n : r0;
+          const float M = g_m[nn];
+          const float nb65 = -kNucScale * __fsub_rn(M, kNucSpan);
+          const float mlog = -M * kLog2e;
+          const float IT = inv_temp(p, has ? s_seq[nn] : -1);
+          const int pre_bits = pre + (kNucKeyBias >> (sh + kNucBinBits));  // the range's key prefix, as bits
+          const int nc = min(32, p.Rs - r0);  // columns of this chunk (multiple of 8)
+#pragma unroll 8
+          for (int k = 0; k < kNucSubs * kNucBins; ++k) hp[k * 32] = 0.f;
+          uint32_t raw[32];
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (8 * q < nc) tmem_ld8(tmem + lane_base + static_cast<uint32_t>(r0 + 8 * q), raw + 8 * q);
+#pragma unroll 1
+          for (int t = 0; t < ntiles; ++t) {
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (i < nc) T[lane * 33 + i] = __uint_as_float(raw[i]);
+            if (t + 1 < ntiles) {
+              const uint32_t col = tmem + lane_base + static_cast<uint32_t>((t + 1) * p.Rs + r0);
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+                if (8 * q < nc) tmem_ld8(col + 8 * q, raw + 8 * q);
+            }
+            __syncwarp();
+            const int nv = min(32, v_hi - (v_lo + t * kTileV + q4 * 32));  // valid entries, warp-uniform
+            if (has) {
+#pragma unroll 1
+              for (int j0 = 0; j0 < nv; j0 += 8) {
+                float x[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) x[u] = T[(j0 + u) * 33 + lane];
+#pragma unroll
+                for (int h = 0; h < 8; h += kNucSubs) {
+                  float e[kNucSubs];
+                  int a[kNucSubs];
+#pragma unroll
+                  for (int u = 0; u < kNucSubs; ++u) {
+                    const float l = __fmul_rn(x[h + u], IT);
+                    const int kbits = nuc_key_bits(l, nb65);
+                    const bool in = j0 + h + u < nv && (kbits >> (sh + kNucBinBits)) == pre_bits;
+                    e[u] = in ? ex2(__fmaf_rn(l, kLog2e, mlog)) : 0.f;
+                    a[u] = (u * kNucBins + ((kbits >> sh) & (kNucBins - 1))) * 32;
+                  }
+                  float v[kNucSubs];
+#pragma unroll
+                  for (int u = 0; u < kNucSubs; ++u) v[u] = hp[a[u]];
+#pragma unroll
+                  for (int u = 0; u < kNucSubs; ++u) hp[a[u]] = v[u] + e[u];
+                }
+              }
+            }
+            __syncwarp();
+          }
+          // The four warps' bins of these rows: thread (ew, lane) adds bins
+          // [8 ew, 8 ew + 8) of row r0 + lane over the warps and copies (fixed
+          // order), converts them to fixed point and stores them to this CTA's slot.
+          named_bar(1, kEpiWarps * 32);
+          if (has) {
+            constexpr int kPer = kNucBins / kEpiWarps;
+            const float sc = 0x1p31f / g_s[n];  // fixed point: 2^31 = all of p
+            uint4 *dst = reinterpret_cast<uint4 *>(p.nhist + (static_cast<size_t>(n) * p.NC + c) * kNucBins + ew * kPer);
+#pragma unroll
+            for (int k4 = 0; k4 < kPer; k4 += 4) {
+              unsigned tot[4];
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                float f = 0.f;
+#pragma unroll
+                for (int w4 = 0; w4 < kEpiWarps; ++w4)
+#pragma unroll
+                  for (int u = 0; u < kNucSubs; ++u)
+                    f += s_hp[((w4 * kNucSubs + u) * kNucBins + ew * kPer + k4 + k) * 32 + lane];
+                tot[k] = __float2uint_rn(f * sc);
+              }
+              __stcg(dst + k4 / 4, make_uint4(tot[0], tot[1], tot[2], tot[3]));
+            }
+          }
+          named_bar(1, kEpiWarps * 32);  // the next chunk clears the bins
+        }
+      }
+      if (!grid_barrier(p.bar, p.NC)) {
+        atomicOr(p.status, SPADE_DEV_TIMEOUT);
+        *s_abort = 1;
+      }
+      // Owner of listed row i: CTA i % NC.  A slot is kNucBins / 4 16-byte
+      // words (four bins each); thread t adds word t % 8 of the slots of CTAs
+      // t / 8, t / 8 + 24, ..., all loads in flight.  Warp 0 then holds bins
+      // 4 q .. 4 q + 3 in lane q < 8, forms the upper masses C_k (mass of keys
+      // at or above bin k, plus the mass above the range) by a suffix scan
+      // over the lanes and keeps the highest bin with C_k >= top_p.  Sums stay
+      // below 2^32 (all of p is 2^31).
+      constexpr int kWps = kNucBins / 4;        // words per slot
+      constexpr int kGroups = kThreads / kWps;  // CTA groups
+      uint4 *s_red = reinterpret_cast<uint4 *>(s_zw);  // [kGroups][kWps] (phase-C buffer)
+#pragma unroll 1
+      for (int i = c; i < nl; i += p.NC) {
+        const int n = s_nl[i];
+        const uint4 *src = reinterpret_cast<const uint4 *>(p.nhist + static_cast<size_t>(n) * p.NC * kNucBins) + tid % kWps;
+        uint4 acc4 = make_uint4(0u, 0u, 0u, 0u);
+        constexpr int kLoads = (kMaxNC + kGroups - 1) / kGroups;
+        uint4 v[kLoads];
+#pragma unroll
+        for (int j = 0; j < kLoads; ++j) {
+          const int k = tid / kWps + j * kGroups;
+          v[j] = k < p.NC ? __ldcg(src + static_cast<size_t>(k) * kWps) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int j = 0; j < kLoads; ++j) {
+          acc4.x += v[j].x; acc4.y += v[j].y; acc4.z += v[j].z; acc4.w += v[j].w;
+        }
+        s_red[tid] = acc4;  // = [tid / kWps][tid % kWps]
+        block_sync();
+        if (warp == 0) {
+          unsigned long long bq[4] = {0, 0, 0, 0};
+          if (lane < kWps) {
+#pragma unroll 4
+            for (int g = 0; g < kGroups; ++g) {
+              const uint4 t = s_red[g * kWps + lane];
+              bq[0] += t.x; bq[1] += t.y; bq[2] += t.z; bq[3] += t.w;
+            }
+          }
+
+          const unsigned long long tq = bq[0] + bq[1] + bq[2] + bq[3];
+          unsigned long long suf = tq;  // inclusive suffix sum over lanes >= this one
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const unsigned long long t = __shfl_down_sync(0xffffffffu, suf, o);
+            if (lane + o < 32) suf += t;
+          }
+          // D[j] = C_{4 lane + j}; D[4] = the mass above this lane's bins.
+          unsigned long long D[5];
+          D[4] = s_nab[n] + (suf - tq);
+#pragma unroll
+          for (int j = 3; j >= 0; --j) D[j] = D[j + 1] + bq[j];
+          // top_p * 2^31 is exact in fp32; the target is its ceiling.
+          const unsigned long long target =
+              static_cast<unsigned long long>(ceilf(seq_top_p(p, s_seq[n]) * 0x1p31f));
+          const int jj = lane >= kWps ? -1 : D[3] >= target ? 3 : D[2] >= target ? 2 : D[1] >= target ? 1
+                                           : D[0] >= target ? 0 : -1;
+          const unsigned ge = __ballot_sync(0xffffffffu, jj >= 0);
+          const int ls = ge ? 31 - __clz(ge) : 0;  // C_k falls with k: the highest lane with a hit
+          unsigned long long ck = D[0], ck1 = D[1];
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (jj == j) { ck = D[j]; ck1 = D[j + 1]; }
+          const int kq = __shfl_sync(0xffffffffu, jj < 0 ? 0 : jj, ls);
+          ck = __shfl_sync(0xffffffffu, ck, ls);
+          ck1 = __shfl_sync(0xffffffffu, ck1, ls);
+          if (lane < kReplicas) {
+            const int kb = ge ? 4 * ls + kq : 0;
+            const uint4 ns = make_uint4(static_cast<unsigned>((s_npre[n] << kNucBinBits) | kb),
+                                        static_cast<unsigned>(min(ck1, 0xffffffffull)),
+                                        static_cast<unsigned>(min(ck, 0xffffffffull)), 0u);
+            __stcg(&p.nstate[static_cast<size_t>(lane) * p.R + n], ns);
+          }
+        }
+        block_sync();  // s_red is free again
+      }
+      if (!grid_barrier(p.bar, p.NC)) {
+        atomicOr(p.status, SPADE_DEV_TIMEOUT);
+        *s_abort = 1;
+      }
+      for (int i = tid; i < nl; i += kThreads) {
+        const int n = s_nl[i];
+        const uint4 ns = __ldcg(&p.nstate[static_cast<size_t>(c % kReplicas) * p.R + n]);
+        s_npre[n] = static_cast<int>(ns.x);
+        // The mass above the new prefix's range; after the last round F(tau).
+        s_nab[n] = r + 1 < kNucRounds ? ns.y : ns.z;
+      }
+      block_sync();
+    }
+    // L_tau = the final prefix followed by zero bits; p on S renormalised by
+    // S_nuc = F(tau).  The accept test of a listed draft row is taken again
+    // under the nucleus (the merge step took it on all of p).
+    for (int i = tid; i < nl; i += kThreads) {
+      const int n = s_nl[i];
+      const unsigned F = s_nab[n];
+      if (F == 0u) continue;  // nothing reached top_p (not expected): all of p
+      const float S = g_s[n] * (static_cast<float>(F) * 0x1p-31f);
+      const int tkey = s_npre[n] << (kNucKeyBits - kNucBinBits * kNucRounds);
+      const float base = __fsub_rn(g_m[n], kNucSpan);
+      g_tkey[n] = tkey;
+      g_s[n] = S;
+      const int b = s_seq[n];
+      const int d = s_draft[n];
+      if (s_pos[n] < s_nd[b] && d >= 0 && d < p.V) {
+        const float ld = __ldcg(&p.ldraft[n]);
+        const float pd = nuc_key(ld, base) >= tkey ? expf(ld - g_m[n]) / S : 0.f;
+        const float qd = s_qd[n];
+        s_ok[n] = (qd > 0.f) ? (s_u[n] < pd / qd) : (pd > 0.f);
+      }
+    }
+    block_sync();
+  }
   if (p.kind != kPresampled) {
   // (4) Accepted length = leading accepts; the row that emits the next token.
   for (int b = tid; b < p.B; b += kThreads) {
@@ -1147,6 +1454,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             // past the slice re-read its last tile and store zeros.
             int n_l = -1, hq_l = 0;
             float m_l = 0.f, is_l = 0.f, it_l = 1.f;
+            int tk_l = INT_MIN;
             if (lane < ng) {
               const int b = s_slist[g0 + lane];
               n_l = (attempt == 0 || s_usep[b]) ? s_rstar[b] : -1;
@@ -1155,6 +1463,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
                 m_l = g_m[n_l];
                 is_l = 1.f / g_s[n_l];
                 it_l = inv_temp(p, s_outb[b]);
+                tk_l = g_tkey[n_l];
               }
             }
 #pragma unroll 1
@@ -1163,6 +1472,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               const bool hasq = __shfl_sync(0xffffffffu, hq_l, gi) != 0;
               const float M = __shfl_sync(0xffffffffu, m_l, gi), invS = __shfl_sync(0xffffffffu, is_l, gi);
               const float IT = __shfl_sync(0xffffffffu, it_l, gi);  // 1 / T of the row
+              const int TK = __shfl_sync(0xffffffffu, tk_l, gi);  // nucleus key threshold
+              const float BASE = __fsub_rn(M, kNucSpan);
               uint32_t raw[kTiles];
               if (n >= 0) {
 #pragma unroll
@@ -1187,7 +1498,9 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
 #pragma unroll
               for (int t = 0; t < kTiles; ++t) {
                 const int e = t * kTileV + q4 * 32 + lane;  // < kFastSlice: inside the row's buffers
-                const float pv = ex2((__uint_as_float(raw[t]) * IT - M) * kLog2e) * invS;
+                const float lv = __fmul_rn(__uint_as_float(raw[t]), IT);
+                const bool in = TK == INT_MIN || nuc_key(lv, BASE) >= TK;
+                const float pv = in ? ex2((lv - M) * kLog2e) * invS : 0.f;
                 const float rv = hasq ? fmaxf(0.f, pv - qv[t]) : pv;
                 rrow[(e >> 5) * kSegPad + (e & 31)] = e < slen ? rv : 0.f;
               }
@@ -1239,6 +1552,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           const float *qrow[kG];
           int nrow[kG];
           float M[kG], invS[kG], IT[kG];
+          int TK[kG];
           ff2 z[kG], zp[kG];
   #pragma unroll
           for (int g = 0; g < kG; ++g) {
@@ -1248,6 +1562,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             M[g] = g_m[nrow[g]];
             invS[g] = 1.f / g_s[nrow[g]];
             IT[g] = inv_temp(p, s_outb[b]);
+            TK[g] = g_tkey[nrow[g]];
             z[g] = ff2{0.f, 0.f};
             zp[g] = ff2{0.f, 0.f};
           }
@@ -1277,7 +1592,9 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
               for (int j = 0; j < 8; ++j) {
                 const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
                 if (g < nb && j < nj && v < v_hi) {
-                  const float pv = ex2((__uint_as_float(raw[g][j]) * IT[g] - M[g]) * kLog2e) * invS[g];
+                  const float lv = __fmul_rn(__uint_as_float(raw[g][j]), IT[g]);
+                  const bool in = TK[g] == INT_MIN || nuc_key(lv, __fsub_rn(M[g], kNucSpan)) >= TK[g];
+                  const float pv = in ? ex2((lv - M[g]) * kLog2e) * invS[g] : 0.f;
                   zp[g] = ff_add_f(zp[g], pv);
                   z[g] = ff_add_f(z[g], qrow[g] ? fmaxf(0.f, pv - qv[g][j]) : pv);
                 }
@@ -1400,6 +1717,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         const float *qrow = (s_qidx[b] >= 0 && !usep) ? p.draft_probs + static_cast<size_t>(s_qidx[b]) * p.V : nullptr;
         const float M = g_m[n], invS = 1.f / g_s[n];
         const float IT = inv_temp(p, s_outb[b]);  // 1 / T of the row
+        const int TK = g_tkey[n];                  // nucleus key threshold (INT_MIN: all of p)
+        const float BASE = __fsub_rn(M, kNucSpan);
         // (1) mass of every 32-entry segment (tile j, lane quarter q4) of the slice:
         //     from phase C's shared-memory sums, else recomputed.
         if (fastc) {
@@ -1428,7 +1747,9 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             const int v = v_lo + (j0 + j) * kTileV + q4 * 32 + lane;
             float rv = 0.f;
             if (j < nj && v < v_hi) {
-              const float pv = ex2((__uint_as_float(raw[j]) * IT - M) * kLog2e) * invS;
+              const float lv = __fmul_rn(__uint_as_float(raw[j]), IT);
+              const bool in = TK == INT_MIN || nuc_key(lv, BASE) >= TK;
+              const float pv = in ? ex2((lv - M) * kLog2e) * invS : 0.f;
               rv = qrow ? fmaxf(0.f, pv - qv[j]) : pv;
             }
             const ff2 seg = warp_sum_ff(ff2{rv, 0.f});
@@ -1467,7 +1788,9 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           tmem_wait_ld();
           float rv = 0.f;
           if (v < v_hi) {
-            const float pv = ex2((__uint_as_float(raw) * IT - M) * kLog2e) * invS;
+            const float lv = __fmul_rn(__uint_as_float(raw), IT);
+            const bool in = TK == INT_MIN || nuc_key(lv, BASE) >= TK;
+            const float pv = in ? ex2((lv - M) * kLog2e) * invS : 0.f;
             rv = qrow ? fmaxf(0.f, pv - qv) : pv;
           }
           const ff2 incl = warp_scan_ff(ff2{rv, 0.f}, lane);
@@ -1572,7 +1895,7 @@ static void slice_shape(int V, int NC, int *tiles_max, int *brs) {
 
 // Scratch of one launch: slice partials, draft logits, merged statistics, slice masses.
 struct WsRegion {
-  size_t pstat, ldraft, gstat, zpart, end;
+  size_t pstat, ldraft, gstat, zpart, nhist, nstate, end;
 };
 static WsRegion ws_region(size_t off, int B, int R, int NC) {
   WsRegion w;
@@ -1584,6 +1907,10 @@ static WsRegion ws_region(size_t off, int B, int R, int NC) {
   off += round_up(static_cast<size_t>(kReplicas) * R * 16, 256);
   w.zpart = off;
   off += round_up(static_cast<size_t>(kReplicas) * NC * B * 8, 256);
+  w.nhist = off;
+  off += round_up(static_cast<size_t>(R) * NC * kNucBins * 4, 256);
+  w.nstate = off;
+  off += round_up(static_cast<size_t>(kReplicas) * R * 16, 256);
   w.end = off;
   return w;
 }
@@ -1739,16 +2066,21 @@ static spade_status prepare(Params &p, int kind, const void *hidden, const void 
   }
   if (p.WS < 2) return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
   // Bytes of the W ring that phases B-D use (the per-row / per-sequence
-  // arrays, then the staging buffers and segment masses of phase C).
+  // arrays, then the staging buffers and segment masses of phase C, which
+  // the nucleus search uses before phase C).
   constexpr size_t kPhaseBBytes = 4 * kMaxR * 4 + 8 * kMaxB * 4 + 16 * 4 + kMaxB * 8 +
-                                  kMaxB * kEpiWarps * 16 + kMaxTilesPerCta * kEpiWarps * 8;
-  constexpr size_t kFastBytes = kPhaseBBytes + 2 * kMaxB * 4 + kFG * (kFastSegs * kSegPad + kQStride) * 4 +
+                                  kMaxB * kEpiWarps * 16 + kMaxTilesPerCta * kEpiWarps * 8 +
+                                  2 * kMaxB * 4 + kMaxR * 4;
+  constexpr size_t kFastBytes = kPhaseBBytes + kFG * (kFastSegs * kSegPad + kQStride) * 4 +
                                 kFastSeqs * kFastSegs * 8;
+  constexpr size_t kNucBytes = kPhaseBBytes + kMaxR * 12 + kEpiWarps * kNucSubs * kNucBins * 32 * 4;  // phase B (3b)
   const size_t ring = static_cast<size_t>(p.WS) * p.KG * kWChunkBytes;
   if (ring < kPhaseBBytes) return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
   // After phase A the W and hidden rings (contiguous) are free.
-  p.fastc = static_cast<size_t>(smem_layout(p).off_bar) >= kFastBytes &&
-            (p.V + p.NC - 1) / p.NC <= kFastSlice;
+  const size_t freeb = static_cast<size_t>(smem_layout(p).off_bar);
+  p.fastc = freeb >= kFastBytes && (p.V + p.NC - 1) / p.NC <= kFastSlice;
+  if (p.top_p != nullptr && freeb < kNucBytes)
+    return fail(SPADE_ERR_SHAPE, "shared memory too small for the top-p search at R = %d", R);
   p.NS = (p.KC + p.KG - 1) / p.KG;
   if (smem_layout(p).total > kSmemMax) return fail(SPADE_ERR_SHAPE, "shared memory plan too large");
 
@@ -1806,6 +2138,8 @@ static void set_region(Params &p, uint8_t *ws, const WsRegion &r) {
   p.ldraft = reinterpret_cast<float *>(ws + r.ldraft);
   p.gstat = reinterpret_cast<float4 *>(ws + r.gstat);
   p.zpart = reinterpret_cast<float2 *>(ws + r.zpart);
+  p.nhist = reinterpret_cast<unsigned *>(ws + r.nhist);
+  p.nstate = reinterpret_cast<uint4 *>(ws + r.nstate);
 }
 
 }  // namespace accept
@@ -1861,7 +2195,8 @@ static spade_status verify_accept_impl(const void *hidden, const void *w_lm,
                                        int32_t R, int32_t H, int32_t V, void *workspace,
                                        size_t workspace_bytes, int32_t *status,
                                        spade_stream_t stream, const CommitArgs *cm,
-                                       const float *temperature = nullptr) {
+                                       const float *temperature = nullptr,
+                                       const float *top_p = nullptr) {
   using namespace accept;
   if (!hidden || !w_lm || !uniforms || !mode || !cu_q || !n_draft || !accepted_len ||
       !next_token || !status || (R > B && !draft_tokens))
@@ -1878,6 +2213,8 @@ static spade_status verify_accept_impl(const void *hidden, const void *w_lm,
   if (st != SPADE_OK) return st;
 
   const WsLayout L = ws_layout(B, R, H, V, sms);
+  if (top_p && L.two_pass)
+    return fail(SPADE_ERR_SHAPE, "top-p needs the logits resident: R = %d rows x V = %d exceed one launch", R, V);
   if (!workspace || workspace_bytes < L.end || !aligned(workspace, 256))
     return fail(SPADE_ERR_WORKSPACE, "accept workspace needs %zu bytes, 256-byte aligned (got %zu)",
                 L.end, workspace_bytes);
@@ -1888,6 +2225,7 @@ static spade_status verify_accept_impl(const void *hidden, const void *w_lm,
   p.draft_tokens = draft_tokens;
   p.draft_probs = draft_probs;
   p.temperature = temperature;
+  p.top_p = top_p;
   p.qbulk = draft_probs != nullptr && aligned(draft_probs, 16) && V % 4 == 0;
   p.uniforms = uniforms;
   p.mode = mode;
@@ -1976,4 +2314,26 @@ extern "C" spade_status spade_verify_accept_temperature(
   return accept::verify_accept_impl(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
                                     accepted_len, next_token, B, R, H, V, workspace, workspace_bytes, status,
                                     stream, nullptr, temperature);
+}
+
+extern "C" spade_status spade_verify_accept_sampling(
+    const void *hidden, const void *w_lm, const int32_t *draft_tokens, const float *draft_probs,
+    const float *uniforms, const int32_t *mode, const float *temperature, const float *top_p,
+    const int32_t *cu_q, const int32_t *n_draft, int32_t *accepted_len, int32_t *next_token, void *k_cache,
+    void *v_cache, int32_t *ctx_lens, int32_t B, int32_t R, int32_t H, int32_t V, int32_t Hkv, int32_t D,
+    int32_t cap, void *workspace, size_t workspace_bytes, int32_t *status, spade_stream_t stream) {
+  const bool commit = k_cache || v_cache || ctx_lens;
+  if (commit) {
+    if (!k_cache || !v_cache || !ctx_lens)
+      return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_sampling: give all of k_cache, v_cache, ctx_lens or none");
+    if (Hkv <= 0 || D <= 0 || cap <= 0)
+      return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_sampling: non-positive cache size");
+    if (D % 8) return fail(SPADE_ERR_SHAPE, "spade_verify_accept_sampling: D = %d must be a multiple of 8", D);
+    if (!aligned(k_cache, 16) || !aligned(v_cache, 16))
+      return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_sampling: caches must be 16-byte aligned");
+  }
+  const accept::CommitArgs cm{k_cache, v_cache, ctx_lens, Hkv, D, cap};
+  return accept::verify_accept_impl(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
+                                    accepted_len, next_token, B, R, H, V, workspace, workspace_bytes, status,
+                                    stream, commit ? &cm : nullptr, temperature, top_p);
 }

@@ -46,6 +46,7 @@ class WorkloadSpec:
     greedy_draft: str = "match" # greedy drafts: "match" (match_prob) or "noisy_argmax"
     seed: int = 0
     rope_theta: float = 10000.0  # base of the rotary frequencies of the model family
+    logit_scale: float = 1.0     # std of the hidden rows: logits ~ N(0, logit_scale^2)
     extra: dict = field(default_factory=dict)
 
 
@@ -148,7 +149,7 @@ def make_workload(spec: WorkloadSpec, device="cpu", cache_pad: int = 0):
         L = int(ctx[b] + kd[b] + 1)
         k_cache[b, :, :L] = _bf16_normal(gen, (spec.Hkv, L, spec.D), 1.0, cpu)
         v_cache[b, :, :L] = _bf16_normal(gen, (spec.Hkv, L, spec.D), 1.0, cpu)
-    hidden = _bf16_normal(gen, (R, spec.H), 1.0, cpu)
+    hidden = _bf16_normal(gen, (R, spec.H), spec.logit_scale, cpu)
     w_lm = _bf16_normal(gen, (spec.V, spec.H), 1.0 / math.sqrt(spec.H), cpu)
 
     # Draft rows: row cu_q[b]+i (i < k_b) holds draft i of sequence b.

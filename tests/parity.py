@@ -81,14 +81,32 @@ def gpu_accept_commit(wl, workspace=None, status=None):
     return acc, tok, workspace, status
 
 
+def gpu_accept_sampling(wl, temperature=None, top_p=None, commit=False, workspace=None, status=None):
+    """spade_verify_accept_sampling on wl (with commit: updates wl's caches and ctx_lens)."""
+    dev = wl["hidden"].device
+    B = wl["B"]
+    acc = torch.full((B,), -7, dtype=torch.int32, device=dev)
+    tok = torch.full((B,), -7, dtype=torch.int32, device=dev)
+    if workspace is None:
+        workspace = spade.accept_workspace(B, wl["R"], wl["H"], wl["V"], device=dev)
+    if status is None:
+        status = spade.status_tensor(dev)
+    cache = dict(k_cache=wl["k_cache"], v_cache=wl["v_cache"], ctx_lens=wl["ctx_lens"]) if commit else {}
+    spade.spade_verify_accept_sampling(wl["hidden"], wl["w_lm"], wl["draft_tokens"], wl["draft_probs"],
+                                       wl["uniforms"], wl["mode"], wl["cu_q"], wl["n_draft"], acc, tok,
+                                       workspace=workspace, status=status, temperature=temperature,
+                                       top_p=top_p, **cache)
+    return acc, tok, status
+
+
 def oracle_logits(wl):
     return O.lm_logits(to_np(wl["hidden"]), to_np(wl["w_lm"]))
 
 
-def oracle_accept_from_logits(wl, logits, temperature=None):
+def oracle_accept_from_logits(wl, logits, temperature=None, top_p=None):
     return O.verify_accept(logits, to_np(wl["draft_tokens"]), to_np(wl["draft_probs"]),
                            to_np(wl["uniforms"]), to_np(wl["mode"]), to_np(wl["cu_q"]),
-                           to_np(wl["n_draft"]), temperature=temperature)
+                           to_np(wl["n_draft"]), temperature=temperature, top_p=top_p)
 
 
 def oracle_attention(wl, rows=None):

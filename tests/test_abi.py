@@ -69,6 +69,25 @@ def test_null_arguments_rejected_before_any_device_work(lib):
     assert rc == 1
     rc = lib.spade_verify_accept_commit(*([None] * 13), 1, 5, 512, 1024, 8, 128, 300, None, 0, None, None)
     assert rc == 1
+    rc = lib.spade_verify_accept_sampling(*([None] * 15), 1, 5, 512, 1024, 0, 0, 0, None, 0, None, None)
+    assert rc == 1
+
+
+def test_sampling_entry_point_validation_before_device_work(lib):
+    p = ctypes.c_void_p(16)
+    base = [p] * 12  # hidden .. next_token, temperature and top_p given
+    # Cache pointers: all three or none.
+    assert lib.spade_verify_accept_sampling(*base, p, None, None, 1, 5, 512, 1024, 8, 128, 300,
+                                            p, 1 << 20, p, None) == 1
+    assert b"all of k_cache" in lib.spade_last_error()
+    # Non-positive cache sizes with a commit.
+    assert lib.spade_verify_accept_sampling(*base, p, p, p, 1, 5, 512, 1024, 0, 128, 300,
+                                            p, 1 << 20, p, None) == 1
+    # Head dim not a multiple of 8 with a commit; hidden size not a multiple of 8.
+    assert lib.spade_verify_accept_sampling(*base, p, p, p, 1, 5, 512, 1024, 8, 12, 300,
+                                            p, 1 << 20, p, None) == 2
+    assert lib.spade_verify_accept_sampling(*base, None, None, None, 1, 5, 500, 1024, 0, 0, 0,
+                                            p, 1 << 20, p, None) == 2
 
 
 def test_selftest_rejects_bad_arguments_before_device_work(lib):
