@@ -455,6 +455,9 @@ def run_spade(args, ws, rank, local):
         base, par = cpu_baseline(wl_cpu, acc.cpu(), tok.cpu())
         line["cpu_baseline"] = base
         line["parity"] = par
+    if rank == 0 and ws == 1 and not args.no_sampling and spade.spade_accept_launches(
+            wl["B"], wl["R"], wl["H"], wl["V"]) == 1:
+        line["sampling"] = sampling_report(wl, dev)
     if rank == 0 and ws == 1 and not args.no_loop:
         line["speculative_loop"] = loop_report(dev)
     if rank == 0 and ws == 1 and not args.no_per_workload:
@@ -582,6 +585,47 @@ def per_workload(args, dev, skip):
                      "steps": args.per_workload_steps, "timing": "median of CUDA-event times per launch"}
         del wl
         torch.cuda.empty_cache()
+    return res
+
+
+def sampling_report(wl, dev, launches=20):
+    """Device time of the LM-head + accept launch with the verifier's sampling options (no
+    commit): p whole, temperature 0.8, top-p 0.9, and both, on every sequence of the step."""
+    import paper_2608_13076_gb300 as spade
+
+    B, R = wl["B"], wl["R"]
+    acc = torch.zeros(B, dtype=torch.int32, device=dev)
+    tok = torch.zeros(B, dtype=torch.int32, device=dev)
+    status = spade.status_tensor(dev)
+    ws_acc = spade.accept_workspace(B, R, wl["H"], wl["V"], device=dev)
+    temp = torch.full((B,), 0.8, dtype=torch.float32, device=dev)
+    top_p = torch.full((B,), 0.9, dtype=torch.float32, device=dev)
+    _, lm_bytes, _, _, _ = _work_bytes(wl)
+    flush_buf = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev) if lm_bytes < 2 * L2_BYTES else None
+    stream = torch.cuda.current_stream()
+    res = {"workload": wl["spec"].name, "launches": launches,
+           "timing": "median of CUDA-event times per launch", "top_p": 0.9, "temperature": 0.8}
+    for name, t, p in (("plain", None, None), ("temperature", temp, None), ("top_p", None, top_p),
+                       ("temperature_top_p", temp, top_p)):
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(launches)]
+        for i in range(3 + launches):
+            if i == 1:
+                torch.cuda.synchronize()
+                _head_start(2.0)
+            if flush_buf is not None:
+                flush_buf.zero_()
+            e = evs[i - 3] if i >= 3 else None
+            if e:
+                e[0].record(stream)
+            spade.spade_verify_accept_sampling(wl["hidden"], wl["w_lm"], wl["draft_tokens"], wl["draft_probs"],
+                                               wl["uniforms"], wl["mode"], wl["cu_q"], wl["n_draft"], acc, tok,
+                                               workspace=ws_acc, status=status, temperature=t, top_p=p)
+            if e:
+                e[1].record(stream)
+        torch.cuda.synchronize()
+        res[name + "_us"] = statistics.median(e[0].elapsed_time(e[1]) * 1e3 for e in evs)
+    if int(status.item()) & ~spade.DEV_FALLBACK:
+        raise RuntimeError(f"device status {int(status.item())} in the sampling report")
     return res
 
 
@@ -738,6 +782,8 @@ def main():
                     help="skip the device timing of the suite's other workloads")
     ap.add_argument("--per-workload-steps", type=int, default=20)
     ap.add_argument("--no-loop", action="store_true", help="skip the decoding-loop report")
+    ap.add_argument("--no-sampling", action="store_true",
+                    help="skip the timing of the temperature / top-p accept launches")
     ap.add_argument("--separate-commit", action="store_true",
                     help="run the KV commit as its own launch instead of inside the LM-head kernel")
     args = ap.parse_args()
