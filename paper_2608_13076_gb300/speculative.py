@@ -30,7 +30,7 @@ from dataclasses import dataclass
 import torch
 
 from . import (accept_workspace, attn_workspace, qkv_workspace, spade_verify_accept_commit,
-               spade_verify_attention, spade_verify_qkv_rope, status_tensor)
+               spade_verify_accept_sampling, spade_verify_attention, spade_verify_qkv_rope, status_tensor)
 
 GREEDY = 0
 STOCHASTIC = 1
@@ -84,10 +84,12 @@ class ToyVerifier:
                               workspace=qkv_workspace(x.shape[0], self.cfg.Hq, self.cfg.Hkv, self.cfg.D,
                                                       device=self.device), status=self.status)
 
-    def verify(self, tokens, kd, cu_q, drafts, draft_probs, uniforms, mode, max_k):
+    def verify(self, tokens, kd, cu_q, drafts, draft_probs, uniforms, mode, max_k, temperature=None, top_p=None):
         """One verify call over the blocks (row cu_q[b] + i holds token i of sequence b's
         block, position ctx_b + i): returns (accepted_len, next_token); the cache and ctx
-        are committed (accepted slots kept, rejected ones cleared, ctx += a + 1)."""
+        are committed (accepted slots kept, rejected ones cleared, ctx += a + 1).  With
+        ``temperature`` / ``top_p`` ([B] float32) the verifier's p is softmax(l / T) cut to
+        its nucleus."""
         c = self.cfg
         R = tokens.numel()
         x = self.emb[tokens].contiguous()
@@ -103,9 +105,15 @@ class ToyVerifier:
         acc = torch.empty(self.B, dtype=torch.int32, device=self.device)
         tok = torch.empty_like(acc)
         wsa = accept_workspace(self.B, R, c.H, c.V, device=self.device)
-        spade_verify_accept_commit(hidden.contiguous(), self.w_lm, drafts, draft_probs, uniforms, mode, cu_q, kd,
-                                   acc, tok, self.k_cache, self.v_cache, self.ctx, workspace=wsa,
-                                   status=self.status)
+        if temperature is None and top_p is None:
+            spade_verify_accept_commit(hidden.contiguous(), self.w_lm, drafts, draft_probs, uniforms, mode, cu_q,
+                                       kd, acc, tok, self.k_cache, self.v_cache, self.ctx, workspace=wsa,
+                                       status=self.status)
+        else:
+            spade_verify_accept_sampling(hidden.contiguous(), self.w_lm, drafts, draft_probs, uniforms, mode, cu_q,
+                                         kd, acc, tok, workspace=wsa, status=self.status, temperature=temperature,
+                                         top_p=top_p, k_cache=self.k_cache, v_cache=self.v_cache,
+                                         ctx_lens=self.ctx)
         self.last_hidden = hidden
         return acc, tok
 
@@ -121,12 +129,14 @@ class LoopResult:
 
 
 def speculative_decode(ver: ToyVerifier, prompts, d: int, max_new: int, mode: int = GREEDY, seed: int = 0,
-                       eos: int | None = None, record_margins: bool = False) -> LoopResult:
+                       eos: int | None = None, record_margins: bool = False, temperature: float | None = None,
+                       top_p: float | None = None) -> LoopResult:
     """Algorithm 1 for a batch of prompts (each at least 2 tokens): rounds of d drafts and one
     verifier call, until every sequence has max_new tokens or has emitted `eos` (default
     V - 1).  d = 0 is plain decoding with the verifier alone.  Stochastic mode draws the
     drafts from q = softmax(drafter logits) and the uniforms from a CPU generator seeded
-    with `seed`.  The verifier's cache must hold every prompt plus max_new * (d + 1) + d + 1
+    with `seed`; `temperature` and `top_p` (one value for every sequence) shape the
+    verifier's p.  The verifier's cache must hold every prompt plus max_new * (d + 1) + d + 1
     slots (sequences that are done keep stepping with the batch)."""
     B, cfg, dev = ver.B, ver.cfg, ver.device
     eos = cfg.V - 1 if eos is None else eos
@@ -145,6 +155,8 @@ def speculative_decode(ver: ToyVerifier, prompts, d: int, max_new: int, mode: in
     ver.ctx.copy_(lens.to(dev))
     last = torch.tensor([p[-1] for p in prompts], dtype=torch.long, device=dev)
     mode_t = torch.full((B,), mode, dtype=torch.int32, device=dev)
+    temp_t = None if temperature is None else torch.full((B,), temperature, dtype=torch.float32, device=dev)
+    top_p_t = None if top_p is None else torch.full((B,), top_p, dtype=torch.float32, device=dev)
     kd = torch.full((B,), d, dtype=torch.int32, device=dev)
     cu_q = (torch.arange(B + 1, dtype=torch.int32) * (d + 1)).to(dev)
     out = [[] for _ in range(B)]
@@ -169,7 +181,7 @@ def speculative_decode(ver: ToyVerifier, prompts, d: int, max_new: int, mode: in
             torch.empty(0, dtype=torch.int32, device=dev)
         qp = torch.stack(qrows, dim=1).reshape(B * d, cfg.V).contiguous() if (d and mode == STOCHASTIC) else None
         u = torch.rand(B * (d + 1), generator=gen).to(dev)
-        acc, tok = ver.verify(rows.reshape(-1), kd, cu_q, dr, qp, u, mode_t, d)
+        acc, tok = ver.verify(rows.reshape(-1), kd, cu_q, dr, qp, u, mode_t, d, temperature=temp_t, top_p=top_p_t)
         calls += 1
         acc_l, tok_l = acc.tolist(), tok.tolist()
         gap_l = None

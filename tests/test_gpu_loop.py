@@ -53,3 +53,28 @@ def test_stochastic_loop_runs_and_accepts(verifier):
         assert 1 <= len(t) <= MAX_NEW and all(0 <= x < V for x in t)
     assert 0 < res.accepted < res.drafted
     assert int(verifier.status.item()) & ~0x8 == 0
+
+
+def test_stochastic_with_a_one_token_nucleus_equals_greedy_decoding(verifier):
+    """top_p -> 0 leaves the verifier's argmax alone in its nucleus: a draft equal to it is
+    accepted (p_S(d) / q(d) = 1 / q(d) >= 1 > u), any other rejected (p_S(d) = 0), and the
+    residual max(0, p_S - q) has its mass on the argmax.  So stochastic speculative decoding
+    through the top-p path must reproduce plain greedy decoding token for token, whatever the
+    drafts and uniforms (a sequence may diverge only at a near tie, as above)."""
+    prompts = _prompts(verifier.cfg.V, seed=6)
+    ref = S.speculative_decode(verifier, prompts, d=0, max_new=MAX_NEW, record_margins=True)
+    for d in (1, 4):
+        res = S.speculative_decode(verifier, prompts, d=d, max_new=MAX_NEW, mode=S.STOCHASTIC, seed=10 + d,
+                                   top_p=1e-6, temperature=0.7)
+        identical = 0
+        for b in range(B):
+            a, r = res.tokens[b], ref.tokens[b]
+            i = next((j for j in range(min(len(a), len(r))) if a[j] != r[j]), None)
+            if i is None:
+                assert len(a) == len(r), (d, b)
+                identical += 1
+            else:
+                assert ref.margins[b][i] < 0.05, (d, b, i, ref.margins[b][i])
+        assert identical >= B - 1, (d, identical)
+        assert 0 < res.accepted < res.drafted  # drafts from q: some match the argmax, some not
+    assert int(verifier.status.item()) & ~0x8 == 0
