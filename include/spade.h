@@ -387,9 +387,9 @@ spade_status spade_kv_commit(void *k_cache, void *v_cache, int32_t *ctx_lens,
  * the pages a call touches are read; a touched entry outside [0, num_pages)
  * sets SPADE_DEV_BAD_INDEX (the attention reads zeros for it; the commit and
  * the QKV write skip that sequence).  Every other argument, and the result,
- * is that of the dense call of the same name.  The fused
- * spade_verify_accept_commit has no paged form: a paged step runs
- * spade_verify_accept and then spade_kv_commit_paged.
+ * is that of the dense call of the same name (spade_verify_accept_commit_paged:
+ * of spade_verify_accept_commit, the commit through the table), so a paged
+ * verify step is two launches like a dense one.
  */
 spade_status spade_verify_attention_paged(const void *q, const void *k_pool, const void *v_pool,
                                           const int32_t *block_table, const int32_t *ctx_lens,
@@ -405,6 +405,14 @@ spade_status spade_kv_commit_paged(void *k_pool, void *v_pool, const int32_t *bl
                                    const int32_t *n_draft, int32_t B, int32_t Hkv, int32_t D,
                                    int32_t page_size, int32_t num_pages, int32_t max_pages,
                                    int32_t *status, spade_stream_t stream);
+
+spade_status spade_verify_accept_commit_paged(
+    const void *hidden, const void *w_lm, const int32_t *draft_tokens, const float *draft_probs,
+    const float *uniforms, const int32_t *mode, const int32_t *cu_q, const int32_t *n_draft,
+    int32_t *accepted_len, int32_t *next_token, void *k_pool, void *v_pool, const int32_t *block_table,
+    int32_t *ctx_lens, int32_t B, int32_t R, int32_t H, int32_t V, int32_t Hkv, int32_t D, int32_t page_size,
+    int32_t num_pages, int32_t max_pages, void *workspace, size_t workspace_bytes, int32_t *status,
+    spade_stream_t stream);
 
 spade_status spade_verify_qkv_rope_paged(const void *x, const void *w_qkv, const int32_t *block_table,
                                          const int32_t *ctx_lens, const int32_t *n_draft,

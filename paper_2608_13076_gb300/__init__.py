@@ -28,7 +28,7 @@ __all__ = [
     "spade_verify_qkv_rope_paged",
     "spade_attn_workspace_size", "spade_accept_workspace_size", "spade_accept_launches",
     "spade_accept_stats_layout", "read_accept_stats", "spade_verify_accept_commit",
-    "spade_verify_accept_sampling", "spade_selftest_wait_timeout",
+    "spade_verify_accept_sampling", "spade_verify_accept_commit_paged", "spade_selftest_wait_timeout",
     "attn_workspace", "accept_workspace", "status_tensor", "check_status",
     "DEV_BAD_INDEX", "DEV_CAPACITY", "DEV_TIMEOUT", "DEV_FALLBACK",
 ]
@@ -102,6 +102,8 @@ def load():
     lib.spade_qkv_workspace_size.argtypes = [_i32] * 4
     lib.spade_verify_attention_paged.restype = _i32
     lib.spade_verify_attention_paged.argtypes = [_vp] * 9 + [_i32] * 9 + [_vp, _sz, _vp, _vp]
+    lib.spade_verify_accept_commit_paged.restype = _i32
+    lib.spade_verify_accept_commit_paged.argtypes = [_vp] * 14 + [_i32] * 9 + [_vp, _sz, _vp, _vp]
     lib.spade_kv_commit_paged.restype = _i32
     lib.spade_kv_commit_paged.argtypes = [_vp] * 6 + [_i32] * 6 + [_vp, _vp]
     lib.spade_verify_qkv_rope_paged.restype = _i32
@@ -380,6 +382,43 @@ def spade_verify_accept_sampling(hidden, w_lm, draft_tokens, draft_probs, unifor
         _ptr(temperature), _ptr(top_p), _ptr(cu_q), _ptr(n_draft), _ptr(accepted_len), _ptr(next_token),
         _ptr(k_cache), _ptr(v_cache), _ptr(ctx_lens), B, R, H, V, Hkv, D, cap, _ptr(workspace),
         workspace.numel(), _ptr(status), _stream(stream))
+    _check_rc(rc)
+    return accepted_len, next_token
+
+
+def spade_verify_accept_commit_paged(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
+                                     accepted_len, next_token, k_pool, v_pool, block_table, ctx_lens, *,
+                                     workspace, status, stream=None):
+    """spade_verify_accept_commit on paged caches: pools [num_pages, Hkv, page_size, D] and a
+    block table [B, max_pages] (see include/spade.h)."""
+    _need(hidden, "hidden", torch.bfloat16, 2)
+    _need(w_lm, "w_lm", torch.bfloat16, 2)
+    _need(uniforms, "uniforms", torch.float32, 1)
+    for t, n in ((draft_tokens, "draft_tokens"), (mode, "mode"), (cu_q, "cu_q"), (n_draft, "n_draft"),
+                 (accepted_len, "accepted_len"), (next_token, "next_token"), (status, "status"),
+                 (ctx_lens, "ctx_lens")):
+        _need(t, n, torch.int32, 1)
+    if draft_probs is not None:
+        _need(draft_probs, "draft_probs", torch.float32, 2)
+    _need(workspace, "workspace", torch.uint8, 1)
+    _need(k_pool, "k_pool", torch.bfloat16, 4)
+    _need(v_pool, "v_pool", torch.bfloat16, 4)
+    _need(block_table, "block_table", torch.int32, 2)
+    R, H = hidden.shape
+    V, H2 = w_lm.shape
+    B = n_draft.numel()
+    num_pages, Hkv, page_size, D = k_pool.shape
+    if H2 != H or uniforms.numel() != R or draft_tokens.numel() != R - B or cu_q.numel() != B + 1 \
+            or mode.numel() != B or accepted_len.numel() != B or next_token.numel() != B \
+            or tuple(v_pool.shape) != tuple(k_pool.shape) or ctx_lens.numel() != B or block_table.shape[0] != B:
+        raise ValueError("inconsistent accept/commit shapes")
+    if draft_probs is not None and tuple(draft_probs.shape) != (R - B, V):
+        raise ValueError("draft_probs must be [R - B, V]")
+    rc = load().spade_verify_accept_commit_paged(
+        _ptr(hidden), _ptr(w_lm), _ptr(draft_tokens), _ptr(draft_probs), _ptr(uniforms), _ptr(mode),
+        _ptr(cu_q), _ptr(n_draft), _ptr(accepted_len), _ptr(next_token), _ptr(k_pool), _ptr(v_pool),
+        _ptr(block_table), _ptr(ctx_lens), B, R, H, V, Hkv, D, page_size, num_pages, block_table.shape[1],
+        _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream))
     _check_rc(rc)
     return accepted_len, next_token
 

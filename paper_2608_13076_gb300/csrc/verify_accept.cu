@@ -109,6 +109,11 @@ struct Params {
   uint4 *kc, *vc;
   int32_t *ctx_lens;
   int Hkv, Dk, cap;
+  // Paged caches (block_table non-null): kc / vc are pools [num_pages, Hkv,
+  // page_size, Dk]; slot s of sequence b is row s % page_size of page
+  // block_table[b * max_pages + s / page_size]; cap = max_pages * page_size.
+  const int32_t *block_table;
+  int page_size, max_pages, num_pages;
   int kind;
   int pair;          // statistics pass on CTA pairs (cta_group::2), see phase A
   int nchunks;       // MMA N-chunks per tile (2 when Ncols > 256)
@@ -163,6 +168,22 @@ __device__ __forceinline__ void named_bar(int id, int threads) {
 __device__ __forceinline__ void block_sync() {
   __syncwarp();
   __syncthreads();
+}
+
+// barrier.red.or over `threads` threads of named barrier `id`: true on every
+// thread if `pred` holds on any.
+__device__ __forceinline__ bool bar_or(int id, int threads, bool pred) {
+  uint32_t r;
+  __syncwarp();
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "barrier.red.or.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(pred)), "r"(id), "r"(threads)
+      : "memory");
+  return r != 0;
 }
 
 __device__ __forceinline__ unsigned ld_relaxed(const unsigned *p) {
@@ -1318,9 +1339,30 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       const int per_head = (k - a) * vec;
       const int total = p.Hkv * per_head;
       const uint4 z = make_uint4(0, 0, 0, 0);
+      const int32_t *bt = p.block_table ? p.block_table + static_cast<int64_t>(b) * p.max_pages : nullptr;
+      if (bt) {
+        // Every page the rejected slots use must exist before anything is cleared.
+        bool bad_page = false;
+        for (int s2 = tid; s2 < k - a; s2 += 64) {
+          const int pg = bt[(lo + s2) / p.page_size];
+          bad_page |= pg < 0 || pg >= p.num_pages;
+        }
+        if (bar_or(2, 64, bad_page)) {
+          if (tid == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
+          continue;
+        }
+      }
       for (int e = tid; e < total; e += 64) {
         const int h = e / per_head;
-        const size_t off = ((static_cast<size_t>(b) * p.Hkv + h) * p.cap + lo) * vec + (e - h * per_head);
+        const int r = e - h * per_head;
+        size_t off;
+        if (bt) {
+          const int slot = lo + r / vec;
+          off = ((static_cast<size_t>(bt[slot / p.page_size]) * p.Hkv + h) * p.page_size + slot % p.page_size) * vec +
+                r % vec;
+        } else {
+          off = ((static_cast<size_t>(b) * p.Hkv + h) * p.cap + lo) * vec + r;
+        }
         p.kc[off] = z;
         p.vc[off] = z;
       }
@@ -2186,6 +2228,8 @@ struct CommitArgs {
   void *k_cache, *v_cache;
   int32_t *ctx_lens;
   int Hkv, D, cap;
+  const int32_t *block_table;  // paged pools when non-null
+  int page_size, max_pages, num_pages;
 };
 static spade_status verify_accept_impl(const void *hidden, const void *w_lm,
                                        const int32_t *draft_tokens, const float *draft_probs,
@@ -2246,6 +2290,10 @@ static spade_status verify_accept_impl(const void *hidden, const void *w_lm,
     p.Hkv = cm->Hkv;
     p.Dk = cm->D;
     p.cap = cm->cap;
+    p.block_table = cm->block_table;
+    p.page_size = cm->page_size;
+    p.max_pages = cm->max_pages;
+    p.num_pages = cm->num_pages;
   }
   set_region(p, ws, L.r1);
   Maps m;
@@ -2299,7 +2347,30 @@ extern "C" spade_status spade_verify_accept_commit(
   if (D % 8) return fail(SPADE_ERR_SHAPE, "spade_verify_accept_commit: D = %d must be a multiple of 8", D);
   if (!aligned(k_cache, 16) || !aligned(v_cache, 16))
     return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_commit: caches must be 16-byte aligned");
-  const accept::CommitArgs cm{k_cache, v_cache, ctx_lens, Hkv, D, cap};
+  const accept::CommitArgs cm{k_cache, v_cache, ctx_lens, Hkv, D, cap, nullptr, 0, 0, 0};
+  return accept::verify_accept_impl(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q,
+                                    n_draft, accepted_len, next_token, B, R, H, V, workspace,
+                                    workspace_bytes, status, stream, &cm);
+}
+
+extern "C" spade_status spade_verify_accept_commit_paged(
+    const void *hidden, const void *w_lm, const int32_t *draft_tokens, const float *draft_probs,
+    const float *uniforms, const int32_t *mode, const int32_t *cu_q, const int32_t *n_draft,
+    int32_t *accepted_len, int32_t *next_token, void *k_pool, void *v_pool, const int32_t *block_table,
+    int32_t *ctx_lens, int32_t B, int32_t R, int32_t H, int32_t V, int32_t Hkv, int32_t D, int32_t page_size,
+    int32_t num_pages, int32_t max_pages, void *workspace, size_t workspace_bytes, int32_t *status,
+    spade_stream_t stream) {
+  if (!k_pool || !v_pool || !block_table || !ctx_lens)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_commit_paged: null pool, table or ctx_lens pointer");
+  if (Hkv <= 0 || D <= 0 || page_size <= 0 || num_pages <= 0 || max_pages <= 0)
+    return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_commit_paged: non-positive size");
+  if (D % 8) return fail(SPADE_ERR_SHAPE, "spade_verify_accept_commit_paged: D = %d must be a multiple of 8", D);
+  if (static_cast<int64_t>(max_pages) * page_size >= (int64_t(1) << 31))
+    return fail(SPADE_ERR_CAPACITY, "max_pages * page_size exceeds 2^31");
+  if (!aligned(k_pool, 16) || !aligned(v_pool, 16))
+    return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_commit_paged: pools must be 16-byte aligned");
+  const accept::CommitArgs cm{k_pool, v_pool, ctx_lens, Hkv, D, max_pages * page_size, block_table,
+                              page_size, max_pages, num_pages};
   return accept::verify_accept_impl(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q,
                                     n_draft, accepted_len, next_token, B, R, H, V, workspace,
                                     workspace_bytes, status, stream, &cm);
@@ -2332,7 +2403,7 @@ extern "C" spade_status spade_verify_accept_sampling(
     if (!aligned(k_cache, 16) || !aligned(v_cache, 16))
       return fail(SPADE_ERR_INVALID_ARG, "spade_verify_accept_sampling: caches must be 16-byte aligned");
   }
-  const accept::CommitArgs cm{k_cache, v_cache, ctx_lens, Hkv, D, cap};
+  const accept::CommitArgs cm{k_cache, v_cache, ctx_lens, Hkv, D, cap, nullptr, 0, 0, 0};
   return accept::verify_accept_impl(hidden, w_lm, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
                                     accepted_len, next_token, B, R, H, V, workspace, workspace_bytes, status,
                                     stream, commit ? &cm : nullptr, temperature, top_p);

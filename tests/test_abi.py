@@ -73,6 +73,19 @@ def test_null_arguments_rejected_before_any_device_work(lib):
     assert rc == 1
 
 
+def test_paged_accept_commit_validation_before_device_work(lib):
+    p = ctypes.c_void_p(16)
+    base = [p] * 10  # hidden .. next_token
+    # Null table.
+    assert lib.spade_verify_accept_commit_paged(*base, p, p, None, p, 1, 5, 512, 1024, 8, 128, 64, 10, 4,
+                                                p, 1 << 20, p, None) == 1
+    # Non-positive page size; head dim not a multiple of 8.
+    assert lib.spade_verify_accept_commit_paged(*base, p, p, p, p, 1, 5, 512, 1024, 8, 128, 0, 10, 4,
+                                                p, 1 << 20, p, None) == 1
+    assert lib.spade_verify_accept_commit_paged(*base, p, p, p, p, 1, 5, 512, 1024, 8, 12, 64, 10, 4,
+                                                p, 1 << 20, p, None) == 2
+
+
 def test_sampling_entry_point_validation_before_device_work(lib):
     p = ctypes.c_void_p(16)
     base = [p] * 12  # hidden .. next_token, temperature and top_p given

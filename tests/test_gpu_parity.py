@@ -561,6 +561,67 @@ def test_paged_commit(dev, page):
     np.testing.assert_array_equal(parity.to_np(pg["v_pool"]), rv)
 
 
+@pytest.mark.parametrize("name,page", [("many_rows", 64), ("many_rows", 16), ("two_pass_mixed", 128)])
+def test_paged_accept_commit(dev, name, page):
+    """The fused accept + commit through a block table (one launch, or the two-pass path's
+    statistics pass committing): the decisions of the plain call, and the pools as the
+    oracle's paged commit leaves them (spare NaN pages untouched)."""
+    wl = W.make_workload(SMALL[name], device=dev, cache_pad=5)
+    pg = W.to_paged(wl, page, seed=8)
+    acc0, tok0, st0 = parity.gpu_accept(wl)
+    k0, v0 = parity.to_np(pg["k_pool"]), parity.to_np(pg["v_pool"])
+    B = wl["B"]
+    acc = torch.full((B,), -7, dtype=torch.int32, device=dev)
+    tok = torch.full((B,), -7, dtype=torch.int32, device=dev)
+    ctx = wl["ctx_lens"].clone()
+    st = spade.status_tensor(dev)
+    spade.spade_verify_accept_commit_paged(wl["hidden"], wl["w_lm"], wl["draft_tokens"], wl["draft_probs"],
+                                           wl["uniforms"], wl["mode"], wl["cu_q"], wl["n_draft"], acc, tok,
+                                           pg["k_pool"], pg["v_pool"], pg["block_table"], ctx,
+                                           workspace=spade.accept_workspace(B, wl["R"], wl["H"], wl["V"], device=dev),
+                                           status=st)
+    torch.cuda.synchronize()
+    assert int(st0.item()) & ~spade.DEV_FALLBACK == 0 and int(st.item()) & ~spade.DEV_FALLBACK == 0
+    assert torch.equal(acc, acc0) and torch.equal(tok, tok0)
+    rk, rv, rctx = O.kv_commit_paged(k0, v0, parity.to_np(pg["block_table"]), parity.to_np(wl["ctx_lens"]),
+                                     parity.to_np(acc), parity.to_np(wl["n_draft"]), page)
+    assert np.array_equal(parity.to_np(ctx), rctx)
+    np.testing.assert_array_equal(parity.to_np(pg["k_pool"]), rk)
+    np.testing.assert_array_equal(parity.to_np(pg["v_pool"]), rv)
+
+
+def test_paged_accept_commit_bad_page_leaves_the_sequence(dev):
+    """A table entry outside the pool on a page the commit would clear: SPADE_DEV_BAD_INDEX,
+    and that sequence's pages and context length stay as they were."""
+    wl = W.make_workload(SMALL["many_rows"], device=dev, cache_pad=5)
+    pg = W.to_paged(wl, 64, seed=8)
+    B = wl["B"]
+    ctx0 = parity.to_np(wl["ctx_lens"]).astype(np.int64)
+    kd = parity.to_np(wl["n_draft"]).astype(np.int64)
+    b = int(np.argmax(kd))  # a sequence with drafts, so some slot may be cleared
+    table = pg["block_table"].clone()
+    last = int((ctx0[b] + kd[b]) // 64)
+    table[b, last] = pg["num_pages"] + 5
+    k0 = pg["k_pool"].clone()
+    acc = torch.zeros(B, dtype=torch.int32, device=dev)
+    tok = torch.zeros(B, dtype=torch.int32, device=dev)
+    ctx = wl["ctx_lens"].clone()
+    st = spade.status_tensor(dev)
+    spade.spade_verify_accept_commit_paged(wl["hidden"], wl["w_lm"], wl["draft_tokens"], wl["draft_probs"],
+                                           wl["uniforms"], wl["mode"], wl["cu_q"], wl["n_draft"], acc, tok,
+                                           pg["k_pool"], pg["v_pool"], table, ctx,
+                                           workspace=spade.accept_workspace(B, wl["R"], wl["H"], wl["V"], device=dev),
+                                           status=st)
+    torch.cuda.synchronize()
+    a_b = int(acc[b])
+    if a_b < kd[b]:  # some slot of the bad page's sequence was to be cleared
+        assert int(st.item()) & spade.DEV_BAD_INDEX
+        assert int(ctx[b]) == ctx0[b]
+    pages_b = [int(x) for x in pg["block_table"][b].tolist()]
+    for pgi in pages_b:
+        assert torch.equal(pg["k_pool"][pgi].view(torch.int16), k0[pgi].view(torch.int16))
+
+
 def test_paged_qkv_rope(dev):
     spec = QKV_SMALL["qkv_gqa_d128"]
     wl = W.make_workload(spec, device=dev, cache_pad=40)
