@@ -268,10 +268,10 @@ spade_status spade_verify_accept_temperature(const void *hidden, const void *w_l
  *   fixes no truncation, this is the usual nucleus rule).  top_p[b] = 1 leaves
  *   p whole; a value outside (0, 1] is reported (SPADE_DEV_BAD_INDEX) and
  *   taken as 1.  Greedy sequences are unaffected.  tau_b is located by a
- *   four-round 32-bin search over integer keys of l / T (2^16 per unit of
- *   log-probability, from 31.5 below the row maximum; the last bit is not
- *   resolved), so tokens whose log-probability lies within 3.1e-5 below the
- *   boundary token's may also be in S_b, and tokens more than 31.5 below the
+ *   four-round 32-bin search over integer keys of l / T (2^15 per unit of
+ *   log-probability, from 31.5 below the row maximum), so tokens whose
+ *   log-probability lies within one key step (3.1e-5) below the boundary
+ *   token's may also be in S_b, and tokens more than 31.5 below the
  *   maximum (at most V e^-31.5 of p) never are.  Needs the one-launch path
  *   (spade_accept_launches == 1): SPADE_ERR_SHAPE otherwise.  The row
  *   statistics of spade_accept_stats_layout stay those of the whole p (the
