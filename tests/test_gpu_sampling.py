@@ -164,3 +164,20 @@ def test_top_p_needs_the_one_launch_path(dev):
     with pytest.raises(spade.SpadeError) as e:
         parity.gpu_accept_sampling(wl, top_p=tp)
     assert e.value.status == 2
+
+
+@pytest.mark.parametrize("T", [0.05, 5.0])
+def test_top_p_at_extreme_temperatures(dev, T):
+    """T = 0.05 scales the logits twentyfold (most tokens fall more than 31.5 below the row
+    maximum, outside the search's span), T = 5 flattens p (large nuclei): both against the oracle."""
+    wl = W.make_workload(TOPP["topp_resident"], device=dev)
+    B = wl["B"]
+    tp = _top_p(B, 11)
+    temp = np.full(B, T, dtype=np.float32)
+    acc, tok, st = parity.gpu_accept_sampling(wl, temperature=_dev_f32(temp, dev), top_p=_dev_f32(tp, dev))
+    torch.cuda.synchronize()
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0
+    ref = parity.oracle_accept_from_logits(wl, parity.oracle_logits(wl), temperature=temp, top_p=tp)
+    cmp = parity.compare_accept(acc, tok, ref)
+    assert cmp["mismatch_unflagged"] == 0, cmp
+    assert cmp["flagged"] < B, cmp  # something is left to compare
