@@ -208,8 +208,11 @@ spade_status spade_verify_attention_noalloc(const void *q, const void *k_cache,
  *   hidden        bf16 [R, H] row-major, 16-byte aligned, H % 8 == 0
  *   w_lm          bf16 [V, H] row-major (nn.Linear layout), 16-byte aligned
  *   draft_tokens  int32 [R - B]
- *   draft_probs   float32 [R - B, V] row-major, or NULL when no sequence is
- *                 stochastic
+ *   draft_probs   float32 [R - B, V] row-major, or NULL when no stochastic
+ *                 sequence has drafts (a stochastic sequence with k_b = 0
+ *                 draws its token from p and reads no q); a stochastic
+ *                 sequence with drafts and NULL draft_probs sets
+ *                 SPADE_DEV_BAD_INDEX and is verified greedily
  *   uniforms      float32 [R] in [0, 1)
  *   mode          int32 [B], 0 greedy / 1 stochastic
  *   cu_q, n_draft int32 [B+1], [B]

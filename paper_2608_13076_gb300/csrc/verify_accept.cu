@@ -1014,7 +1014,12 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   for (int b = tid; p.kind != kPresampled && b < p.B; b += kThreads) {
     const int md = s_md[b];
     if (md != 0 && md != 1 && c == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
-    s_stoch[b] = (md == 1) && p.draft_probs != nullptr;
+    // Stochastic: mode 1 with q for its drafts (a sequence without drafts
+    // samples its bonus token from p and needs none).  Drafts without q are
+    // reported and verified greedily.
+    const bool noq = md == 1 && p.draft_probs == nullptr && s_nd[b] > 0;
+    if (noq && c == 0) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
+    s_stoch[b] = md == 1 && !noq;
     if (p.top_p != nullptr && c == 0) {
       const float t = __ldg(p.top_p + b);
       if (!(t > 0.f && t <= 1.f)) atomicOr(p.status, SPADE_DEV_BAD_INDEX);
@@ -1042,7 +1047,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       for (int n0 = 0; n0 < p.R; n0 += 32) {
         const int n = n0 + lane;
         const int b = n < p.R ? s_seq[n] : -1;
-        const bool want = b >= 0 && s_md[b] == 1 && p.draft_probs != nullptr && seq_top_p(p, b) < 1.f &&
+        const bool want = b >= 0 && s_md[b] == 1 && (p.draft_probs != nullptr || s_nd[b] == 0) &&
+                          seq_top_p(p, b) < 1.f &&
                           isfinite(g_m[n]) && g_s[n] > 0.f;
         const unsigned bal = __ballot_sync(0xffffffffu, want);
         if (want) s_nl[base + __popc(bal & ((1u << lane) - 1u))] = n;

@@ -181,3 +181,42 @@ def test_top_p_at_extreme_temperatures(dev, T):
     cmp = parity.compare_accept(acc, tok, ref)
     assert cmp["mismatch_unflagged"] == 0, cmp
     assert cmp["flagged"] < B, cmp  # something is left to compare
+
+
+@pytest.mark.parametrize("opts", ["plain", "temperature", "top_p"])
+def test_stochastic_sequences_without_drafts(dev, opts):
+    """k_b = 0 everywhere: no draft rows, so draft_probs is empty (a null pointer), and every
+    stochastic sequence draws its token from p (Algorithm 1's bonus draw) -- not the argmax."""
+    spec = W.WorkloadSpec("stoch_k0", B=24, Hq=4, Hkv=4, D=64, H=256, V=5000, ctx=(1, 64), k=(0, 0),
+                          mode="mixed", seed=77)
+    wl = W.make_workload(spec, device=dev)
+    B = wl["B"]
+    assert wl["draft_probs"] is None or wl["draft_probs"].numel() == 0
+    temp = np.full(B, 1.3, dtype=np.float32) if opts == "temperature" else None
+    tp = np.full(B, 0.9, dtype=np.float32) if opts == "top_p" else None
+    acc, tok, st = parity.gpu_accept_sampling(wl, temperature=_dev_f32(temp, dev), top_p=_dev_f32(tp, dev))
+    torch.cuda.synchronize()
+    assert int(st.item()) & ~spade.DEV_FALLBACK == 0
+    logits = parity.oracle_logits(wl)
+    ref = parity.oracle_accept_from_logits(wl, logits, temperature=temp, top_p=tp)
+    cmp = parity.compare_accept(acc, tok, ref)
+    assert cmp["mismatch_unflagged"] == 0, cmp
+    # Flat logits: the draws are not the argmax for most stochastic sequences.
+    am = logits.argmax(-1)
+    t = parity.to_np(tok)
+    stoch = parity.to_np(wl["mode"]) == 1
+    assert np.sum(t[stoch] != am[stoch]) >= stoch.sum() // 2
+
+
+def test_stochastic_drafts_without_q_are_reported_and_verified_greedily(dev):
+    spec = W.WorkloadSpec("stoch_noq", B=8, Hq=4, Hkv=4, D=64, H=256, V=3000, ctx=(1, 64), k=(1, 5),
+                          mode="stochastic", match_prob=0.7, seed=78)
+    wl = W.make_workload(spec, device=dev)
+    acc, tok, st = parity.gpu_accept_sampling(dict(wl, draft_probs=None))
+    torch.cuda.synchronize()
+    assert int(st.item()) & spade.DEV_BAD_INDEX
+    greedy = dict(wl, mode=torch.zeros_like(wl["mode"]), draft_probs=None)
+    acc_g, tok_g, st_g = parity.gpu_accept_sampling(greedy)
+    torch.cuda.synchronize()
+    assert int(st_g.item()) == 0
+    assert torch.equal(acc, acc_g) and torch.equal(tok, tok_g)
