@@ -193,7 +193,7 @@ def _top2_margin(l):
 
 
 def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_draft,
-                  margin=1e-3, temperature=None, top_p=None):
+                  margin=1e-3, temperature=None, top_p=None, logit_rel_err=1.5e-5):
     """Accept/reject of every sequence, given its verifier logits.
 
     logits [R, V] (rows as in ``verify_attention``); draft_tokens [R-B] with
@@ -206,12 +206,19 @@ def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_dra
       flag_decision [B]  some decided position has top-2 logit margin (greedy)
                          or |u - p/q| (stochastic) below ``margin``;
       flag_sample [B]    the sampled token's u*Z lies within margin*r(x) of an
-                         edge of its CDF interval (stochastic only);
+                         edge of its CDF interval, or within the spread that
+                         logit errors give the cumulative mass (below; stochastic
+                         only);
       fallback [B]       residual had no mass, p used instead.
 
     ``temperature`` [B] (optional): the verifier samples from p = softmax(l / T_b)
     (the paper mentions sampling for diversity, Sec. III-A, without fixing it);
-    greedy decisions, which take the argmax, are unaffected.  ``top_p`` [B] (optional): p is
+    greedy decisions, which take the argmax, are unaffected.  ``logit_rel_err``: the
+    error a computed logit l may carry, as a fraction of max(1, |l|) (fp32 sums of a bf16
+    product over the hidden size); each term of p then moves by p_x times that error and
+    the cumulative mass at a draw's edges by about
+    sqrt(sum over the tokens with mass of (p_x * logit_rel_err * max(1, |l_x / T|))^2),
+    so a draw that close to an edge is flagged too.  ``top_p`` [B] (optional): p is
     then truncated to its nucleus (``nucleus``) for stochastic sequences; a nucleus boundary
     within the margin (1e-3 of mass, 1e-4 of log probability) at a deciding row flags the
     sequence's decision.
@@ -273,7 +280,14 @@ def verify_accept(logits, draft_tokens, draft_probs, uniforms, mode, cu_q, n_dra
             fallback[b] = fb
             x, m = inverse_cdf(r, Z, float(uniforms[r0 + k]))
             tok[b] = x
-            if m < margin:
+            # Two ways a draw sits on an edge: u*Z within margin * r(x) of one (a
+            # relative measure), or within the spread of the cumulative mass when
+            # each logit carries its own error (a peaked row moves its edges that
+            # far even when the drawn token's own interval is tiny).
+            lt = lr / t_b
+            terms = np.where(r > 0, p * logit_rel_err * np.maximum(1.0, np.abs(lt)), 0.0)
+            spread = float(np.sqrt(np.sum(terms ** 2)))
+            if m < margin or m * r[x] < spread:
                 flag_smp[b] = True
     return dict(accepted_len=acc, next_token=tok, flag_decision=flag_dec,
                 flag_sample=flag_smp, fallback=fallback)

@@ -201,6 +201,19 @@ def check_margin_worked_examples(o):
         assert abs(m - ex["margin"]) < 1e-9, (ex["why"], m)
 
 
+def check_sample_spread_worked_examples(o):
+    """The sampled-token flag from the spread logit errors give the cumulative mass: hand-derived
+    bonus draws (k = 0) that the relative edge margin alone does not flag, a control, a row
+    where only tokens with mass may count, and one where the logits' magnitude decides."""
+    g = _golden()["sample_spread"]
+    for ex in g["cases"]:
+        res = o.verify_accept(np.asarray([ex["logits"]], dtype=np.float64), [], np.zeros((0, len(ex["logits"]))),
+                              [ex["u"]], [1], [0, 1], [0], logit_rel_err=g["logit_rel_err"])
+        assert res["next_token"][0] == ex["next"], ex["about"]
+        assert bool(res["flag_sample"][0]) == ex["flag_sample"], ex["about"]
+        assert not res["flag_decision"][0], ex["about"]
+
+
 def check_residual_properties(o, seed=4):
     rng = np.random.default_rng(seed)
     for _ in range(50):
@@ -600,7 +613,7 @@ def check_top_p_output_law(o, n=40000, seed=15):
 ALL_CHECKS = [
     check_attention_worked_examples, check_attention_vs_sdpa, check_attention_special_cases,
     check_attention_gqa_mapping, check_logits_one_hot, check_acceptance_worked_examples,
-    check_margin_worked_examples, check_residual_properties, check_q_equals_p_accepts_all, check_strict_comparison,
+    check_margin_worked_examples, check_sample_spread_worked_examples, check_residual_properties, check_q_equals_p_accepts_all, check_strict_comparison,
     check_stochastic_output_law, check_progress_and_bounds, check_greedy_identity,
     check_kv_commit, check_rope_worked_examples, check_rope_vs_complex_rotation,
     check_rope_relative_position, check_qkv_projection_layout, check_kv_write_slots,

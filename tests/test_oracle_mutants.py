@@ -38,6 +38,11 @@ MUTANTS = {
                              "margin = min(T - lo, c[x] - T) / Z if r[x] > 0 else 0.0"),
     "sample_margin_always_zero": ("margin = min(T - lo, c[x] - T) / r[x] if r[x] > 0 else 0.0",
                                   "margin = 0.0"),
+    "sample_spread_dropped": ("if m < margin or m * r[x] < spread:", "if m < margin:"),
+    "sample_spread_over_every_token": ("terms = np.where(r > 0, p * logit_rel_err * np.maximum(1.0, np.abs(lt)), 0.0)",
+                                       "terms = logit_rel_err * np.maximum(1.0, np.abs(lt))"),
+    "sample_spread_without_magnitude": ("terms = np.where(r > 0, p * logit_rel_err * np.maximum(1.0, np.abs(lt)), 0.0)",
+                                        "terms = np.where(r > 0, p * logit_rel_err, 0.0)"),
     "flag_every_sequence": ("flag_dec = np.zeros(B, dtype=bool)", "flag_dec = np.ones(B, dtype=bool)"),
     "flag_every_sample": ("flag_smp = np.zeros(B, dtype=bool)", "flag_smp = np.ones(B, dtype=bool)"),
     "greedy_draft_rows_never_flag": ("                if _top2_margin(l) < margin:",
