@@ -730,7 +730,7 @@ def cpu_baseline(wl_cpu, acc_gpu, tok_gpu):
     par = {"sequences_checked": n, "of": B, "flagged": int(flagged), "mismatch_unflagged": int(mism),
            "mismatch_flagged": int(mism_flagged), "accepted_len_oracle": acc_oracle,
            "rule": "accepted length and next token bit-exact except at positions whose float64 top-2 logit "
-                   "gap, |u - p/q| or sampled-edge margin is below 1e-3 (flagged, counted here)"}
+                   "gap, |u - p/q| or sampled-edge margin is below 1e-3, or whose draw lies within the spread fp32 logit errors give the cumulative mass (flagged, counted here)"}
     return base, par
 
 
