@@ -187,3 +187,44 @@ def test_two_pass_accept_fuzz(dev, j):
     ref = parity.oracle_accept_from_logits(wl, parity.oracle_logits(wl), temperature=temp)
     cmp = parity.compare_accept(acc, tok, ref)
     assert cmp["mismatch_unflagged"] == 0, cmp
+
+
+def _wide_spec(i):
+    """Wide vocabularies (slices past the shared-memory staging: the register path of the
+    residual sums) and long contexts (units split across many CTAs)."""
+    g = np.random.default_rng(9700 + i)
+    D = int(g.choice([64, 128]))
+    Hkv = int(g.choice([1, 2, 4]))
+    G = int(g.choice([1, 4, 8]))
+    B = int(g.integers(1, 12))
+    k_hi = int(g.integers(0, 9))
+    c_hi = int(g.choice([4000, 12000, 20000]))
+    return W.WorkloadSpec(f"fuzz_wide{i}", B=B, Hq=Hkv * G, Hkv=Hkv, D=D, H=int(g.choice([128, 256])),
+                          V=int(g.integers(100000, 160000)), ctx=(int(g.integers(0, c_hi)), c_hi),
+                          k=(int(g.integers(0, k_hi + 1)), k_hi),
+                          mode=str(g.choice(["stochastic", "mixed"])), target_accept=0.7,
+                          logit_scale=float(g.choice([1.0, 4.0, 8.0])), seed=9800 + i)
+
+
+@pytest.mark.parametrize("i", range(10))
+def test_wide_fuzz(dev, i):
+    spec = _wide_spec(i)
+    wl = W.make_workload(spec, device=dev, cache_pad=5)
+    out, lse, st = parity.gpu_attention(wl)
+    B = wl["B"]
+    g = np.random.default_rng(9900 + i)
+    temp = g.uniform(0.5, 1.6, B).astype(np.float32) if g.random() < 0.5 else None
+    one_launch = spade.spade_accept_launches(B, wl["R"], wl["H"], wl["V"]) == 1
+    tp = g.uniform(0.5, 1.0, B).astype(np.float32) if (one_launch and g.random() < 0.6) else None
+    acc, tok, st2 = parity.gpu_accept_sampling(wl, temperature=None if temp is None else torch.from_numpy(temp).to(dev),
+                                               top_p=None if tp is None else torch.from_numpy(tp).to(dev))
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0 and int(st2.item()) & ~spade.DEV_FALLBACK == 0
+    R, Hq = wl["R"], wl["Hq"]
+    pairs = sorted({(int(r), int(h)) for r, h in zip(g.integers(0, R, 48), g.integers(0, Hq, 48))})
+    ref, _ = parity.oracle_attention(wl, rows=pairs)
+    n, bad, worst = parity.compare_attention(out, ref, rows=pairs)
+    assert bad == 0, (spec, worst)
+    ref_a = parity.oracle_accept_from_logits(wl, parity.oracle_logits(wl), temperature=temp, top_p=tp)
+    cmp = parity.compare_accept(acc, tok, ref_a)
+    assert cmp["mismatch_unflagged"] == 0, (spec, temp is not None, tp is not None, cmp)
