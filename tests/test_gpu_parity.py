@@ -706,3 +706,114 @@ def test_accept_temperature_row_stats(dev):
     scaled = logits / T.numpy().astype(np.float64)[seq][:, None]
     rs = parity.compare_row_stats(spade.read_accept_stats(ws, wl["B"], wl["R"], wl["H"], wl["V"]), scaled, wl)
     assert rs["max"] <= 1 and rs["lse"] <= 1 and rs["draft_logit"] <= 1 and rs["argmax_mismatch"] == 0, rs
+
+
+# ---------------------------------------------------------------------------
+# Invalid inputs: reported in the status word, confined to their sequence.
+
+def _greedy_wl(dev, seed=81):
+    spec = W.WorkloadSpec("invalid", B=6, Hq=8, Hkv=2, D=128, H=256, V=3000, ctx=(20, 200), k=(2, 5),
+                          mode="greedy", match_prob=0.8, seed=seed)
+    return W.make_workload(spec, device=dev, cache_pad=4)
+
+
+def test_accept_draft_id_out_of_range(dev):
+    """A draft id outside [0, V) is reported and rejected; every other decision is the oracle's."""
+    wl = _greedy_wl(dev)
+    b = 2
+    i0 = int(wl["cu_q"][b]) - b  # sequence b's first draft
+    bad = wl["draft_tokens"].clone()
+    bad[i0] = wl["V"] + 5
+    acc, tok, st = parity.gpu_accept(dict(wl, draft_tokens=bad))
+    torch.cuda.synchronize()
+    assert int(st.item()) & spade.DEV_BAD_INDEX
+    logits = parity.oracle_logits(wl)
+    # For the oracle the bad id is a token that is certainly rejected: one that is not the argmax.
+    stand_in = bad.clone()
+    r0 = int(wl["cu_q"][b])
+    stand_in[i0] = int(np.argmin(logits[r0]))
+    ref = O.verify_accept(logits, parity.to_np(stand_in), None, parity.to_np(wl["uniforms"]), parity.to_np(wl["mode"]),
+                          parity.to_np(wl["cu_q"]), parity.to_np(wl["n_draft"]))
+    assert int(acc[b]) == 0 and int(ref["accepted_len"][b]) == 0
+    cmp = parity.compare_accept(acc, tok, ref)
+    assert cmp["mismatch_unflagged"] == 0, cmp
+
+
+def test_accept_inconsistent_cu_q(dev):
+    """n_draft of the last sequence disagreeing with cu_q: reported, accepted_len 0 and
+    next_token -1 for it; the others as the oracle decides."""
+    wl = _greedy_wl(dev)
+    B = wl["B"]
+    kd_bad = wl["n_draft"].clone()
+    kd_bad[B - 1] += 1
+    acc, tok, st = parity.gpu_accept(dict(wl, n_draft=kd_bad))
+    torch.cuda.synchronize()
+    assert int(st.item()) & spade.DEV_BAD_INDEX
+    assert int(acc[B - 1]) == 0 and int(tok[B - 1]) == -1
+    ref = parity.oracle_accept(wl)
+    cmp = parity.compare_accept(acc[:B - 1], tok[:B - 1], {k: v[:B - 1] for k, v in ref.items()})
+    assert cmp["mismatch_unflagged"] == 0, cmp
+
+
+def test_accept_unknown_mode_is_reported_and_greedy(dev):
+    wl = W.make_workload(SMALL["d64_stochastic"], device=dev)
+    mode = wl["mode"].clone()
+    mode[0] = 2
+    acc, tok, st = parity.gpu_accept(dict(wl, mode=mode))
+    torch.cuda.synchronize()
+    assert int(st.item()) & spade.DEV_BAD_INDEX
+    as_greedy = mode.clone()
+    as_greedy[0] = 0
+    ref = O.verify_accept(parity.oracle_logits(wl), parity.to_np(wl["draft_tokens"]), parity.to_np(wl["draft_probs"]),
+                          parity.to_np(wl["uniforms"]), parity.to_np(as_greedy), parity.to_np(wl["cu_q"]),
+                          parity.to_np(wl["n_draft"]))
+    cmp = parity.compare_accept(acc, tok, ref)
+    assert cmp["mismatch_unflagged"] == 0, cmp
+
+
+def test_commit_accepted_beyond_drafts(dev):
+    """accepted_len > k_b: reported, that sequence's cache and context untouched; the others
+    committed as the oracle commits them."""
+    wl = _greedy_wl(dev)
+    B = wl["B"]
+    acc, tok, st = parity.gpu_accept(wl)
+    torch.cuda.synchronize()
+    bad = acc.clone()
+    bad[1] = int(wl["n_draft"][1]) + 1
+    k0, v0, ctx0 = (parity.to_np(wl[k]) for k in ("k_cache", "v_cache", "ctx_lens"))
+    kc, vc, ctx = wl["k_cache"].clone(), wl["v_cache"].clone(), wl["ctx_lens"].clone()
+    st2 = spade.status_tensor(dev)
+    spade.spade_kv_commit(kc, vc, ctx, bad, wl["n_draft"], status=st2)
+    torch.cuda.synchronize()
+    assert int(st2.item()) & spade.DEV_BAD_INDEX
+    good = [b for b in range(B) if b != 1]
+    rk, rv, rctx = O.kv_commit(k0[good], v0[good], ctx0[good], parity.to_np(acc)[good],
+                               parity.to_np(wl["n_draft"])[good])
+    np.testing.assert_array_equal(parity.to_np(kc)[good], rk)
+    np.testing.assert_array_equal(parity.to_np(vc)[good], rv)
+    np.testing.assert_array_equal(parity.to_np(ctx)[good], rctx)
+    assert torch.equal(kc[1], wl["k_cache"][1]) and torch.equal(vc[1], wl["v_cache"][1])
+    assert int(ctx[1]) == int(ctx0[1])
+
+
+def test_attention_sequence_beyond_capacity(dev):
+    """A sequence whose block does not fit its cache: SPADE_DEV_CAPACITY, its output rows left
+    as they were; every other row as the oracle computes it."""
+    wl = _greedy_wl(dev)
+    b = 3
+    ctx = wl["ctx_lens"].clone()
+    ctx[b] = wl["cap"]  # ctx + k + 1 > cap
+    out = torch.full_like(wl["q"], float("nan"))
+    st = spade.status_tensor(dev)
+    max_k = int(wl["n_draft"].max())
+    ws = spade.attn_workspace(wl["B"], wl["Hq"], wl["Hkv"], wl["D"], wl["cap"], max_k, device=dev)
+    spade.spade_verify_attention(wl["q"], wl["k_cache"], wl["v_cache"], ctx, wl["n_draft"], wl["cu_q"], out, None,
+                                 max_k=max_k, workspace=ws, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & spade.DEV_CAPACITY
+    r0, r1 = int(wl["cu_q"][b]), int(wl["cu_q"][b + 1])
+    assert torch.isnan(out[r0:r1].float()).all()
+    rows = [(r, h) for r in range(wl["R"]) if not r0 <= r < r1 for h in range(wl["Hq"])]
+    ref, _ = parity.oracle_attention(wl, rows=rows)
+    n, bad, worst = parity.compare_attention(out, ref, rows=rows)
+    assert bad == 0, worst
