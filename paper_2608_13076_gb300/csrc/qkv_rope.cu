@@ -274,36 +274,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(s_tmem, p.tmem_cols);
     tmem_relinquish();
   }
+  tc_fence_before();
+  __syncthreads();  // barriers and the tensor-memory allocation
+  tc_fence_after();
+  // Inputs written by earlier kernels in the stream are visible from here on.
   griddep_wait();
   griddep_launch_dependents();
-  // ---- row table: sequence and position of every verify row ---------------
-  for (int r = tid; r < p.R; r += kThreads) s_rseq[r] = -1;
-  __syncthreads();
-  for (int b = tid; b < p.B; b += kThreads) {
-    const int c = p.ctx_lens[b], k = p.n_draft[b];
-    const int q0 = p.cu_q[b], q1 = p.cu_q[b + 1];
-    int bad = 0;
-    if (c < 0 || k < 0 || k > p.max_k || q0 < 0 || q1 > p.R || q1 - q0 != k + 1) bad = SPADE_DEV_BAD_INDEX;
-    else if (static_cast<int64_t>(c) + k + 1 > p.cap) bad = SPADE_DEV_CAPACITY;
-    if (!bad && p.block_table) {
-      // Every page the block writes must exist.
-      for (int i = 0; i <= k; ++i) {
-        const int pg = p.block_table[static_cast<int64_t>(b) * p.max_pages + (c + i) / p.page_size];
-        if (pg < 0 || pg >= p.num_pages) bad = SPADE_DEV_BAD_INDEX;
-      }
-    }
-    if (bad) {
-      if (blockIdx.x == 0) atomicOr(p.status, bad);
-      continue;
-    }
-    for (int i = 0; i <= k; ++i) {
-      s_rseq[q0 + i] = b;
-      s_rpos[q0 + i] = c + i;
-    }
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
   const uint32_t tmem = *s_tmem;
   const uint32_t smem_base = smem_u32(smem);
   const int n0 = p.Ncols > 256 ? 256 : p.Ncols;  // first MMA N-chunk (and x box rows)
@@ -379,6 +355,34 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ===================== epilogue warps: drain, publish, reduce ==========
     const int et = tid - 64;         // 0..127
     const int q4 = warp & 3;         // tensor-memory lane quadrant this warp may access
+    // Row table: sequence and position of every verify row.  Only the tile
+    // reductions read it, so it is built here while the producer and the MMA
+    // warp already stream the first units.
+    for (int r = et; r < p.R; r += kEpiThreads) s_rseq[r] = -1;
+    epi_bar();
+    for (int b = et; b < p.B; b += kEpiThreads) {
+      const int c = p.ctx_lens[b], k = p.n_draft[b];
+      const int q0 = p.cu_q[b], q1 = p.cu_q[b + 1];
+      int bad = 0;
+      if (c < 0 || k < 0 || k > p.max_k || q0 < 0 || q1 > p.R || q1 - q0 != k + 1) bad = SPADE_DEV_BAD_INDEX;
+      else if (static_cast<int64_t>(c) + k + 1 > p.cap) bad = SPADE_DEV_CAPACITY;
+      if (!bad && p.block_table) {
+        // Every page the block writes must exist.
+        for (int i = 0; i <= k; ++i) {
+          const int pg = p.block_table[static_cast<int64_t>(b) * p.max_pages + (c + i) / p.page_size];
+          if (pg < 0 || pg >= p.num_pages) bad = SPADE_DEV_BAD_INDEX;
+        }
+      }
+      if (bad) {
+        if (blockIdx.x == 0) atomicOr(p.status, bad);
+        continue;
+      }
+      for (int i = 0; i <= k; ++i) {
+        s_rseq[q0 + i] = b;
+        s_rpos[q0 + i] = c + i;
+      }
+    }
+    epi_bar();
     bool expired = false;
     int seg = 0;
     for (int u = u0; u < u1; ++seg) {
