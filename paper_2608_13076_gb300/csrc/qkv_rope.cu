@@ -11,7 +11,10 @@
 //    rows on the MMA M side (128-row tiles: one head of dimension 128, or two
 //    of dimension 64, per tile) and the R verify rows on N.  At R = 72 the
 //    work is bound by streaming W from HBM (50 MB for the Llama-3-8B layer).
-//  * Stream-K over (tile, k-chunk) units: the units are laid end to end and
+//  * Stream-K over (tile, k-step) units, a k-step being KG k-chunks of 64
+//    (KG = 2 when the hidden size allows: W then arrives in 3-D boxes of
+//    128 rows x 256 contiguous bytes, which stream from HBM faster than
+//    128-byte rows; KG = 1 otherwise): the units are laid end to end and
 //    cut into one equal range per SM, so every SM streams the same share of W
 //    whatever the tile count.  A CTA's range covers pieces of one to three
 //    tiles ("segments"); each segment accumulates in one of two tensor-memory
@@ -63,7 +66,9 @@ struct Params {
   int B, R, H, Hq, Hkv, D, cap, max_k;
   int tiles;    // (Hq + 2 Hkv) D / 128
   int KC;       // k-chunks (ceil(H / 64))
-  int units;    // tiles * KC
+  int KG;       // k-chunks per unit (1 or 2; 2 only when H is a multiple of 128)
+  int KS;       // units per tile (ceil(KC / KG))
+  int units;    // tiles * KS
   int num_ctas;
   int Ncols;    // R rounded up to 16: MMA N (two MMAs of <= 256 when above 256)
   int stages;   // ring depth
@@ -80,9 +85,9 @@ struct Params {
 struct Layout {
   int stage_bytes, ring, rseq, rpos, bars, misc, freq, total;
 };
-__host__ __device__ inline Layout layout(int Ncols, int stages) {
+__host__ __device__ inline Layout layout(int Ncols, int stages, int KG) {
   Layout L;
-  L.stage_bytes = kWBytes + Ncols * 128;
+  L.stage_bytes = KG * (kWBytes + Ncols * 128);  // KG W chunks, then KG x chunks
   L.ring = 0;
   L.rseq = stages * L.stage_bytes;   // int32 [kMaxR]: sequence of each row (-1: skip)
   L.rpos = L.rseq + kMaxR * 4;       // int32 [kMaxR]: position of each row
@@ -229,10 +234,11 @@ __device__ __noinline__ void reduce_tile(const Params &p, const int32_t *s_rseq,
 
 __global__ void __launch_bounds__(kThreads, 1)
     qkv_rope_kernel(const __grid_constant__ Params p, const __grid_constant__ CUtensorMap tm_w,
-                    const __grid_constant__ CUtensorMap tm_x0, const __grid_constant__ CUtensorMap tm_x1) {
+                    const __grid_constant__ CUtensorMap tm_x0, const __grid_constant__ CUtensorMap tm_x1,
+                    const __grid_constant__ CUtensorMap tm_w3) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-  const Layout L = layout(p.Ncols, p.stages);
+  const Layout L = layout(p.Ncols, p.stages, p.KG);
   int32_t *s_rseq = reinterpret_cast<int32_t *>(smem + L.rseq);
   int32_t *s_rpos = reinterpret_cast<int32_t *>(smem + L.rpos);
   uint64_t *bar_full = reinterpret_cast<uint64_t *>(smem + L.bars);
@@ -255,7 +261,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) { *s_abort = 0; s_fin[0] = -1; }
   for (int j = tid; j < 64; j += kThreads) s_freq[j] = p.inv_freq[j];
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&tm_w);
+    tma_prefetch_desc(p.KG > 1 ? &tm_w3 : &tm_w);
     tma_prefetch_desc(&tm_x0);
     if (p.Ncols > 256) tma_prefetch_desc(&tm_x1);
   } else if (warp == 1) {
@@ -290,7 +296,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       const uint64_t pol_w = l2_policy_evict_first();  // W streams once
       const uint64_t pol_x = l2_policy_evict_last();   // x is re-read for every unit
-      const uint32_t bytes = kWBytes + p.Ncols * 128;
+      const uint32_t xbytes = p.Ncols * 128;  // x rows of one k-chunk
       bool expired = false;
       int issued = 0;
       for (int u = u0, i = 0; u < u1; ++u, ++i) {
@@ -300,11 +306,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (*s_abort) break;
         issued = i + 1;
         uint8_t *stage = smem + L.ring + st * L.stage_bytes;
-        const int t = u / p.KC, kx = (u - t * p.KC) * kKChunk;
-        mbar_arrive_expect_tx(&bar_full[st], bytes);
-        tma_load_2d(stage, &tm_w, kx, t * kTileM, &bar_full[st], pol_w);
-        tma_load_2d(stage + kWBytes, &tm_x0, kx, 0, &bar_full[st], pol_x);
-        if (n1) tma_load_2d(stage + kWBytes + n0 * 128, &tm_x1, kx, n0, &bar_full[st], pol_x);
+        const int t = u / p.KS, c0 = (u - t * p.KS) * p.KG;
+        const int nch = min(p.KG, p.KC - c0);  // == KG whenever KG > 1 (H a multiple of 64 KG)
+        mbar_arrive_expect_tx(&bar_full[st], nch * (kWBytes + xbytes));
+        if (p.KG > 1)
+          tma_load_3d(stage, &tm_w3, 0, t * kTileM, c0, &bar_full[st], pol_w);  // KG chunks, 16 KB apart
+        else
+          tma_load_2d(stage, &tm_w, c0 * kKChunk, t * kTileM, &bar_full[st], pol_w);
+        uint8_t *xs = stage + p.KG * kWBytes;
+        for (int j = 0; j < nch; ++j) {
+          tma_load_2d(xs + j * xbytes, &tm_x0, (c0 + j) * kKChunk, 0, &bar_full[st], pol_x);
+          if (n1) tma_load_2d(xs + j * xbytes + n0 * 128, &tm_x1, (c0 + j) * kKChunk, n0, &bar_full[st], pol_x);
+        }
       }
       if (expired || *s_abort) {
         atomicOr(p.status, SPADE_DEV_TIMEOUT);
@@ -321,8 +334,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool expired = false;
       int i = 0, seg = 0;
       for (int u = u0; u < u1; ++seg) {
-        const int t = u / p.KC;
-        const int se = min(u1, (t + 1) * p.KC);
+        const int t = u / p.KS;
+        const int se = min(u1, (t + 1) * p.KS);
         const int buf = seg % p.nbuf, use = seg / p.nbuf;
         // The buffer's previous segment has been drained by the epilogue warps.
         if (use > 0 && !mbar_wait(&acc_empty[buf], (use - 1) & 1, s_abort)) expired = true;
@@ -334,15 +347,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!mbar_wait(&bar_full[st], ph, s_abort)) expired = true;
           tc_fence_after();
           if (!*s_abort) {
-            const uint32_t a = smem_base + L.ring + st * L.stage_bytes;
-            const uint32_t b = a + kWBytes;
+            const uint32_t a0 = smem_base + L.ring + st * L.stage_bytes;
+            const int nch = min(p.KG, p.KC - (u - t * p.KS) * p.KG);
+            for (int j = 0; j < nch; ++j) {
+              const uint32_t a = a0 + j * kWBytes;
+              const uint32_t b = a0 + p.KG * kWBytes + j * p.Ncols * 128;
 #pragma unroll
-            for (int kk = 0; kk < kKChunk / 16; ++kk) {
-              const uint32_t acc = (u > us || kk > 0) ? 1u : 0u;
-              tc_mma_f16(acc_addr, smem_desc_sw128(a + kk * 32), smem_desc_sw128(b + kk * 32), idesc0, acc);
-              if (n1)
-                tc_mma_f16(acc_addr + 256, smem_desc_sw128(a + kk * 32),
-                           smem_desc_sw128(b + n0 * 128 + kk * 32), idesc1, acc);
+              for (int kk = 0; kk < kKChunk / 16; ++kk) {
+                const uint32_t acc = (u > us || j > 0 || kk > 0) ? 1u : 0u;
+                tc_mma_f16(acc_addr, smem_desc_sw128(a + kk * 32), smem_desc_sw128(b + kk * 32), idesc0, acc);
+                if (n1)
+                  tc_mma_f16(acc_addr + 256, smem_desc_sw128(a + kk * 32),
+                             smem_desc_sw128(b + n0 * 128 + kk * 32), idesc1, acc);
+              }
             }
           }
           tc_commit(&bar_empty[st]);
@@ -386,8 +403,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool expired = false;
     int seg = 0;
     for (int u = u0; u < u1; ++seg) {
-      const int t = u / p.KC;
-      const int se = min(u1, (t + 1) * p.KC);
+      const int t = u / p.KS;
+      const int se = min(u1, (t + 1) * p.KS);
       const int buf = seg % p.nbuf, use = seg / p.nbuf;
       if (!mbar_wait(&acc_full[buf], use & 1, s_abort)) expired = true;
       tc_fence_after();
@@ -405,8 +422,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty[buf]);
       // Publish; the CTA that completes the tile reduces it.
-      const int c_first = unit_owner(p.units, p.num_ctas, t * p.KC);
-      const int c_last = unit_owner(p.units, p.num_ctas, (t + 1) * p.KC - 1);
+      const int c_first = unit_owner(p.units, p.num_ctas, t * p.KS);
+      const int c_last = unit_owner(p.units, p.num_ctas, (t + 1) * p.KS - 1);
       const int nparts = c_last - c_first + 1;
       epi_bar();
       if (et == 0) *s_last = nparts == 1 ? 1 : arrive_tile(&p.counters[t], nparts);
@@ -514,19 +531,25 @@ static spade_status qkv_rope_impl(const void *x, const void *w_qkv, const int32_
   p.num_pages = pg ? pg->num_pages : 0;
   p.tiles = tiles;
   p.KC = (H + kKChunk - 1) / kKChunk;
-  p.units = tiles * p.KC;
-  p.num_ctas = p.units < sms ? p.units : sms;
   p.Ncols = (R + 15) / 16 * 16;
   p.buf_cols = 32;
   while (p.buf_cols < static_cast<uint32_t>(p.Ncols)) p.buf_cols *= 2;
   p.nbuf = p.buf_cols * 2 <= 512 ? 2 : 1;
   p.tmem_cols = p.buf_cols * p.nbuf;
   for (int j = 0; j < D / 2; ++j) p.inv_freq[j] = static_cast<float>(pow(static_cast<double>(rope_theta), -2.0 * j / D));
-  const int stage = kWBytes + p.Ncols * 128;
-  p.stages = (kSmemBudget - layout(p.Ncols, 0).total) / stage;
+  // Two k-chunks per unit when H allows the 3-D view and the ring still
+  // holds three stages; otherwise one.
+  p.KG = 1;
+  if (H % (2 * kKChunk) == 0 &&
+      (kSmemBudget - layout(p.Ncols, 0, 2).total) / layout(p.Ncols, 0, 2).stage_bytes >= 3)
+    p.KG = 2;
+  p.KS = (p.KC + p.KG - 1) / p.KG;
+  p.units = tiles * p.KS;
+  p.num_ctas = p.units < sms ? p.units : sms;
+  p.stages = (kSmemBudget - layout(p.Ncols, 0, p.KG).total) / layout(p.Ncols, 0, p.KG).stage_bytes;
   if (p.stages > kMaxStages) p.stages = kMaxStages;
   if (p.stages < 2) return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
-  const int smem = layout(p.Ncols, p.stages).total;
+  const int smem = layout(p.Ncols, p.stages, p.KG).total;
   static bool configured = false;
   if (!configured) {
     // The plan above never exceeds kSmemBudget (alignment slack included).
@@ -534,14 +557,20 @@ static spade_status qkv_rope_impl(const void *x, const void *w_qkv, const int32_
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(qkv_rope)");
     configured = true;
   }
-  CUtensorMap tw, tx0, tx1;
+  CUtensorMap tw, tx0, tx1, tw3;
   const int n0 = p.Ncols > 256 ? 256 : p.Ncols;
   const int n1 = p.Ncols - n0;
-  if (!encode_tmap_bf16_sw128(&tw, w_qkv, H, static_cast<uint64_t>(Hq + 2 * Hkv) * D, static_cast<uint64_t>(H) * 2,
-                              kKChunk, kTileM) ||
+  const uint64_t wrows = static_cast<uint64_t>(Hq + 2 * Hkv) * D;
+  if (!encode_tmap_bf16_sw128(&tw, w_qkv, H, wrows, static_cast<uint64_t>(H) * 2, kKChunk, kTileM) ||
       !encode_tmap_bf16_sw128(&tx0, x, H, R, static_cast<uint64_t>(H) * 2, kKChunk, n0) ||
       !encode_tmap_bf16_sw128(&tx1, x, H, R, static_cast<uint64_t>(H) * 2, kKChunk, n1 ? n1 : 16))
     return SPADE_ERR_CUDA;
+  if (p.KG > 1) {
+    if (!encode_tmap_rows_by_slab(&tw3, w_qkv, wrows, static_cast<uint32_t>(H), kTileM, static_cast<uint32_t>(p.KG)))
+      return SPADE_ERR_CUDA;
+  } else {
+    tw3 = tw;  // unused
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.num_ctas);
   cfg.blockDim = dim3(kThreads);
@@ -552,7 +581,7 @@ static spade_status qkv_rope_impl(const void *x, const void *w_qkv, const int32_
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, qkv_rope_kernel, p, tw, tx0, tx1);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, qkv_rope_kernel, p, tw, tx0, tx1, tw3);
   if (e != cudaSuccess) return cuda_fail(e, "qkv_rope launch");
   return SPADE_OK;
 }
