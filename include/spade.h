@@ -102,11 +102,15 @@ typedef enum {
  *   workspace   device scratch of at least spade_qkv_workspace_size(R, Hq, Hkv, D)
  *               bytes, 256-byte aligned, ZEROED ONCE by the caller after
  *               allocation; every call that completes leaves its counters
- *               zeroed again.  Calls that share a workspace must be ordered.
+ *               zeroed again (a call that reported SPADE_DEV_TIMEOUT may not:
+ *               zero the workspace again before the next one).  Calls that
+ *               share a workspace must be ordered.
  * Every pointer is a 16-byte aligned device pointer.  The contraction is split
  * over every SM; the split parts' fp32 sums meet in the workspace and are
- * added in a fixed order, so results do not depend on timing.  Launched with
- * programmatic dependent launch.
+ * added in a fixed order, so results do not depend on timing.  The kernel
+ * keeps every block of the grid resident at once (cooperative launch, with
+ * programmatic dependent launch): the CTAs that finish a split tile wait,
+ * bounded, for the other CTAs' partial sums.
  */
 spade_status spade_verify_qkv_rope(const void *x, const void *w_qkv, const int32_t *ctx_lens,
                                    const int32_t *n_draft, const int32_t *cu_q, void *q_out,

@@ -11,17 +11,22 @@
 //    rows on the MMA M side (128-row tiles: one head of dimension 128, or two
 //    of dimension 64, per tile) and the R verify rows on N.  At R = 72 the
 //    work is bound by streaming W from HBM (50 MB for the Llama-3-8B layer).
-//  * Stream-K over (tile, k-step) units, a k-step being KG k-chunks of 64
-//    (KG = 2 when the hidden size allows: W then arrives in 3-D boxes of
-//    128 rows x 256 contiguous bytes, which stream from HBM faster than
-//    128-byte rows; KG = 1 otherwise): the units are laid end to end and
-//    cut into one equal range per SM, so every SM streams the same share of W
-//    whatever the tile count.  A CTA's range covers pieces of one to three
+//  * Stream-K over (tile, k-chunk of 64) units: the units are laid end to end
+//    and cut into one equal range per SM, so every SM streams the same share
+//    of W whatever the tile count.  A ring stage holds up to KG = 2 chunks of
+//    one tile (two consecutive chunks of the range in the same tile arrive as
+//    one 3-D box of 128 rows x 256 contiguous bytes; KG = 1 when H is not a
+//    multiple of 64).  A CTA's range covers pieces of one to three
 //    tiles ("segments"); each segment accumulates in one of two tensor-memory
 //    buffers (the next segment's MMAs start while the last one is drained),
-//    and its fp32 partial goes to the CTA's own workspace slot.  The CTA that
-//    completes a tile last sums the tile's partials in CTA order -- the same
-//    order every call, so results do not depend on arrival order -- rotates
+//    and its fp32 partial goes to the CTA's own workspace slot.  A tile
+//    computed by one CTA is finished by that CTA.  A tile split over several
+//    CTAs is finished by the CTA whose part arrives last, or, when the grid
+//    has CTAs to spare (two or more per tile), after every CTA's stream in
+//    row slabs spread over the whole grid (the launch is cooperative, so
+//    every CTA is resident and a slab's CTA may wait for the tile's parts).
+//    Either way the parts are summed in CTA order -- the same order every
+//    call, so results do not depend on arrival order -- and the finisher rotates
 //    query and key pairs (dimension j with j + D/2, angle pos *
 //    theta^(-2j/D), pos = ctx_b + i) and stores bf16: queries to q_out, keys
 //    and values to cache slot ctx_b + i of their sequence (or, for a paged
@@ -62,17 +67,17 @@ struct Params {
   __nv_bfloat16 *v_cache;
   int32_t *status;
   float *partials;         // [num_ctas + tiles slots][Ncols][128] fp32 (workspace)
-  int32_t *counters;       // [tiles], zero between calls (workspace)
+  int32_t *counters;       // [2][tiles]: parts published, slabs done; zero between calls (workspace)
   int B, R, H, Hq, Hkv, D, cap, max_k;
   int tiles;    // (Hq + 2 Hkv) D / 128
   int KC;       // k-chunks (ceil(H / 64))
-  int KG;       // k-chunks per unit (1 or 2; 2 only when H is a multiple of 128)
-  int KS;       // units per tile (ceil(KC / KG))
-  int units;    // tiles * KS
+  int KG;       // k-chunks per ring stage at most (1 or 2; 2 only when H is a multiple of 64)
+  int units;    // tiles * KC
   int num_ctas;
   int Ncols;    // R rounded up to 16: MMA N (two MMAs of <= 256 when above 256)
   int stages;   // ring depth
   int nbuf;     // accumulator buffers (2 when two fit in tensor memory)
+  int slabs;    // row slabs per split tile in the final reduction
   uint32_t buf_cols, tmem_cols;
   float inv_freq[64];  // theta^(-2j/D), j < D/2, rounded from double on the host
   // Paged caches (block_table null: dense [B, Hkv, cap, D]): pools
@@ -107,13 +112,20 @@ __device__ inline int unit_owner(int units, int n, int u) {
   return static_cast<int>((static_cast<int64_t>(u + 1) * n + units - 1) / units - 1);
 }
 
-// Arrival of one partial at its tile's counter (one thread, after a barrier
-// that orders the partial's stores before it): release publishes this CTA's
-// partial; for the last arrival, acquire makes every other one visible.
-__device__ __forceinline__ bool arrive_tile(int32_t *counter, int nparts) {
+// Publication of one partial at its tile's counter (one thread, after a
+// barrier that orders the partial's stores before it).
+__device__ __forceinline__ void publish_part(int32_t *counter) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(counter) : "memory");
+}
+__device__ __forceinline__ int load_acquire(const int32_t *a) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ int add_acq_rel(int32_t *a, int v) {
   int old;
-  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;" : "=r"(old) : "l"(counter) : "memory");
-  return old == nparts - 1;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(a), "r"(v) : "memory");
+  return old;
 }
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory"); }
@@ -132,17 +144,21 @@ __device__ __forceinline__ void rope_angle(int pos, float f, float *sn, float *c
   __sincosf(r + e, sn, cs);
 }
 
-// The reduction of tile t once every part has been published: for each verify
-// row and each 4 consecutive dimension pairs of a head (thread th of nth takes
-// items th, th + nth, ...), the sum of the partials of CTAs c_first ..
-// c_first + nparts - 1 in that order, the rotation of query and key pairs and
-// the bf16 stores (q_out, or the cache slot ctx_b + i of the row's sequence).
+// The reduction of verify rows [r0, r1) of tile t once every part has been
+// published: for each row and each 4 consecutive dimension pairs of a head
+// (thread th of nth takes items th, th + nth, ...), the sum of the partials
+// of CTAs c_first .. c_first + nparts - 1 in that order, the rotation of
+// query and key pairs and the bf16 stores (q_out, or the cache slot ctx_b + i
+// of the row's sequence).  Each thread takes kIB items at a time and issues
+// the loads of every item and kPB parts before using any (the reduction is
+// bound by L2 latency, so the rounds of loads are what it costs).
+template <int kIB, int kPB>
 __device__ __noinline__ void reduce_tile(const Params &p, const int32_t *s_rseq, const int32_t *s_rpos,
-                                         const float *s_freq, int t, int c_first, int nparts, int th,
-                                         int nth) {
+                                         const float *s_freq, int t, int c_first, int nparts, int r0,
+                                         int r1, int th, int nth) {
   // Every field used below in a local: the stores through dst could alias
   // the parameter block as far as the compiler knows, and it would reload them.
-  const int D = p.D, R = p.R, Hq = p.Hq, Hkv = p.Hkv, cap = p.cap, Ncols = p.Ncols;
+  const int D = p.D, Hq = p.Hq, Hkv = p.Hkv, cap = p.cap, Ncols = p.Ncols;
   const int max_pages = p.max_pages, page_size = p.page_size;
   const int32_t *block_table = p.block_table;
   __nv_bfloat16 *q_out = p.q_out, *k_cache = p.k_cache, *v_cache = p.v_cache;
@@ -154,17 +170,14 @@ __device__ __noinline__ void reduce_tile(const Params &p, const int32_t *s_rseq,
   constexpr int kQuads = kTileM / 8;
   const float *base = partials + static_cast<size_t>(c_first + t) * Ncols * kTileM;
   const size_t slot = static_cast<size_t>(Ncols) * kTileM;
-  // Each thread takes kIB items at a time and issues the loads of every item
-  // and two parts before using any: the reduction is bound by L2 latency.
-  constexpr int kIB = 4;
-  const int nitems = R * kQuads;
+  const int nitems = (r1 - r0) * kQuads;
   for (int it0 = th; it0 < nitems; it0 += nth * kIB) {
     int rr[kIB], d1[kIB], hl[kIB], jj[kIB], bb[kIB];
     float y1[kIB][4], y2[kIB][4];
 #pragma unroll
     for (int i = 0; i < kIB; ++i) {
       const int it = it0 + i * nth;
-      rr[i] = it < nitems ? it / kQuads : 0;
+      rr[i] = it < nitems ? r0 + it / kQuads : 0;
       const int pp = (it % kQuads) * 4;
       hl[i] = pp / half;
       jj[i] = pp % half;
@@ -173,12 +186,12 @@ __device__ __noinline__ void reduce_tile(const Params &p, const int32_t *s_rseq,
 #pragma unroll
       for (int e = 0; e < 4; ++e) y1[i][e] = y2[i][e] = 0.f;
     }
-    for (int s0 = 0; s0 < nparts; s0 += 2) {
-      float4 a[kIB][2], c[kIB][2];
+    for (int s0 = 0; s0 < nparts; s0 += kPB) {
+      float4 a[kIB][kPB], c[kIB][kPB];
 #pragma unroll
       for (int i = 0; i < kIB; ++i)
 #pragma unroll
-        for (int s = 0; s < 2; ++s)
+        for (int s = 0; s < kPB; ++s)
           if (bb[i] >= 0 && s0 + s < nparts) {
             const float *ps = base + (s0 + s) * slot + rr[i] * kTileM + d1[i];
             a[i][s] = __ldcg(reinterpret_cast<const float4 *>(ps));
@@ -187,7 +200,7 @@ __device__ __noinline__ void reduce_tile(const Params &p, const int32_t *s_rseq,
 #pragma unroll
       for (int i = 0; i < kIB; ++i)
 #pragma unroll
-        for (int s = 0; s < 2; ++s)
+        for (int s = 0; s < kPB; ++s)
           if (bb[i] >= 0 && s0 + s < nparts) {
             y1[i][0] += a[i][s].x; y1[i][1] += a[i][s].y; y1[i][2] += a[i][s].z; y1[i][3] += a[i][s].w;
             y2[i][0] += c[i][s].x; y2[i][1] += c[i][s].y; y2[i][2] += c[i][s].z; y2[i][3] += c[i][s].w;
@@ -247,9 +260,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t *acc_empty = acc_full + 2;           // [2]
   uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + L.misc);
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L.misc + 8);
-  volatile int *s_last = reinterpret_cast<volatile int *>(smem + L.misc + 16);
   float *s_freq = reinterpret_cast<float *>(smem + L.freq);
-  volatile int *s_fin = reinterpret_cast<volatile int *>(smem + L.misc + 32);  // last tile, c_first, nparts
+  volatile int *s_last = reinterpret_cast<volatile int *>(smem + L.misc + 16);
+  volatile int *s_fin = reinterpret_cast<volatile int *>(smem + L.misc + 32);  // last tile, c_first, nparts; slab flag
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
@@ -299,18 +312,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t xbytes = p.Ncols * 128;  // x rows of one k-chunk
       bool expired = false;
       int issued = 0;
-      for (int u = u0, i = 0; u < u1; ++u, ++i) {
+      for (int u = u0, i = 0; u < u1; ++i) {
         const int st = i % p.stages;
         const uint32_t ph = (i / p.stages) & 1;
         if (!mbar_wait(&bar_empty[st], ph ^ 1, s_abort)) expired = true;
         if (*s_abort) break;
         issued = i + 1;
         uint8_t *stage = smem + L.ring + st * L.stage_bytes;
-        const int t = u / p.KS, c0 = (u - t * p.KS) * p.KG;
-        const int nch = min(p.KG, p.KC - c0);  // == KG whenever KG > 1 (H a multiple of 64 KG)
+        const int t = u / p.KC, c0 = u - t * p.KC;
+        const int nch = min(p.KG, min(u1, (t + 1) * p.KC) - u);  // chunks of one tile and this range
         mbar_arrive_expect_tx(&bar_full[st], nch * (kWBytes + xbytes));
-        if (p.KG > 1)
-          tma_load_3d(stage, &tm_w3, 0, t * kTileM, c0, &bar_full[st], pol_w);  // KG chunks, 16 KB apart
+        if (nch > 1)
+          tma_load_3d(stage, &tm_w3, 0, t * kTileM, c0, &bar_full[st], pol_w);  // nch chunks, 16 KB apart
         else
           tma_load_2d(stage, &tm_w, c0 * kKChunk, t * kTileM, &bar_full[st], pol_w);
         uint8_t *xs = stage + p.KG * kWBytes;
@@ -318,6 +331,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_2d(xs + j * xbytes, &tm_x0, (c0 + j) * kKChunk, 0, &bar_full[st], pol_x);
           if (n1) tma_load_2d(xs + j * xbytes + n0 * 128, &tm_x1, (c0 + j) * kKChunk, n0, &bar_full[st], pol_x);
         }
+        u += nch;
       }
       if (expired || *s_abort) {
         atomicOr(p.status, SPADE_DEV_TIMEOUT);
@@ -334,21 +348,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool expired = false;
       int i = 0, seg = 0;
       for (int u = u0; u < u1; ++seg) {
-        const int t = u / p.KS;
-        const int se = min(u1, (t + 1) * p.KS);
+        const int t = u / p.KC;
+        const int se = min(u1, (t + 1) * p.KC);
         const int buf = seg % p.nbuf, use = seg / p.nbuf;
         // The buffer's previous segment has been drained by the epilogue warps.
         if (use > 0 && !mbar_wait(&acc_empty[buf], (use - 1) & 1, s_abort)) expired = true;
         tc_fence_after();
         const uint32_t acc_addr = tmem + static_cast<uint32_t>(buf) * p.buf_cols;
-        for (const int us = u; u < se; ++u, ++i) {
+        for (const int us = u; u < se; ++i) {
           const int st = i % p.stages;
           const uint32_t ph = (i / p.stages) & 1;
+          const int nch = min(p.KG, se - u);  // as the producer cut the stage
           if (!mbar_wait(&bar_full[st], ph, s_abort)) expired = true;
           tc_fence_after();
           if (!*s_abort) {
             const uint32_t a0 = smem_base + L.ring + st * L.stage_bytes;
-            const int nch = min(p.KG, p.KC - (u - t * p.KS) * p.KG);
             for (int j = 0; j < nch; ++j) {
               const uint32_t a = a0 + j * kWBytes;
               const uint32_t b = a0 + p.KG * kWBytes + j * p.Ncols * 128;
@@ -363,6 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           tc_commit(&bar_empty[st]);
+          u += nch;
         }
         tc_commit(&acc_full[buf]);
       }
@@ -403,8 +418,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool expired = false;
     int seg = 0;
     for (int u = u0; u < u1; ++seg) {
-      const int t = u / p.KS;
-      const int se = min(u1, (t + 1) * p.KS);
+      const int t = u / p.KC;
+      const int se = min(u1, (t + 1) * p.KC);
       const int buf = seg % p.nbuf, use = seg / p.nbuf;
       if (!mbar_wait(&acc_full[buf], use & 1, s_abort)) expired = true;
       tc_fence_after();
@@ -421,32 +436,81 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty[buf]);
-      // Publish; the CTA that completes the tile reduces it.
-      const int c_first = unit_owner(p.units, p.num_ctas, t * p.KS);
-      const int c_last = unit_owner(p.units, p.num_ctas, (t + 1) * p.KS - 1);
-      const int nparts = c_last - c_first + 1;
+      // Publish the part.  With slabs, a split tile is finished after the
+      // stream; otherwise the CTA whose part completes the tile (every
+      // CTA of a whole tile) finishes it here, or, for the CTA's last tile,
+      // below with every thread of the CTA.
+      const int c_first = unit_owner(p.units, p.num_ctas, t * p.KC);
+      const int nparts = unit_owner(p.units, p.num_ctas, (t + 1) * p.KC - 1) - c_first + 1;
       epi_bar();
-      if (et == 0) *s_last = nparts == 1 ? 1 : arrive_tile(&p.counters[t], nparts);
-      epi_bar();
-      if (*s_last) {
-        if (se == u1) {
-          // The CTA's last tile: reduced below by every thread of the CTA.
-          if (et == 0) { s_fin[0] = t; s_fin[1] = c_first; s_fin[2] = nparts; }
-        } else {
-          reduce_tile(p, s_rseq, s_rpos, s_freq, t, c_first, nparts, et, kEpiThreads);
-          if (et == 0 && nparts > 1) p.counters[t] = 0;  // every part has arrived: reset for the next call
+      if (nparts > 1 && p.slabs > 1) {
+        if (et == 0) publish_part(&p.counters[t]);
+      } else {
+        // Release publishes this part; for the last one, acquire makes the others visible.
+        if (et == 0) *s_last = nparts == 1 || add_acq_rel(&p.counters[t], 1) == nparts - 1;
+        epi_bar();
+        if (*s_last) {
+          if (se == u1) {
+            if (et == 0) { s_fin[0] = t; s_fin[1] = c_first; s_fin[2] = nparts; }
+          } else {
+            if (nparts == 1)
+              reduce_tile<6, 1>(p, s_rseq, s_rpos, s_freq, t, c_first, 1, 0, p.R, et, kEpiThreads);
+            else
+              reduce_tile<3, 3>(p, s_rseq, s_rpos, s_freq, t, c_first, nparts, 0, p.R, et, kEpiThreads);
+            if (et == 0 && nparts > 1) p.counters[t] = 0;  // every part has arrived: reset for the next call
+          }
         }
       }
       u = se;
     }
     if (expired) atomicOr(p.status, SPADE_DEV_TIMEOUT);
   }
-  // The CTA's last tile, if this CTA completed it, with every thread.
+  // The CTA's last tile, if this CTA finishes it, with every thread.
   __syncwarp();
   __syncthreads();
   if (s_fin[0] >= 0) {
-    reduce_tile(p, s_rseq, s_rpos, s_freq, s_fin[0], s_fin[1], s_fin[2], tid, kThreads);
-    if (tid == 0 && s_fin[2] > 1) p.counters[s_fin[0]] = 0;  // every part has arrived: reset for the next call
+    const int t = s_fin[0], c_first = s_fin[1], nparts = s_fin[2];
+    if (nparts == 1)
+      reduce_tile<6, 1>(p, s_rseq, s_rpos, s_freq, t, c_first, 1, 0, p.R, tid, kThreads);
+    else
+      reduce_tile<3, 3>(p, s_rseq, s_rpos, s_freq, t, c_first, nparts, 0, p.R, tid, kThreads);
+    if (tid == 0 && nparts > 1) p.counters[t] = 0;  // every part has arrived: reset for the next call
+  }
+  // Row slabs of the split tiles (slabs > 1): item i = t * slabs + s goes to
+  // CTA i mod num_ctas.  The slab waits until all of the tile's parts are
+  // published (acquire, bounded), and the tile's last slab to finish resets
+  // both counters for the next call.
+  int32_t *published = p.counters, *slabs_done = p.counters + p.tiles;
+  for (int item = blockIdx.x; p.slabs > 1 && item < p.tiles * p.slabs; item += p.num_ctas) {
+    const int t = item / p.slabs, sl = item - t * p.slabs;
+    const int c_first = unit_owner(p.units, p.num_ctas, t * p.KC);
+    const int nparts = unit_owner(p.units, p.num_ctas, (t + 1) * p.KC - 1) - c_first + 1;
+    if (nparts == 1) continue;  // a whole tile: finished by its CTA
+    if (tid == 0) {
+      s_fin[3] = 1;
+      if (load_acquire(&published[t]) != nparts) {
+        const uint64_t t0 = globaltimer();
+        while (load_acquire(&published[t]) != nparts) {
+          if (globaltimer() - t0 > kWaitLimitNs) {
+            atomicOr(p.status, SPADE_DEV_TIMEOUT);
+            s_fin[3] = 0;
+            break;
+          }
+        }
+      }
+    }
+    __syncthreads();
+    const int ok = s_fin[3];
+    if (ok) {
+      const int r0 = static_cast<int>(static_cast<int64_t>(p.R) * sl / p.slabs);
+      const int r1 = static_cast<int>(static_cast<int64_t>(p.R) * (sl + 1) / p.slabs);
+      reduce_tile<2, 6>(p, s_rseq, s_rpos, s_freq, t, c_first, nparts, r0, r1, tid, kThreads);
+    }
+    __syncthreads();  // every load of the parts is done
+    if (tid == 0 && ok && add_acq_rel(&slabs_done[t], 1) == p.slabs - 1) {
+      published[t] = 0;
+      slabs_done[t] = 0;
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -465,9 +529,10 @@ struct Paging {
   const int32_t *block_table;
   int page_size, max_pages, num_pages;
 };
+static size_t counter_bytes(int tiles) { return round_up(static_cast<size_t>(tiles) * 8, 256); }
 static size_t workspace_bytes_for(int R, int tiles, int sms) {
   const size_t ncols = static_cast<size_t>((R + 15) / 16 * 16);
-  return round_up(static_cast<size_t>(tiles) * 4, 256) + static_cast<size_t>(sms + tiles) * ncols * kTileM * 4;
+  return counter_bytes(tiles) + static_cast<size_t>(sms + tiles) * ncols * kTileM * 4;
 }
 }  // namespace qkv
 }  // namespace spade
@@ -523,7 +588,7 @@ static spade_status qkv_rope_impl(const void *x, const void *w_qkv, const int32_
   p.v_cache = static_cast<__nv_bfloat16 *>(v_cache);
   p.status = status;
   p.counters = static_cast<int32_t *>(workspace);
-  p.partials = reinterpret_cast<float *>(static_cast<uint8_t *>(workspace) + round_up(static_cast<size_t>(tiles) * 4, 256));
+  p.partials = reinterpret_cast<float *>(static_cast<uint8_t *>(workspace) + counter_bytes(tiles));
   p.B = B; p.R = R; p.H = H; p.Hq = Hq; p.Hkv = Hkv; p.D = D; p.cap = cap; p.max_k = max_k;
   p.block_table = pg ? pg->block_table : nullptr;
   p.page_size = pg ? pg->page_size : 0;
@@ -537,15 +602,18 @@ static spade_status qkv_rope_impl(const void *x, const void *w_qkv, const int32_
   p.nbuf = p.buf_cols * 2 <= 512 ? 2 : 1;
   p.tmem_cols = p.buf_cols * p.nbuf;
   for (int j = 0; j < D / 2; ++j) p.inv_freq[j] = static_cast<float>(pow(static_cast<double>(rope_theta), -2.0 * j / D));
-  // Two k-chunks per unit when H allows the 3-D view and the ring still
-  // holds three stages; otherwise one.
+  // Stages of up to two k-chunks when H allows the 3-D view and the ring
+  // still holds three of them; otherwise one chunk per stage.
   p.KG = 1;
-  if (H % (2 * kKChunk) == 0 &&
-      (kSmemBudget - layout(p.Ncols, 0, 2).total) / layout(p.Ncols, 0, 2).stage_bytes >= 3)
+  if (H % kKChunk == 0 && (kSmemBudget - layout(p.Ncols, 0, 2).total) / layout(p.Ncols, 0, 2).stage_bytes >= 3)
     p.KG = 2;
-  p.KS = (p.KC + p.KG - 1) / p.KG;
-  p.units = tiles * p.KS;
+  p.units = tiles * p.KC;
   p.num_ctas = p.units < sms ? p.units : sms;
+  // Slabs: as many as keep every CTA busy in the final reduction, of at
+  // least 8 rows each (one: split tiles are finished by their last part's CTA).
+  p.slabs = p.num_ctas / tiles;
+  if (p.slabs > R / 8) p.slabs = R / 8;
+  if (p.slabs < 1) p.slabs = 1;
   p.stages = (kSmemBudget - layout(p.Ncols, 0, p.KG).total) / layout(p.Ncols, 0, p.KG).stage_bytes;
   if (p.stages > kMaxStages) p.stages = kMaxStages;
   if (p.stages < 2) return fail(SPADE_ERR_SHAPE, "shared memory too small for R = %d", R);
@@ -576,11 +644,15 @@ static spade_status qkv_rope_impl(const void *x, const void *w_qkv, const int32_
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = reinterpret_cast<cudaStream_t>(stream);
-  cudaLaunchAttribute attr[1];
+  // Cooperative: the final reduction's slabs wait for other CTAs' partials,
+  // so every CTA must be resident (one per SM at most).
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeCooperative;
+  attr[1].val.cooperative = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   const cudaError_t e = cudaLaunchKernelEx(&cfg, qkv_rope_kernel, p, tw, tx0, tx1, tw3);
   if (e != cudaSuccess) return cuda_fail(e, "qkv_rope launch");
   return SPADE_OK;
