@@ -89,10 +89,13 @@ def _job_rate(tokens_local, t_local, ws, device):
     return tokens_local / t_local, t_local
 
 
-def _head_start(ms=3.0):
-    """Queues a spin kernel of about `ms` milliseconds so that the host can enqueue the
-    timed launches ahead of the GPU: a timed region must not contain GPU idle time spent
-    waiting for Python to issue the next launch."""
+def _head_start(iterations):
+    """Queues a spin kernel so that the host can enqueue the timed launches ahead of the
+    GPU: a timed region must not contain GPU idle time spent waiting for Python to issue
+    the next launch.  It gives the host 0.5 ms per loop iteration (at least 3 ms), far
+    above what an iteration takes (tens of microseconds), so a slow or busy host cannot
+    leak into a kernel's time."""
+    ms = max(3.0, 0.5 * iterations)
     torch.cuda._sleep(int(ms * 2.0e6))  # cycles at about 2 GHz
 
 
@@ -281,7 +284,7 @@ def run_spade(args, ws, rank, local):
     torch.cuda.synchronize()
     with Clocks(local) as clk:
         t_wall0 = time.perf_counter()
-        _head_start(3.0)
+        _head_start(args.steps)
         for s in range(args.steps):
             wl["ctx_lens"].copy_(ctx0)
             if flush:
@@ -401,7 +404,7 @@ def run_spade(args, ws, rank, local):
         acc_g = torch.zeros_like(acc)
         tok_g = torch.zeros_like(tok)
         ev1 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
-        _head_start(3.0)
+        _head_start(13)
         for i in range(13):
             if flush:
                 flush_buf.zero_()
@@ -492,7 +495,7 @@ def _time_qkv(spec, wl, dev, flush_buf=None, launches=20):
     call()
     torch.cuda.synchronize()
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(launches)]
-    _head_start(3.0)
+    _head_start(launches + 3)
     for i in range(launches + 3):
         flush_buf.zero_()
         if i >= 3:
@@ -538,7 +541,7 @@ def _time_step(wl, dev, steps, warmup):
             # The first step of a shape runs one-time host work; the timed steps must not
             # wait on the host, so the GPU gets a head start after it.
             torch.cuda.synchronize()
-            _head_start(3.0)
+            _head_start(warmup + steps)
         wl["ctx_lens"].copy_(ctx0)
         if flush:
             flush_buf.zero_()
@@ -611,7 +614,7 @@ def sampling_report(wl, dev, launches=20):
         for i in range(3 + launches):
             if i == 1:
                 torch.cuda.synchronize()
-                _head_start(2.0)
+                _head_start(3 + launches)
             if flush_buf is not None:
                 flush_buf.zero_()
             e = evs[i - 3] if i >= 3 else None

@@ -4,6 +4,8 @@ Small cases span several key chunks, vocabulary tiles and ragged tails and are
 checked element by element; the benchmark workloads are checked at full size
 (attention on sampled (row, head) pairs, accept decisions on every sequence).
 """
+import time
+
 import numpy as np
 import pytest
 import torch
@@ -456,6 +458,65 @@ def test_qkv_rope_skips_invalid_sequences(dev):
     wl["ctx_lens"][1] = 0  # a harmless stand-in position for the oracle call; its rows are skipped
     parity.check_qkv_rope(wl, x, w, q, k0, v0, skip=(1,))
     wl["ctx_lens"].copy_(ctx)
+
+
+def _qkv_call(wl, x, w, q, ws, st):
+    spade.spade_verify_qkv_rope(x, w, wl["ctx_lens"], wl["n_draft"], wl["cu_q"], q, wl["k_cache"], wl["v_cache"],
+                                Hq=wl["Hq"], Hkv=wl["Hkv"], rope_theta=wl["spec"].rope_theta,
+                                max_k=int(wl["n_draft"].max()), workspace=ws, status=st)
+
+
+@pytest.mark.parametrize("name", ["qkv_many_rows", "llama3_8b", "long_70b"])
+def test_qkv_rope_repeated_calls_share_a_workspace(dev, name):
+    """Calls that share one workspace give the same q, K and V bit for bit, so every call
+    leaves its counters zeroed: split tiles finished in row slabs over the grid (the small
+    shape and Llama-3-8B have two or more CTAs per tile) and split tiles finished by the CTA
+    whose part completes them (the 70B shape has fewer than two)."""
+    spec = QKV_SMALL[name] if name in QKV_SMALL else W.SPECS[name]
+    wl = W.make_workload(spec, device=dev)
+    x, w = W.make_qkv_inputs(spec, wl["R"], device=dev)
+    ws = spade.qkv_workspace(wl["R"], wl["Hq"], wl["Hkv"], wl["D"], device=dev)
+    st = spade.status_tensor(dev)
+    outs = []
+    for _ in range(3):
+        q = torch.full((wl["R"], wl["Hq"], wl["D"]), float("nan"), dtype=torch.bfloat16, device=dev)
+        _qkv_call(wl, x, w, q, ws, st)
+        torch.cuda.synchronize()
+        assert int(st.item()) == 0
+        outs.append((q, wl["k_cache"].clone(), wl["v_cache"].clone()))
+        assert int(ws[:4 * 2 * ((wl["Hq"] + 2 * wl["Hkv"]) * wl["D"] // 128)].view(torch.int32).abs().sum()) == 0
+    for q, k, v in outs[1:]:
+        assert torch.equal(q, outs[0][0]) and torch.equal(k, outs[0][1]) and torch.equal(v, outs[0][2])
+    assert not torch.isnan(outs[0][0].float()).any()
+
+
+def test_qkv_rope_split_tile_wait_is_bounded(dev):
+    """A workspace whose counter of a split tile was left dirty (as after an interrupted call)
+    makes that tile's row slabs wait for a part count that never comes: each wait gives up
+    after its limit, the call reports SPADE_DEV_TIMEOUT, and the GPU stays usable (a clean
+    call right after matches the oracle)."""
+    spec = QKV_SMALL["qkv_many_rows"]
+    wl = W.make_workload(spec, device=dev)
+    x, w = W.make_qkv_inputs(spec, wl["R"], device=dev)
+    k0, v0 = wl["k_cache"].clone(), wl["v_cache"].clone()
+    ws = spade.qkv_workspace(wl["R"], wl["Hq"], wl["Hkv"], wl["D"], device=dev)
+    ws[:4].view(torch.int32).fill_(1000)  # parts published for tile 0: never equal to its part count
+    st = spade.status_tensor(dev)
+    q = torch.full((wl["R"], wl["Hq"], wl["D"]), float("nan"), dtype=torch.bfloat16, device=dev)
+    t0 = time.perf_counter()
+    _qkv_call(wl, x, w, q, ws, st)
+    torch.cuda.synchronize()
+    assert time.perf_counter() - t0 < 30
+    assert int(st.item()) & spade.DEV_TIMEOUT
+    ws.zero_()
+    st.zero_()
+    wl["k_cache"].copy_(k0)
+    wl["v_cache"].copy_(v0)
+    q = torch.full((wl["R"], wl["Hq"], wl["D"]), float("nan"), dtype=torch.bfloat16, device=dev)
+    _qkv_call(wl, x, w, q, ws, st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    parity.check_qkv_rope(wl, x, w, q, k0, v0)
 
 
 def test_qkv_then_attention_matches_oracle_chain(dev):
