@@ -59,6 +59,7 @@ constexpr int kMaxRounds = 32;
 // already taken.
 constexpr int kResident = 0, kStatsOnly = 1, kPresampled = 2;
 constexpr int kMaxTilesPerCta = 32;
+constexpr int kMaxPairSlots = 16;  // W-ring slots of the short last tile's own round
 constexpr int kMaxNC = 256;  // CTAs (vocabulary slices) per launch
 
 // Residual masses through shared memory (phase C): groups of kFG sampled rows
@@ -148,7 +149,7 @@ __host__ __device__ inline Smem smem_layout(const Params &p) {
   s.off_bar = s.off_h + p.HS * s.h_slot;
   // 128-byte aligned: the float4 statistics in the transpose region below
   // inherit this alignment.
-  s.off_misc = (s.off_bar + (2 * p.WS + 2 * p.HS + 3) * 8 + 127) & ~127;
+  s.off_misc = (s.off_bar + (2 * p.WS + 2 * p.HS + 3 + 2 * kMaxPairSlots) * 8 + 127) & ~127;
   s.off_rows = s.off_misc + 64;  // int/float [5][kMaxR] + int [3][kMaxB + 1]
   // Per epilogue warp a 32 x 33 float transpose buffer.  After the last round
   // the warps' per-row statistics (float4 [kEpiWarps][R], at most 32 KB) go to
@@ -391,6 +392,8 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   uint64_t *acc_full = h_empty + p.HS;
   uint64_t *acc_empty = acc_full + 1;
   uint64_t *fin = acc_empty + 1;  // pair mode: teardown handshake
+  uint64_t *pp_full = fin + 1;    // [kMaxPairSlots]: the short tile's round, see comb_ok
+  uint64_t *pp_empty = pp_full + kMaxPairSlots;
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L.off_misc);
   uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + L.off_misc + 8);
   int *s_any_stoch = reinterpret_cast<int *>(smem + L.off_misc + 16);
@@ -433,6 +436,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
     mbar_init(acc_full, 1);
     mbar_init(acc_empty, PAIR ? 2 * kEpiWarps : kEpiWarps);  // pair: both CTAs' epilogues
     mbar_init(fin, 1);
+    for (int j = 0; j < kMaxPairSlots; ++j) { mbar_init(&pp_full[j], 1); mbar_init(&pp_empty[j], 1); }
     if (PAIR && rank == 0) {
       // Pair mode: arm every slot's first use with both CTAs' bytes.
       for (int s = 0; s < p.WS; ++s) mbar_arrive_expect_tx(&w_full[s], 2 * kWChunkBytes);
@@ -483,12 +487,19 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   // stage c mod NS, so at any moment about NC / NS CTAs (not all of them) load
   // the same hidden lines from L2.  Each logit's sum over K changes order only.
   const int k_rot = sl % p.NS;  // a pair walks its stages in one order
-  // A round that holds only the short last tile streams one k-chunk per stage
-  // with its W rows and hidden rows together in one slot of either ring, so all
-  // 4 + 3 slots are in flight (a two-ring stage keeps at most HS = 3 in flight,
-  // and its W slots would be 60 % empty).  Needs both boxes to fit an H slot.
+  // A round that holds only the short last tile streams one k-chunk per slot,
+  // its W rows and hidden rows together, through the H ring's slots and through
+  // npw slots of that size carved anew from the W ring (own barriers; each one
+  // first written once round 1 has released the W slots it overlaps): at
+  // Llama-3-8B sizes 6 + 3 = 9 k-chunks in flight.  The round is bound by its
+  // loads' latency: one slot per chunk keeps each slot's release right after
+  // its own MMAs (chunks spread over fewer, larger slots measured slower), and a
+  // two-ring stage would keep at most HS = 3 in flight.  Needs both boxes to fit
+  // an H slot.
   const bool comb_ok = p.kind != kStatsOnly && short_last && p.nchunks == 1 && p.h_boxes == 1 &&
                        (p.BRS + p.h_box_rows) * 128 <= L.h_slot;
+  const int comb_pb = (p.BRS + p.h_box_rows) * 128;  // one k-chunk's W rows and hidden rows
+  const int comb_npw = min(kMaxPairSlots, p.WS * L.w_slot / comb_pb);
 
   // ======================= phase A: logits + slice statistics =============
   if (warp == 0) {
@@ -550,6 +561,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
       const uint64_t pol_w = l2_policy_evict_first();
       const uint64_t pol_h = l2_policy_evict_last();
       uint32_t wi = 0, hi = 0, w_issued = 0, h_issued = 0;
+      int comb_issued = 0;  // chunks of the short tile's round issued (carved slots' uses follow from it)
       // Ring slots and parities advance by counters (no per-stage divisions).
       int ws_ = 0, hs_ = 0;
       uint32_t wph_ = 0, hph_ = 0;
@@ -559,26 +571,39 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         if (comb_ok && nt == 1 && tdone == ntiles - 1) {
           const int row0 = v_lo + tdone * kTileV;
           const int kr = c % p.KC;
+          // The slots in turn: npw carved from the W ring, then the H slots;
+          // slot index and pass (parity) advance by counters.
+          int si = 0, use = 0;
           for (int it = 0; it < p.KC; ++it) {
             const int kc = it + kr < p.KC ? it + kr : it + kr - p.KC;
-            const bool use_w = it % 7 < 4;  // four W slots, then three H slots
-            const int s = use_w ? ws_ : hs_;
-            uint64_t *full = use_w ? &w_full[s] : &h_full[s];
-            mbar_wait(use_w ? &w_empty[s] : &h_empty[s], (use_w ? wph_ : hph_) ^ 1, s_abort);
+            const bool carved = si < comb_npw;
+            uint8_t *dst;
+            uint64_t *full;
+            if (carved) {
+              if (use == 0) {
+                // Round 1's last use of every W slot this one overlaps is released.
+                for (int s = si * comb_pb / L.w_slot; s <= ((si + 1) * comb_pb - 1) / L.w_slot; ++s)
+                  mbar_wait(&w_empty[s], (s >= ws_ ? wph_ : wph_ ^ 1u) ^ 1u, s_abort);
+              }
+              mbar_wait(&pp_empty[si], (use & 1) ^ 1, s_abort);
+              dst = w_ring + si * comb_pb;
+              full = &pp_full[si];
+            } else {
+              mbar_wait(&h_empty[hs_], hph_ ^ 1, s_abort);
+              dst = h_ring + hs_ * L.h_slot;
+              full = &h_full[hs_];
+            }
             if (!*s_abort) {
-              uint8_t *dst = use_w ? w_ring + s * L.w_slot : h_ring + s * L.h_slot;
-              mbar_arrive_expect_tx(full, (p.BRS + p.h_box_rows) * 128);
+              mbar_arrive_expect_tx(full, comb_pb);
               tma_load_2d(dst, &tm_w2s, kc * kKChunk, row0, full, pol_w);
               tma_load_2d(dst + p.BRS * 128, &tm_h2, kc * kKChunk, 0, full, pol_h);
-              if (use_w) w_issued = wi + 1; else h_issued = hi + 1;
+              if (carved) comb_issued = it + 1; else h_issued = hi + 1;
             }
-            if (use_w) {
-              ++wi;
-              if (++ws_ == p.WS) { ws_ = 0; wph_ ^= 1u; }
-            } else {
+            if (!carved) {
               ++hi;
               if (++hs_ == p.HS) { hs_ = 0; hph_ ^= 1u; }
             }
+            if (++si == comb_npw + p.HS) { si = 0; ++use; }
           }
           tdone += nt;
           continue;
@@ -648,6 +673,11 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
           mbar_wait_unabortable(&w_full[j % p.WS], (j / p.WS) & 1);
         for (uint32_t j = (h_issued > (uint32_t)p.HS ? h_issued - p.HS : 0); j < h_issued; ++j)
           mbar_wait_unabortable(&h_full[j % p.HS], (j / p.HS) & 1);
+        // Carved slot j was filled once for every issued chunk it = j (mod the cycle).
+        for (int j = 0; j < comb_npw && j < comb_issued; ++j) {
+          const int fills = (comb_issued - 1 - j) / (comb_npw + p.HS) + 1;
+          mbar_wait_unabortable(&pp_full[j], (fills - 1) & 1);
+        }
       }
     }
   } else if (warp == 1) {
@@ -705,23 +735,36 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
         if (r > 0) mbar_wait(acc_empty, (r - 1) & 1, s_abort);
         tc_fence_after();
         if (comb_ok && nt == 1 && tdone == ntiles - 1) {
+          // Slot index and pass by counters, and each chunk's two operand
+          // descriptors built once (a K step of 16 adds 32 bytes, 2 in the
+          // descriptor's address field): the loop issues as few instructions
+          // per MMA as it can.
           const uint32_t d_tmem = tmem + static_cast<uint32_t>(used);
+          const uint32_t idesc = p.idesc, boff = static_cast<uint32_t>(p.BRS) * 128u;
+          const uint32_t carved0 = smem_u32(w_ring), h0 = smem_u32(h_ring);
+          int si = 0;
+          uint32_t cph = 0;
           for (int it = 0; it < p.KC; ++it) {
-            const bool use_w = it % 7 < 4;
-            const int s = use_w ? ws_ : hs_;
-            mbar_wait(use_w ? &w_full[s] : &h_full[s], use_w ? wph_ : hph_, s_abort);
-            tc_fence_after();
-            const uint32_t base = smem_u32(use_w ? w_ring + s * L.w_slot : h_ring + s * L.h_slot);
-#pragma unroll
-            for (int k16 = 0; k16 < kKChunk / 16; ++k16)
-              tc_mma_f16(d_tmem, smem_desc_sw128(base + 32 * k16), smem_desc_sw128(base + p.BRS * 128 + 32 * k16),
-                         p.idesc, (it | k16) != 0);
-            tc_commit(use_w ? &w_empty[s] : &h_empty[s]);
-            if (use_w) {
-              if (++ws_ == p.WS) { ws_ = 0; wph_ ^= 1u; }
+            const bool carved = si < comb_npw;
+            uint32_t base;
+            uint64_t *empty;
+            if (carved) {
+              mbar_wait(&pp_full[si], cph, s_abort);
+              base = carved0 + static_cast<uint32_t>(si * comb_pb);
+              empty = &pp_empty[si];
             } else {
+              mbar_wait(&h_full[hs_], hph_, s_abort);
+              base = h0 + static_cast<uint32_t>(hs_ * L.h_slot);
+              empty = &h_empty[hs_];
               if (++hs_ == p.HS) { hs_ = 0; hph_ ^= 1u; }
             }
+            if (++si == comb_npw + p.HS) { si = 0; cph ^= 1u; }
+            tc_fence_after();
+            const uint64_t da = smem_desc_sw128(base), db = smem_desc_sw128(base + boff);
+#pragma unroll
+            for (int k16 = 0; k16 < kKChunk / 16; ++k16)
+              tc_mma_f16(d_tmem, da + 2u * k16, db + 2u * k16, idesc, (it | k16) != 0);
+            tc_commit(empty);
           }
           tc_commit(acc_full);
           ++rounds_issued;
