@@ -792,14 +792,16 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
             const int hk = p.h_boxes * p.h_box_rows * 128;
             for (int jj = 0; jj < nch; ++jj) {
               for (int ci = 0; ci < p.nchunks; ++ci) {
-                // N-chunk ci: TMEM columns and hidden rows from noff on.
+                // N-chunk ci: TMEM columns and hidden rows from noff on.  Each
+                // operand's descriptor is built once per k-chunk; a K step of
+                // 16 adds 32 bytes, 2 in the descriptor's address field.
                 const uint32_t noff = ci ? static_cast<uint32_t>(p.n0w) : 0u;
+                const uint64_t da = smem_desc_sw128(w_addr + jj * w_chunk);
+                const uint64_t db = smem_desc_sw128(h_addr + jj * hk + noff * 128);
+                const uint32_t idesc = ci ? p.idesc1 : p.idesc;
 #pragma unroll
-                for (int k16 = 0; k16 < kKChunk / 16; ++k16) {
-                  tc_mma_f16(d_tmem + noff, smem_desc_sw128(w_addr + jj * w_chunk + 32 * k16),
-                             smem_desc_sw128(h_addr + jj * hk + noff * 128 + 32 * k16),
-                             ci ? p.idesc1 : p.idesc, (it | jj | k16) != 0);
-                }
+                for (int k16 = 0; k16 < kKChunk / 16; ++k16)
+                  tc_mma_f16(d_tmem + noff, da + 2u * k16, db + 2u * k16, idesc, (it | jj | k16) != 0);
               }
             }
             tc_commit(&w_empty[ws]);
