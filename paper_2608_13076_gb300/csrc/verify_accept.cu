@@ -491,11 +491,12 @@ __global__ void __launch_bounds__(kThreads, 1) verify_accept_kernel(
   // its W rows and hidden rows together, through the H ring's slots and through
   // npw slots of that size carved anew from the W ring (own barriers; each one
   // first written once round 1 has released the W slots it overlaps): at
-  // Llama-3-8B sizes 6 + 3 = 9 k-chunks in flight.  The round is bound by its
-  // loads' latency: one slot per chunk keeps each slot's release right after
-  // its own MMAs (chunks spread over fewer, larger slots measured slower), and a
-  // two-ring stage would keep at most HS = 3 in flight.  Needs both boxes to fit
-  // an H slot.
+  // Llama-3-8B sizes 6 + 3 = 9 k-chunks in flight.  That round is bound by the
+  // slots' round trip (MMAs done, slot released, refilled, MMA thread woken) and
+  // by the MMA thread's issue rate, not by its bytes, so it takes as many slots
+  // as fit and keeps each to one chunk, released right after its own MMAs
+  // (chunks spread over fewer, larger slots measured slower); a two-ring stage
+  // would keep at most HS = 3 in flight.  Needs both boxes to fit an H slot.
   const bool comb_ok = p.kind != kStatsOnly && short_last && p.nchunks == 1 && p.h_boxes == 1 &&
                        (p.BRS + p.h_box_rows) * 128 <= L.h_slot;
   const int comb_pb = (p.BRS + p.h_box_rows) * 128;  // one k-chunk's W rows and hidden rows
